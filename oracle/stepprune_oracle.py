@@ -1,0 +1,478 @@
+"""StepPrune inference path -- CPU oracle (TEST INFRASTRUCTURE ONLY).
+
+A plain, slow, fp64 restatement of what the inference path of StepPrune
+(arXiv 2609.13804) computes, written from the paper:
+
+  * text projection and cross-modal input encoder      (Sec. 3.2, Eq. 3)
+  * candidate memory with the learned STOP row          (Sec. 3.2, "Learned STOP Action")
+  * pointer decoder, one hard step per round            (Sec. 3.2, Eq. 4)
+  * grouped execution, TopG per non-STOP round          (Sec. 3.5, Eq. 11)
+  * Algorithm 1: loop, restore to native order, gather  (Algorithm 1; Sec. 3.3, last paragraph)
+  * frozen projector and LM prefill over the packed prefix (Sec. 3.3-3.4; LM dims of the
+    evaluated backbones, Sec. 4.1)
+
+Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline leg may import
+this module.  It shares no code with the CUDA library and imports nothing from
+the package; inputs arrive as numpy arrays from the seeded generators.
+
+Readings of points the paper leaves open are stated at each function (see the
+'Reading' notes); the list is repeated in the design notes of the repository.
+
+Parity status of each function:
+  layer_norm, rms_norm, gelu, silu      pinned (torch.nn.functional, closed forms)
+  attention                             pinned (torch scaled_dot_product_attention, brute force)
+  text_projection, encoder              pinned (torch.nn.TransformerEncoderLayer, fp64)
+  pointer logits / select_episode       pinned (brute-force from-scratch decoder; torch
+                                        nn.MultiheadAttention decoder; history-free top-K
+                                        special case, Eq. 1; invariants of Alg. 1 and Eq. 11)
+  restore / compact                     pinned (hand-worked golden fixture; invariants)
+  rope                                  pinned (rotation closed form, relative-position property)
+  projector, prefill_layer, prefill     pinned through their parts plus special cases
+                                        (zero output weights -> identity; uniform attention);
+                                        the composition of a whole random-weight LM is
+                                        parity unpinned beyond those checks.
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Optional, Sequence
+
+import numpy as np
+from scipy.special import erf as _erf
+
+F64 = np.float64
+NEG_INF = -np.inf
+
+
+def _f(x) -> np.ndarray:
+    return np.asarray(x, dtype=F64)
+
+
+# ----------------------------------------------------------------------------
+# elementary layers
+# ----------------------------------------------------------------------------
+
+def layer_norm(x, eps: float, gain=None, bias=None) -> np.ndarray:
+    """LayerNorm over the last axis, biased variance: (x - mu) / sqrt(var + eps) * g + b."""
+    x = _f(x)
+    mu = x.mean(axis=-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=-1, keepdims=True)
+    y = (x - mu) / np.sqrt(var + eps)
+    if gain is not None:
+        y = y * _f(gain)
+    if bias is not None:
+        y = y + _f(bias)
+    return y
+
+
+def rms_norm(x, eps: float, gain=None) -> np.ndarray:
+    """RMSNorm over the last axis: x / sqrt(mean(x^2) + eps) * g."""
+    x = _f(x)
+    y = x / np.sqrt((x * x).mean(axis=-1, keepdims=True) + eps)
+    if gain is not None:
+        y = y * _f(gain)
+    return y
+
+
+def gelu(x) -> np.ndarray:
+    """Exact GELU, x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2))."""
+    x = _f(x)
+    return 0.5 * x * (1.0 + _erf(x / math.sqrt(2.0)))
+
+
+def silu(x) -> np.ndarray:
+    x = _f(x)
+    return x / (1.0 + np.exp(-x))
+
+
+def softmax(x, axis: int = -1) -> np.ndarray:
+    x = _f(x)
+    m = np.max(x, axis=axis, keepdims=True)
+    e = np.exp(x - m)
+    return e / e.sum(axis=axis, keepdims=True)
+
+
+def attention(q, k, v, n_heads: int, n_kv_heads: int, causal: bool) -> np.ndarray:
+    """Scaled dot-product attention of one sequence.
+
+    q [L, Hq*dh], k/v [L, Hkv*dh].  Query head i reads key/value head
+    floor(i * Hkv / Hq) (grouped-query attention; Hkv == Hq is plain MHA).
+    Causal: position p attends to positions 0..p.
+    """
+    q, k, v = _f(q), _f(k), _f(v)
+    L = q.shape[0]
+    dh = q.shape[1] // n_heads
+    out = np.zeros((L, n_heads * dh), dtype=F64)
+    mask = np.zeros((L, L), dtype=F64)
+    if causal:
+        mask[np.triu_indices(L, 1)] = NEG_INF
+    for i in range(n_heads):
+        j = (i * n_kv_heads) // n_heads
+        qi = q[:, i * dh:(i + 1) * dh]
+        kj = k[:, j * dh:(j + 1) * dh]
+        vj = v[:, j * dh:(j + 1) * dh]
+        s = qi @ kj.T / math.sqrt(dh) + mask
+        out[:, i * dh:(i + 1) * dh] = softmax(s, axis=-1) @ vj
+    return out
+
+
+# ----------------------------------------------------------------------------
+# selector: text projection and cross-modal encoder (Sec. 3.2, Eq. 3)
+# ----------------------------------------------------------------------------
+
+def text_projection(E_text, sel: Dict, eps: float, g_text: float = 1.0) -> np.ndarray:
+    """E~_text = g_text * LN(W_p E_text) (Sec. 3.2).  Rows of E_text are tokens.
+
+    Reading: g_text = 1 at inference (it is only ramped during training).
+    """
+    P = _f(E_text) @ _f(sel["W_p"]).T
+    return g_text * layer_norm(P, eps, sel.get("ln_text_g"), sel.get("ln_text_b"))
+
+
+def encoder_block(x, L: Dict, n_heads: int, eps: float) -> np.ndarray:
+    """One pre-norm ViT block with bidirectional self-attention (Sec. 3.2; the
+    bidirectional mask is the default of Table 7(a)).
+
+    Reading: no linear biases; MLP is W2 GELU(W1 x) with exact GELU.
+    """
+    x = _f(x)
+    D = x.shape[1]
+    a = layer_norm(x, eps, L.get("ln1_g"), L.get("ln1_b"))
+    qkv = a @ _f(L["Wqkv"]).T
+    o = attention(qkv[:, :D], qkv[:, D:2 * D], qkv[:, 2 * D:], n_heads, n_heads, causal=False)
+    x = x + o @ _f(L["Wo"]).T
+    m = layer_norm(x, eps, L.get("ln2_g"), L.get("ln2_b"))
+    x = x + gelu(m @ _f(L["W1"]).T) @ _f(L["W2"]).T
+    return x
+
+
+def encoder(X, E_tilde, sel: Dict, n_heads: int, eps: float) -> np.ndarray:
+    """H = Enc([X; E~_text])_[1:N] (Eq. 3): joint encoding, visual rows kept.
+
+    Reading: the blocks are followed by no final norm.
+    """
+    X = _f(X)
+    x = np.concatenate([X, _f(E_tilde)], axis=0)
+    for L in sel["enc"]:
+        x = encoder_block(x, L, n_heads, eps)
+    return x[:X.shape[0]]
+
+
+# ----------------------------------------------------------------------------
+# pointer decoder (Sec. 3.2, Eq. 4) and grouped execution (Sec. 3.5, Eq. 11)
+# ----------------------------------------------------------------------------
+#
+# Reading of the decoder the paper leaves unspecified (layer count, width):
+#   one pre-LN decoder layer of width h with single-head attention.  A decoder
+#   token is W_in q_t, where q_1 = s_start and q_{t+1} = M[a_t] is the hard
+#   forward value of M^T p~_t.  Causal self-attention over the history gives
+#     u_t = y_t + Wo_s * sum_i softmax_i(<Wq_s x_t, Wk_s x_i> / sqrt h) Wv_s x_i,
+#     x_i = LN1(y_i),
+#   and the pointer logits are the cross-attention scores of that layer:
+#     l_t(j) = <Wq_p LN2(u_t), Wk_p M_j> / sqrt h,  j in 1..N+1 (N+1 = STOP).
+#   In the last layer the cross-attention values and the FFN do not feed the
+#   logits, so they are not computed.  The STOP logit gets an extra per-episode
+#   stop_bias (the knob that sets the mean retained count of random-init models).
+
+def decoder_tokens(rows, dec: Dict) -> np.ndarray:
+    """Decoder input tokens y = W_in m for rows m in the D-wide memory space."""
+    return _f(rows) @ _f(dec["W_in"]).T
+
+
+def pointer_keys(M, dec: Dict) -> np.ndarray:
+    """Cross-attention keys Wk_p M_j of all N+1 candidates."""
+    return _f(M) @ _f(dec["Wk_p"]).T
+
+
+def pointer_logits_from_scratch(history_rows, M, dec: Dict, eps: float) -> np.ndarray:
+    """Raw pointer logits l_t over all N+1 rows of M, recomputing the whole
+    decoder over the history [q_1, ..., q_t] (no cached state)."""
+    h = dec["W_in"].shape[0]
+    Y = decoder_tokens(history_rows, dec)
+    X1 = layer_norm(Y, eps, dec.get("ln1_g"), dec.get("ln1_b"))
+    Q = X1 @ _f(dec["Wq_s"]).T
+    K = X1 @ _f(dec["Wk_s"]).T
+    V = X1 @ _f(dec["Wv_s"]).T
+    t = Y.shape[0]
+    S = Q @ K.T / math.sqrt(h)
+    S[np.triu_indices(t, 1)] = NEG_INF
+    U = Y + (softmax(S, axis=-1) @ V) @ _f(dec["Wo_s"]).T
+    query = layer_norm(U[-1], eps, dec.get("ln2_g"), dec.get("ln2_b")) @ _f(dec["Wq_p"]).T
+    return pointer_keys(M, dec) @ query / math.sqrt(h)
+
+
+class _IncrementalDecoder:
+    """The same decoder with the history's keys and values cached; each step
+    adds the new tokens and evaluates only the last position."""
+
+    def __init__(self, M, dec: Dict, eps: float):
+        self.dec, self.eps = dec, eps
+        self.h = dec["W_in"].shape[0]
+        self.Kp = pointer_keys(M, dec)
+        self.Y: List[np.ndarray] = []
+        self.Ks: List[np.ndarray] = []
+        self.Vs: List[np.ndarray] = []
+
+    def append(self, rows):
+        d = self.dec
+        for y in decoder_tokens(np.atleast_2d(rows), d):
+            x = layer_norm(y, self.eps, d.get("ln1_g"), d.get("ln1_b"))
+            self.Y.append(y)
+            self.Ks.append(x @ _f(d["Wk_s"]).T)
+            self.Vs.append(x @ _f(d["Wv_s"]).T)
+
+    def logits(self) -> np.ndarray:
+        d, h = self.dec, self.h
+        y = self.Y[-1]
+        x = layer_norm(y, self.eps, d.get("ln1_g"), d.get("ln1_b"))
+        q = x @ _f(d["Wq_s"]).T
+        a = softmax(np.stack(self.Ks) @ q / math.sqrt(h))
+        u = y + (a @ np.stack(self.Vs)) @ _f(d["Wo_s"]).T
+        query = layer_norm(u, self.eps, d.get("ln2_g"), d.get("ln2_b")) @ _f(d["Wq_p"]).T
+        return self.Kp @ query / math.sqrt(h)
+
+
+def select_episode(H, dec: Dict, *, k_max: int, g: int = 1, stop_bias: float = 0.0,
+                   eps: float = 1e-5, mode: str = "incremental") -> Dict:
+    """Algorithm 1, steps 2-3, over one candidate memory.
+
+    H: [N, D] encoded visual candidates; M = [H; s_stop] (STOP is row N).
+    Each round: l_r = PtrAttn(q_r, M) + Mask_r (+ stop_bias on STOP).
+      * STOP wins when its logit is strictly above every still-available visual
+        logit (ties go to the lower index, and STOP has the highest index);
+        the round is counted and the episode ends.
+      * Otherwise U_r = TopG of the available visual logits (Eq. 11), ordered by
+        (logit desc, index asc), truncated to k_max - |S|; U_r joins S, is
+        masked, and its rows M[U_r] join the causal history in that order.
+      * The loop ends without another evaluation once |S| = k_max (reading of the
+        cap: the paper's T_max counts steps, the workloads state a token cap).
+      * With every visual candidate taken, only STOP is left and wins.
+
+    Returns the step-order selection, its count, and per evaluated round:
+    'margin' (smallest gap between consecutive values among the top g+1 of the
+    available visual logits and STOP: the sensitivity of the round's decision)
+    and 'gap' (best available visual logit minus the raw STOP logit, before
+    stop_bias).
+    """
+    H = _f(H)
+    N = H.shape[0]
+    M = np.concatenate([H, _f(dec["s_stop"])[None, :]], axis=0)
+    stop = N
+    taken = np.zeros(N, dtype=bool)
+    S: List[int] = []
+    margins: List[float] = []
+    gaps: List[float] = []
+    stopped = False
+    history = [_f(dec["s_start"])]
+    inc = None
+    if mode == "incremental":
+        inc = _IncrementalDecoder(M, dec, eps)
+        inc.append(history[0])
+    elif mode != "scratch":
+        raise ValueError(mode)
+
+    while len(S) < k_max:
+        if inc is not None:
+            raw = inc.logits()
+        else:
+            raw = pointer_logits_from_scratch(np.stack(history), M, dec, eps)
+        logits = raw.copy()
+        logits[stop] += stop_bias
+        logits[:N][taken] = NEG_INF
+        avail = np.flatnonzero(~taken)
+        if avail.size == 0:
+            gaps.append(NEG_INF)
+            margins.append(np.inf)
+            stopped = True
+            break
+        vis = logits[avail]
+        # candidates ranked by (logit desc, index asc); STOP ranks after equal visual logits
+        rank = np.lexsort((avail, -vis))
+        best = vis[rank[0]]
+        gaps.append(float(best - raw[stop]))
+        top = sorted([float(v) for v in vis[rank[:g + 1]]] + [float(logits[stop])], reverse=True)
+        top = top[:g + 1]
+        margins.append(min((top[i] - top[i + 1] for i in range(len(top) - 1)), default=np.inf))
+        if logits[stop] > best:
+            stopped = True
+            break
+        take = min(g, k_max - len(S), avail.size)
+        U = [int(avail[i]) for i in rank[:take]]
+        S.extend(U)
+        taken[U] = True
+        if inc is not None:
+            inc.append(M[U])
+        else:
+            history.extend(M[U])
+    return {"order": S, "count": len(S), "margin": margins, "gap": gaps,
+            "rounds": len(margins), "stopped": stopped}
+
+
+def restore(S: Sequence[int]) -> np.ndarray:
+    """Algorithm 1 step 4: the retained indices in native visual order."""
+    return np.sort(np.asarray(S, dtype=np.int64))
+
+
+def select_image(H_b, dec: Dict, *, k_max: int, g: int, group_size: int,
+                 stop_bias: Sequence[float], eps: float = 1e-5,
+                 mode: str = "incremental") -> Dict:
+    """Selection over one image whose candidates may be split into groups.
+
+    Reading (candidate groups; the paper's 'grouped' means g tokens per round):
+    each contiguous group of group_size candidates is an independent episode with
+    its own mask, history and cap, the shared s_start / s_stop, and its own
+    stop_bias entry; the image keeps the union of the groups' selections,
+    offset to image positions and restored to native order.  group_size 0 means
+    one episode over the whole image.
+    """
+    H_b = _f(H_b)
+    N = H_b.shape[0]
+    gs = group_size if group_size > 0 else N
+    starts = list(range(0, N, gs))
+    if len(stop_bias) != len(starts):
+        raise ValueError("one stop_bias per episode")
+    eps_out, idx = [], []
+    for e, s in enumerate(starts):
+        r = select_episode(H_b[s:s + gs], dec, k_max=k_max, g=g, stop_bias=float(stop_bias[e]),
+                           eps=eps, mode=mode)
+        eps_out.append(r)
+        idx.extend(s + i for i in r["order"])
+    return {"idx": restore(idx), "count": len(idx), "episodes": eps_out}
+
+
+# ----------------------------------------------------------------------------
+# compaction, projector, LM prefill
+# ----------------------------------------------------------------------------
+
+def compact(X, n_vis: Sequence[int], idx_list: Sequence[Sequence[int]], text, n_txt: Sequence[int]):
+    """Algorithm 1 step 5 plus the LM input layout: per image the gathered visual
+    rows X_b[idx_b] (native order) followed by the image's text rows.
+
+    Reading: positions restart at 0 for every sequence (1-D RoPE of the LLaVA /
+    Llama convention), and the visual prefix precedes the text (Sec. 3.3-3.4).
+    Returns the packed rows, cu_seqlens [B+1] and positions [T].
+    """
+    X, text = _f(X), _f(text)
+    rows, lens = [], []
+    v0 = t0 = 0
+    for b in range(len(n_vis)):
+        Xb = X[v0:v0 + n_vis[b]]
+        sel = np.asarray(idx_list[b], dtype=np.int64)
+        rows.append(Xb[sel])
+        rows.append(text[t0:t0 + n_txt[b]])
+        lens.append(len(sel) + n_txt[b])
+        v0 += n_vis[b]
+        t0 += n_txt[b]
+    packed = np.concatenate(rows, axis=0) if rows else np.zeros((0, X.shape[1]))
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    pos = np.concatenate([np.arange(n) for n in lens]).astype(np.int64) if lens else np.zeros(0, np.int64)
+    return packed, cu, pos
+
+
+def projector(rows, head: Dict) -> np.ndarray:
+    """Frozen multimodal projector applied to the kept visual rows after the
+    restore (Sec. 3.3): linear W1 x, or the two-layer W2 GELU(W1 x)."""
+    kind = head["proj_kind"]
+    rows = _f(rows)
+    if kind == "none":
+        return rows
+    if kind == "linear":
+        return rows @ _f(head["proj_W1"]).T
+    if kind == "mlp2":
+        return gelu(rows @ _f(head["proj_W1"]).T) @ _f(head["proj_W2"]).T
+    raise ValueError(kind)
+
+
+def rope(x, pos, n_heads: int, head_dim: int, theta: float) -> np.ndarray:
+    """Rotate-half rotary embedding: in every head, pair (i, i + dh/2) is rotated
+    by angle pos * theta^(-2i/dh)."""
+    x = _f(x).reshape(x.shape[0], n_heads, head_dim)
+    half = head_dim // 2
+    inv = theta ** (-(2.0 * np.arange(half, dtype=F64)) / head_dim)
+    ang = _f(pos)[:, None] * inv[None, :]
+    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    a, b = x[..., :half], x[..., half:]
+    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1).reshape(x.shape[0], -1)
+
+
+def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos) -> np.ndarray:
+    """One pre-norm decoder layer of the frozen LM over the packed sequences:
+    h += Wo Attn(RoPE(Wq x), RoPE(Wk x), Wv x), x = RMSNorm(h);
+    h += Wdown (SiLU(Wg x') * Wu x'), x' = RMSNorm(h).  Attention is causal and
+    never crosses a sequence boundary."""
+    h = _f(h).copy()
+    Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
+    x = rms_norm(h, m.rms_eps, L.get("attn_norm"))
+    qkv = x @ _f(L["Wqkv"]).T
+    q = rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta)
+    k = rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta)
+    v = qkv[:, (Hq + Hkv) * dh:]
+    o = np.zeros((h.shape[0], Hq * dh), dtype=F64)
+    for b in range(len(cu) - 1):
+        s, e = int(cu[b]), int(cu[b + 1])
+        if e > s:
+            o[s:e] = attention(q[s:e], k[s:e], v[s:e], Hq, Hkv, causal=True)
+    h = h + o @ _f(L["Wo"]).T
+    x2 = rms_norm(h, m.rms_eps, L.get("mlp_norm"))
+    gu = x2 @ _f(L["Wgu"]).T
+    h = h + (silu(gu[:, :F]) * gu[:, F:]) @ _f(L["Wdown"]).T
+    return h
+
+
+def final_norm(h, m, gain=None) -> np.ndarray:
+    """Output hidden states: RMSNorm of the last residual (the convention of
+    returning the normalised last hidden state)."""
+    return rms_norm(h, m.rms_eps, gain)
+
+
+def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None) -> np.ndarray:
+    h = _f(x)
+    for L in layers:
+        h = prefill_layer(h, L, m, cu, pos)
+    return final_norm(h, m, final_gain)
+
+
+# ----------------------------------------------------------------------------
+# the whole path (Algorithm 1 followed by the pruned prefill)
+# ----------------------------------------------------------------------------
+
+def run_pipeline(X, E_text, n_vis, n_txt, sel: Dict, sel_shape, head: Dict, layers, model_shape,
+                 *, k_max: int, g: int, group_size: int, stop_bias: Sequence[float],
+                 mode: str = "incremental") -> Dict:
+    """Selector encoder -> selection -> restore -> gather -> projector -> prefill."""
+    X, E_text = _f(X), _f(E_text)
+    n_heads = sel_shape.D // sel_shape.enc_head_dim
+    idx_list, eps_per_img = [], []
+    v0 = t0 = e0 = 0
+    H_all = []
+    for b in range(len(n_vis)):
+        Et = text_projection(E_text[t0:t0 + n_txt[b]], sel, sel_shape.ln_eps, sel_shape.g_text)
+        Hb = encoder(X[v0:v0 + n_vis[b]], Et, sel, n_heads, sel_shape.ln_eps)
+        H_all.append(Hb)
+        gs = group_size if group_size > 0 else n_vis[b]
+        ne = (n_vis[b] + gs - 1) // gs
+        r = select_image(Hb, sel, k_max=k_max, g=g, group_size=group_size,
+                         stop_bias=stop_bias[e0:e0 + ne], eps=sel_shape.ln_eps, mode=mode)
+        idx_list.append(r["idx"])
+        eps_per_img.append(r)
+        v0 += n_vis[b]
+        t0 += n_txt[b]
+        e0 += ne
+    # gather (native order) then project the kept rows, then lay out [visual; text]
+    v0 = 0
+    vis_proj = []
+    for b in range(len(n_vis)):
+        vis_proj.append(projector(X[v0:v0 + n_vis[b]][idx_list[b]], head))
+        v0 += n_vis[b]
+    packed_rows, lens = [], []
+    t0 = 0
+    for b in range(len(n_vis)):
+        packed_rows += [vis_proj[b], E_text[t0:t0 + n_txt[b]]]
+        lens.append(len(idx_list[b]) + n_txt[b])
+        t0 += n_txt[b]
+    x = np.concatenate(packed_rows, axis=0)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    pos = np.concatenate([np.arange(n) for n in lens])
+    hidden = prefill(x, layers, model_shape, cu, pos, head.get("final_norm"))
+    return {"H": H_all, "idx": idx_list, "images": eps_per_img, "x": x, "cu_seqlens": cu,
+            "pos": pos, "hidden": hidden}

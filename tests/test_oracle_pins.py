@@ -1,0 +1,380 @@
+"""Pins of the CPU oracle against things other than itself: library routines
+(torch fp64 modules), closed forms, brute force and the special cases the paper's
+definitions reduce to.  No GPU, no CUDA library."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import core as O
+from paper_2609_13804_gb300 import synth as S
+
+torch.set_default_dtype(torch.float64)
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def t64(x):
+    return torch.as_tensor(np.asarray(x, dtype=np.float64))
+
+
+# ---------------------------------------------------------------- elementary
+
+def test_norms_and_activations_match_torch():
+    x = S.normal(1, "x", (7, 33)).astype(np.float64) * 3
+    g = S.normal(1, "g", (33,)).astype(np.float64)
+    b = S.normal(1, "b", (33,)).astype(np.float64)
+    ref = torch.nn.functional.layer_norm(t64(x), (33,), t64(g), t64(b), 1e-5).numpy()
+    np.testing.assert_allclose(O.layer_norm(x, 1e-5, g, b), ref, rtol=0, atol=1e-12)
+    ref = torch.nn.functional.rms_norm(t64(x), (33,), t64(g), 1e-6).numpy()
+    np.testing.assert_allclose(O.rms_norm(x, 1e-6, g), ref, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(O.gelu(x), torch.nn.functional.gelu(t64(x)).numpy(), atol=1e-12)
+    np.testing.assert_allclose(O.silu(x), torch.nn.functional.silu(t64(x)).numpy(), atol=1e-12)
+
+
+def test_gelu_closed_form_points():
+    # Phi(0) = 1/2, Phi(1) = 0.8413447460685429, Phi(-1) = 0.15865525393145707
+    np.testing.assert_allclose(O.gelu([0.0, 1.0, -1.0]),
+                               [0.0, 0.8413447460685429, -0.15865525393145707], atol=1e-15)
+
+
+@pytest.mark.parametrize("hq,hkv,causal", [(4, 4, True), (4, 2, True), (6, 1, False), (2, 2, False)])
+def test_attention_matches_torch_sdpa(hq, hkv, causal):
+    L, dh = 9, 8
+    q = S.normal(2, "q", (L, hq * dh)).astype(np.float64)
+    k = S.normal(2, "k", (L, hkv * dh)).astype(np.float64)
+    v = S.normal(2, "v", (L, hkv * dh)).astype(np.float64)
+    out = O.attention(q, k, v, hq, hkv, causal)
+    # torch layout [heads, L, dh]; expand kv heads explicitly (group of hq/hkv queries per kv head)
+    Q = t64(q).view(L, hq, dh).transpose(0, 1)
+    K = t64(k).view(L, hkv, dh).transpose(0, 1).repeat_interleave(hq // hkv, dim=0)
+    V = t64(v).view(L, hkv, dh).transpose(0, 1).repeat_interleave(hq // hkv, dim=0)
+    ref = torch.nn.functional.scaled_dot_product_attention(Q, K, V, is_causal=causal)
+    np.testing.assert_allclose(out, ref.transpose(0, 1).reshape(L, hq * dh).numpy(), atol=1e-12)
+
+
+def test_attention_single_token_returns_value_and_is_causal():
+    dh = 4
+    q = S.normal(3, "q", (5, 2 * dh)).astype(np.float64)
+    k = S.normal(3, "k", (5, 2 * dh)).astype(np.float64)
+    v = S.normal(3, "v", (5, 2 * dh)).astype(np.float64)
+    np.testing.assert_allclose(O.attention(q[:1], k[:1], v[:1], 2, 2, True), v[:1], atol=1e-15)
+    base = O.attention(q, k, v, 2, 2, True)
+    k2, v2 = k.copy(), v.copy()
+    k2[3:] += 5.0
+    v2[3:] -= 7.0
+    pert = O.attention(q, k2, v2, 2, 2, True)
+    np.testing.assert_allclose(pert[:3], base[:3], atol=1e-15)
+    assert np.abs(pert[3:] - base[3:]).max() > 1e-3
+
+
+# ---------------------------------------------------------------- selector encoder (Eq. 3)
+
+def test_encoder_matches_torch_transformer_encoder_layer():
+    w = S.tiny_workload(4, [10], [6], D=32, D_text=48, enc_head_dim=16)
+    sel = S.make_selector_weights(w, ln_affine=True)
+    for L in sel["enc"]:                 # torch's bias-free layer has bias-free LayerNorms
+        L["ln1_b"] = np.zeros_like(L["ln1_b"])
+        L["ln2_b"] = np.zeros_like(L["ln2_b"])
+    inp = S.make_inputs(w)
+    X, E = inp["X"].astype(np.float64), inp["E_text"].astype(np.float64)
+    s = w.selector
+    Et = O.text_projection(E, sel, s.ln_eps)
+    ref_Et = torch.nn.functional.layer_norm(
+        torch.nn.functional.linear(t64(E), t64(sel["W_p"])), (s.D,),
+        t64(sel["ln_text_g"]), t64(sel["ln_text_b"]), s.ln_eps).numpy()
+    np.testing.assert_allclose(Et, ref_Et, atol=1e-12)
+    H = O.encoder(X, Et, sel, s.enc_heads, s.ln_eps)
+
+    x = t64(np.concatenate([X, Et]))[None]
+    for L in sel["enc"]:
+        layer = torch.nn.TransformerEncoderLayer(
+            s.D, s.enc_heads, s.enc_ffn, dropout=0.0, activation="gelu", layer_norm_eps=s.ln_eps,
+            batch_first=True, norm_first=True, bias=False, dtype=torch.float64)
+        with torch.no_grad():
+            layer.self_attn.in_proj_weight.copy_(t64(L["Wqkv"]))
+            layer.self_attn.out_proj.weight.copy_(t64(L["Wo"]))
+            layer.linear1.weight.copy_(t64(L["W1"]))
+            layer.linear2.weight.copy_(t64(L["W2"]))
+            layer.norm1.weight.copy_(t64(L["ln1_g"]))
+            layer.norm2.weight.copy_(t64(L["ln2_g"]))
+        layer.eval()
+        with torch.no_grad():
+            x = layer(x)
+    np.testing.assert_allclose(H, x[0, :10].numpy(), atol=1e-10)
+    assert H.shape == (10, s.D)
+
+
+# ---------------------------------------------------------------- pointer decoder (Eq. 4)
+
+def _scaled_selector(seed, N=14, D=24, h=16, scale=0.3, ln_affine=True):
+    """Tiny selector whose logits are O(1) so that near-ties are rare."""
+    w = S.tiny_workload(seed, [N], [3], D=D, h=h)
+    sel = S.make_selector_weights(w, ln_affine=ln_affine)
+    for n in ("W_in", "Wq_s", "Wk_s", "Wv_s", "Wo_s", "Wq_p", "Wk_p", "s_start", "s_stop"):
+        sel[n] = (sel[n] / 0.02 * scale / math.sqrt(sel[n].shape[-1])).astype(np.float32)
+    H = S.make_memory(w).astype(np.float64)
+    return sel, H
+
+
+def test_pointer_logits_match_torch_multihead_attention_decoder():
+    """The decoder of Eq. 4 built from torch.nn.MultiheadAttention (1 head, no
+    biases): causal self-attention with residual, then cross-attention to M whose
+    attention probabilities are softmax(l_t + Mask_t)."""
+    sel, H = _scaled_selector(5)
+    N, D = H.shape
+    h = sel["W_in"].shape[0]
+    M = np.concatenate([H, sel["s_stop"][None].astype(np.float64)])
+    hist = np.stack([sel["s_start"], M[3], M[7], M[1]]).astype(np.float64)
+    ours = O.pointer_logits_from_scratch(hist, M, sel, 1e-5)
+
+    sa = torch.nn.MultiheadAttention(h, 1, bias=False, batch_first=True)
+    ca = torch.nn.MultiheadAttention(h, 1, bias=False, kdim=D, vdim=D, batch_first=True)
+    with torch.no_grad():
+        sa.in_proj_weight.copy_(t64(np.concatenate([sel["Wq_s"], sel["Wk_s"], sel["Wv_s"]])))
+        sa.out_proj.weight.copy_(t64(sel["Wo_s"]))
+        ca.q_proj_weight.copy_(t64(sel["Wq_p"]))
+        ca.k_proj_weight.copy_(t64(sel["Wk_p"]))
+        ca.v_proj_weight.copy_(torch.randn(h, D))
+    ln1 = lambda y: torch.nn.functional.layer_norm(y, (h,), t64(sel["ln1_g"]), t64(sel["ln1_b"]), 1e-5)
+    ln2 = lambda y: torch.nn.functional.layer_norm(y, (h,), t64(sel["ln2_g"]), t64(sel["ln2_b"]), 1e-5)
+    with torch.no_grad():
+        y = torch.nn.functional.linear(t64(hist), t64(sel["W_in"]))[None]
+        causal = torch.triu(torch.full((4, 4), float("-inf")), 1)
+        x = ln1(y)
+        u = y + sa(x, x, x, attn_mask=causal, need_weights=False)[0]
+        mask = torch.zeros(1, N + 1)
+        mask[0, [3, 7, 1]] = float("-inf")
+        _, p = ca(ln2(u[:, -1:]), t64(M)[None], t64(M)[None], attn_mask=mask, need_weights=True)
+    logp = torch.log(p[0, 0]).numpy()
+    avail = [j for j in range(N + 1) if j not in (3, 7, 1)]
+    d_ours = ours[avail] - ours[avail].max()
+    d_ref = logp[avail] - logp[avail].max()
+    np.testing.assert_allclose(d_ours, d_ref, atol=1e-10)
+
+
+@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("g", [1, 3])
+def test_incremental_selection_equals_brute_force(seed, g):
+    sel, H = _scaled_selector(100 + seed, N=11 + seed % 5)
+    N = H.shape[0]
+    for bias in (-0.4, 0.0, 0.5, -1e9):
+        for k_max in (3, 8, N + 3):
+            a = O.select_episode(H, sel, k_max=k_max, g=g, stop_bias=bias)
+            b = O.select_episode(H, sel, k_max=k_max, g=g, stop_bias=bias, mode="scratch")
+            assert a["order"] == b["order"]
+            assert a["stopped"] == b["stopped"]
+            np.testing.assert_allclose(a["gap"], b["gap"], atol=1e-12)
+            np.testing.assert_allclose(a["margin"], b["margin"], atol=1e-12)
+
+
+def _exhaustive_greedy(H, sel, k_max, g, bias):
+    """Brute force written from Alg. 1 without the oracle's episode loop: at every
+    round rescore all N+1 candidates from scratch, then pick by a full sort."""
+    N = H.shape[0]
+    M = np.concatenate([H, sel["s_stop"][None].astype(np.float64)])
+    hist, S_ = [sel["s_start"].astype(np.float64)], []
+    while len(S_) < k_max:
+        l = O.pointer_logits_from_scratch(np.stack(hist), M, sel, 1e-5)
+        l[N] += bias
+        cand = [(-l[j], j) for j in range(N) if j not in S_]
+        if not cand:
+            break
+        cand.sort()
+        if l[N] > -cand[0][0]:
+            break
+        for _, j in cand[:min(g, k_max - len(S_))]:
+            S_.append(j)
+            hist.append(M[j])
+    return S_
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_selection_equals_exhaustive_greedy(seed):
+    sel, H = _scaled_selector(200 + seed, N=9)
+    for g in (1, 2, 5):
+        for bias in (-0.3, 0.2, -1e9):
+            ref = _exhaustive_greedy(H, sel, 7, g, bias)
+            assert O.select_episode(H, sel, k_max=7, g=g, stop_bias=bias)["order"] == ref
+
+
+def test_history_free_case_reduces_to_static_top_k():
+    """With W_in = 0 every decoder token is 0, LN1 returns its bias, so queries,
+    keys and values are the same at every position and the pointer query does
+    not depend on the history: the policy is Eq. 1's independent top-K whose K
+    is the number of static scores strictly above the STOP logit (capped)."""
+    sel, H = _scaled_selector(7, N=40)
+    sel["W_in"] = np.zeros_like(sel["W_in"])
+    N = H.shape[0]
+    h = sel["W_in"].shape[0]
+    x = sel["ln1_b"].astype(np.float64)                       # LN1(0) = bias
+    u = (x @ sel["Wv_s"].T.astype(np.float64)) @ sel["Wo_s"].T.astype(np.float64)
+    q = O.layer_norm(u, 1e-5, sel["ln2_g"], sel["ln2_b"]) @ sel["Wq_p"].T.astype(np.float64)
+    M = np.concatenate([H, sel["s_stop"][None].astype(np.float64)])
+    static = (M @ sel["Wk_p"].T.astype(np.float64)) @ q / math.sqrt(h)
+    order = sorted(range(N), key=lambda j: (-static[j], j))
+    for bias in (-0.5, 0.0, 0.3, -1e9):
+        stop = static[N] + bias
+        K = sum(1 for j in range(N) if static[j] > stop)
+        for k_max in (5, 12, 50):
+            for g in (1, 5):
+                # Sec. 3.5: STOP is only checked at the start of a round, so with
+                # g tokens per round the kept set is the top g*ceil(K/g) (capped)
+                want = order[:min(g * math.ceil(K / g), N, k_max)]
+                r = O.select_episode(H, sel, k_max=k_max, g=g, stop_bias=bias)
+                assert r["order"] == want
+                k = len(want)
+                stopped = k < k_max
+                assert r["rounds"] == math.ceil(k / g) + (1 if stopped else 0)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_selection_invariants_and_bias_monotonicity(seed):
+    sel, H = _scaled_selector(300 + seed, N=30)
+    N = H.shape[0]
+    base = O.select_episode(H, sel, k_max=N, g=1, stop_bias=-1e9)
+    gaps = np.array(base["gap"])
+    prev_k = None
+    for bias in np.linspace(-1.5, 1.5, 13):
+        r = O.select_episode(H, sel, k_max=20, g=1, stop_bias=bias)
+        o = r["order"]
+        assert len(set(o)) == len(o) and r["count"] == len(o) <= 20
+        assert all(0 <= i < N for i in o)
+        # the trajectory does not depend on the bias until STOP wins
+        assert o == base["order"][:len(o)]
+        # closed form: K(b) = first round t with gap_t < b, minus one; capped by k_max
+        t = next((i for i, gp in enumerate(gaps) if gp < bias), len(gaps))
+        assert r["count"] == min(t, 20)
+        if prev_k is not None:
+            assert r["count"] <= prev_k
+        prev_k = r["count"]
+    assert list(O.restore(o)) == sorted(o)
+
+
+def test_selection_extremes():
+    sel, H = _scaled_selector(9, N=6)
+    assert O.select_episode(H, sel, k_max=4, stop_bias=1e9)["count"] == 0
+    r = O.select_episode(H, sel, k_max=100, stop_bias=-1e9)
+    assert sorted(r["order"]) == list(range(6)) and r["stopped"]
+    r = O.select_episode(H[:1], sel, k_max=3, stop_bias=-1e9)
+    assert r["order"] == [0] and r["rounds"] == 2
+    r = O.select_episode(H, sel, k_max=5, g=50, stop_bias=-1e9)
+    assert r["count"] == 5 and r["rounds"] == 1
+    img = O.select_image(H, sel, k_max=2, g=1, group_size=1, stop_bias=[-1e9] * 6)
+    assert list(img["idx"]) == list(range(6))
+
+
+def test_candidate_groups_are_independent_episodes():
+    sel, H = _scaled_selector(10, N=23)
+    biases = [-0.1, 0.2, -1e9]
+    img = O.select_image(H, sel, k_max=4, g=2, group_size=10, stop_bias=biases)
+    want = []
+    for e, s in enumerate((0, 10, 20)):
+        r = O.select_episode(H[s:s + 10], sel, k_max=4, g=2, stop_bias=biases[e])
+        want += [s + i for i in r["order"]]
+    assert list(img["idx"]) == sorted(want)
+
+
+# ---------------------------------------------------------------- compaction (Alg. 1 step 5)
+
+def test_compaction_golden_fixture():
+    with open(os.path.join(GOLDEN, "compact_tiny.json")) as f:
+        gold = json.load(f)
+    packed, cu, pos = O.compact(np.array(gold["X"]), gold["n_vis"], gold["idx"],
+                                np.array(gold["text"]), gold["n_txt"])
+    np.testing.assert_array_equal(packed, np.array(gold["packed"]))
+    np.testing.assert_array_equal(cu, gold["cu_seqlens"])
+    np.testing.assert_array_equal(pos, gold["pos"])
+
+
+# ---------------------------------------------------------------- RoPE and the LM layer
+
+def test_rope_is_a_rotation_with_relative_positions():
+    dh, H = 8, 2
+    x = S.normal(11, "x", (5, H * dh)).astype(np.float64)
+    pos = np.array([0, 1, 2, 7, 100])
+    r = O.rope(x, pos, H, dh, 1e4)
+    np.testing.assert_allclose(r[0], x[0], atol=1e-15)
+    xr, rr = x.reshape(5, H, dh), r.reshape(5, H, dh)
+    for i in range(dh // 2):   # each (i, i + dh/2) pair keeps its length
+        np.testing.assert_allclose(xr[..., i] ** 2 + xr[..., i + 4] ** 2,
+                                   rr[..., i] ** 2 + rr[..., i + 4] ** 2, atol=1e-12)
+    # pair 0 rotates by exactly pos radians (inv_freq_0 = 1)
+    e = np.zeros((1, dh)); e[0, 0] = 1.0
+    rot = O.rope(e, np.array([1.0]), 1, dh, 1e4)
+    np.testing.assert_allclose([rot[0, 0], rot[0, 4]], [math.cos(1.0), math.sin(1.0)], atol=1e-15)
+    # <R_m q, R_n k> depends only on m - n
+    q = S.normal(11, "q", (1, dh)).astype(np.float64)
+    k = S.normal(11, "k", (1, dh)).astype(np.float64)
+    d1 = O.rope(q, [5], 1, dh, 1e4) @ O.rope(k, [2], 1, dh, 1e4).T
+    d2 = O.rope(q, [33], 1, dh, 1e4) @ O.rope(k, [30], 1, dh, 1e4).T
+    np.testing.assert_allclose(d1, d2, atol=1e-12)
+
+
+def _tiny_lm(seed, hq=4, hkv=2):
+    w = S.tiny_workload(seed, [5, 3], [2, 4], d=32, n_heads=hq, n_kv_heads=hkv, head_dim=8, ffn=40)
+    L = S.make_layer_weights(w, 0, norm_affine=True)
+    for k in ("Wqkv", "Wo", "Wgu", "Wdown"):
+        L[k] = L[k] / 0.02 * 0.15
+    return w, L
+
+
+def test_prefill_layer_zero_output_weights_is_identity():
+    w, L = _tiny_lm(12)
+    L["Wo"] = np.zeros_like(L["Wo"])
+    L["Wdown"] = np.zeros_like(L["Wdown"])
+    x = S.normal(12, "x", (14, 32)).astype(np.float64)
+    cu, pos = [0, 7, 14], np.r_[np.arange(7), np.arange(7)]
+    np.testing.assert_allclose(O.prefill_layer(x, L, w.model, cu, pos), x, atol=1e-15)
+
+
+def test_prefill_layer_uniform_attention_closed_form():
+    """Wq = 0 makes every causal score equal: the attention output at position p
+    is the mean of the values at 0..p of its own sequence."""
+    w, L = _tiny_lm(13, hq=4, hkv=4)
+    m = w.model
+    dq = m.n_heads * m.head_dim
+    L["Wqkv"][:dq] = 0.0
+    L["Wo"] = np.eye(m.d, dq)
+    L["Wdown"] = np.zeros_like(L["Wdown"])
+    x = S.normal(13, "x", (9, m.d)).astype(np.float64)
+    cu, pos = [0, 4, 9], np.r_[np.arange(4), np.arange(5)]
+    out = O.prefill_layer(x, L, m, cu, pos)
+    v = O.rms_norm(x, m.rms_eps, L["attn_norm"]) @ L["Wqkv"][2 * dq:].astype(np.float64).T
+    want = np.zeros_like(v)
+    for s, e in ((0, 4), (4, 9)):
+        for p in range(s, e):
+            want[p] = v[s:p + 1].mean(axis=0)
+    np.testing.assert_allclose(out - x, want, atol=1e-12)
+
+
+def test_prefill_varlen_isolation_and_causality():
+    w, L = _tiny_lm(14)
+    m = w.model
+    x = S.normal(14, "x", (11, m.d)).astype(np.float64)
+    cu, pos = [0, 6, 11], np.r_[np.arange(6), np.arange(5)]
+    both = O.prefill(x, [L, L], m, cu, pos)
+    alone0 = O.prefill(x[:6], [L, L], m, [0, 6], np.arange(6))
+    alone1 = O.prefill(x[6:], [L, L], m, [0, 5], np.arange(5))
+    np.testing.assert_allclose(both, np.concatenate([alone0, alone1]), atol=1e-12)
+    x2 = x.copy()
+    x2[3:6] += 1.0
+    pert = O.prefill(x2, [L, L], m, cu, pos)
+    np.testing.assert_allclose(pert[:3], both[:3], atol=1e-12)
+    np.testing.assert_allclose(pert[6:], both[6:], atol=1e-12)
+
+
+def test_projector_forms():
+    w = S.tiny_workload(15, [4], [2], D=12, d=20)
+    head = S.make_model_head(w)
+    x = S.normal(15, "x", (3, 12)).astype(np.float64)
+    W1, W2 = head["proj_W1"].astype(np.float64), head["proj_W2"].astype(np.float64)
+    ref = torch.nn.Sequential(torch.nn.Linear(12, 20, bias=False), torch.nn.GELU(),
+                              torch.nn.Linear(20, 20, bias=False))
+    with torch.no_grad():
+        ref[0].weight.copy_(t64(W1))
+        ref[2].weight.copy_(t64(W2))
+        want = ref(t64(x)).numpy()
+    np.testing.assert_allclose(O.projector(x, head), want, atol=1e-12)
