@@ -1,0 +1,402 @@
+/*
+ * stepprune.h -- C ABI of the GB300 (sm_103a) StepPrune inference path.
+ *
+ * StepPrune (arXiv 2609.13804) prunes the visual prefix of a multimodal LLM by
+ * sequential selection: a pointer decoder picks visual tokens one round at a
+ * time, conditioned on what it already picked and on the text, until a learned
+ * STOP action wins (Sec. 3.1-3.2, Eq. 2 and Eq. 4; grouped rounds of g tokens,
+ * Sec. 3.5, Eq. 11).  The kept tokens are restored to native order and
+ * physically gathered before the language-model prefill (Algorithm 1 steps 4-5).
+ * This library runs that path on one GPU:
+ *
+ *   sp_select    text projection + cross-modal encoder (Eq. 3), candidate
+ *                precompute, the sequential selection loop, restore.
+ *   sp_compact   gather of the kept visual rows and the text rows into a packed
+ *                variable-length buffer with cu_seqlens and positions.
+ *   sp_project   the frozen multimodal projector on the kept rows, scattered
+ *                into their packed slots.
+ *   sp_prefill   the LM prefill over the packed prefix (hidden states after the
+ *                final RMSNorm).
+ *   sp_pipeline  all four, back to back on one stream.
+ *
+ * Conventions (all entry points):
+ *   - Pointers marked DEVICE are device memory owned by the caller; HOST marks
+ *     host memory read during the call only.  Matrices are row-major; weights
+ *     use the nn.Linear layout [out_features, in_features].  bf16 data is
+ *     passed as raw 16-bit patterns (void*).
+ *   - Calls are asynchronous on the given stream and never synchronise the
+ *     host.  Hot calls (sp_select, sp_compact, sp_project, sp_prefill,
+ *     sp_pipeline) allocate nothing: scratch comes from the caller's workspace,
+ *     sized by the matching *_workspace() query.  Handles allocate at create
+ *     time only and free at destroy.
+ *   - Sizes that depend on the selection (the kept counts, the packed length T)
+ *     stay on the device; grids are sized from host-known caps and kernels
+ *     skip rows past the device count, so no call reads results back.
+ *   - A status is returned for every call; argument problems are detected on
+ *     the host before any launch (nothing is launched then).  The message of
+ *     the last failure on the calling thread is in sp_last_error().
+ *   - Device-side failures (a bounded wait that ran out, an index out of
+ *     range) set bits in the optional DEVICE int error word passed in the
+ *     call; read it after synchronising (see SP_DEVERR_*).  Kernels never trap.
+ *   - No C++ exception crosses the ABI.
+ */
+#ifndef STEPPRUNE_H
+#define STEPPRUNE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SP_API __attribute__((visibility("default")))
+#else
+#define SP_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SP_ABI_VERSION 1
+
+/* Limits checked on the host (SP_ERR_SHAPE when exceeded). */
+#define SP_MAX_BATCH 256          /* images per call */
+#define SP_MAX_ENC_LAYERS 4       /* cross-modal encoder blocks */
+#define SP_MAX_LM_LAYERS 96       /* decoder layers of the LM */
+#define SP_MAX_KMAX 1024          /* per-episode cap on retained tokens */
+#define SP_MAX_NVIS 16384         /* visual tokens of one image */
+
+typedef enum {
+  SP_OK = 0,
+  SP_ERR_INVALID_ARG = 1,   /* NULL where a pointer is required, bad enum, ... */
+  SP_ERR_SHAPE = 2,         /* a size outside the supported set or a limit */
+  SP_ERR_ALIGN = 3,         /* a device pointer not 16-byte aligned */
+  SP_ERR_WORKSPACE = 4,     /* workspace NULL or smaller than *_workspace() */
+  SP_ERR_CUDA = 5,          /* a CUDA runtime call failed (message has the code) */
+  SP_ERR_TIMEOUT = 6,       /* reported by sp_device_error_status() */
+  SP_ERR_UNSUPPORTED = 7,   /* device is not sm_103 / feature not built */
+  SP_ERR_DEVICE = 8         /* reported by sp_device_error_status() */
+} sp_status;
+
+/* Bits of the DEVICE error word. */
+#define SP_DEVERR_TIMEOUT 0x1   /* a bounded wait (mbarrier / flag) ran out */
+#define SP_DEVERR_INDEX 0x2     /* an index outside its range was skipped */
+
+typedef struct CUstream_st* sp_stream; /* a cudaStream_t; NULL is the legacy default stream */
+
+/* Thread-local message of the last failed call ("" if none). */
+SP_API const char* sp_last_error(void);
+/* SP_ABI_VERSION of the loaded library. */
+SP_API int sp_abi_version(void);
+/* Maps a device error word read back by the caller to SP_OK / SP_ERR_TIMEOUT / SP_ERR_DEVICE. */
+SP_API sp_status sp_device_error_status(int device_error_word);
+
+/* ------------------------------------------------------------------------ */
+/* Selector (Sec. 3.2: cross-modal encoder, STOP row, pointer decoder).      */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+  int D;             /* visual feature width = width of the candidate memory M; multiple of 128 */
+  int D_text;        /* width of the prompt embeddings E_text */
+  int h;             /* pointer-decoder width; multiple of 128 in 128..1024 */
+  int n_enc_layers;  /* encoder blocks (the paper uses 2); 0..SP_MAX_ENC_LAYERS */
+  int enc_head_dim;  /* encoder head dim: 64 or 128; D must be a multiple */
+  int enc_ffn;       /* encoder MLP width (4 D in a ViT block) */
+  float ln_eps;      /* LayerNorm epsilon */
+  float g_text;      /* text gate g_text of E~ = g_text LN(W_p E) (1 at inference) */
+} sp_selector_cfg;
+
+/*
+ * Weights of the selector.  The encoder and text projection are bf16 (tensor
+ * cores); the pointer decoder is fp32.  LayerNorm gain/bias pointers may be
+ * NULL (gain 1 / bias 0).  All DEVICE; borrowed by the handle, so they must
+ * outlive it (the handle keeps folded copies of the decoder matrices).
+ *
+ * Reading of the decoder (Sec. 3.2, Eq. 4; the paper fixes no layer count or
+ * width): one pre-LN decoder layer of width h with single-head attention.  A
+ * decoder token is y = W_in q with q_1 = s_start and q_{t+1} = M[a_t]; causal
+ * self-attention gives u_t = y_t + Wo_s sum_i softmax_i(<Wq_s x_t, Wk_s x_i>/sqrt h)
+ * Wv_s x_i with x_i = LN1(y_i); the pointer logits are the cross-attention
+ * scores l_t(j) = <Wq_p LN2(u_t), Wk_p M_j>/sqrt h over the N+1 rows of
+ * M = [H; s_stop], plus a per-episode stop_bias on the STOP row.
+ */
+typedef struct {
+  const void* W_p;                         /* [D, D_text] bf16 text projection */
+  const float* ln_text_g; const float* ln_text_b;    /* [D] */
+  const void* enc_wqkv[SP_MAX_ENC_LAYERS]; /* [3D, D] bf16, rows q|k|v */
+  const void* enc_wo[SP_MAX_ENC_LAYERS];   /* [D, D] bf16 */
+  const void* enc_w1[SP_MAX_ENC_LAYERS];   /* [enc_ffn, D] bf16 */
+  const void* enc_w2[SP_MAX_ENC_LAYERS];   /* [D, enc_ffn] bf16 */
+  const float* enc_ln1_g[SP_MAX_ENC_LAYERS]; const float* enc_ln1_b[SP_MAX_ENC_LAYERS];
+  const float* enc_ln2_g[SP_MAX_ENC_LAYERS]; const float* enc_ln2_b[SP_MAX_ENC_LAYERS];
+  const float* s_stop;                     /* [D] learned STOP embedding */
+  const float* s_start;                    /* [D] learned START embedding (q_1) */
+  const float* W_in;                       /* [h, D] decoder input projection */
+  const float* ln1_g; const float* ln1_b;  /* [h] */
+  const float* Wq_s; const float* Wk_s; const float* Wv_s; const float* Wo_s; /* [h, h] */
+  const float* ln2_g; const float* ln2_b;  /* [h] */
+  const float* Wq_p;                       /* [h, h] pointer query */
+  const float* Wk_p;                       /* [h, D] pointer key */
+} sp_selector_weights;
+
+typedef struct sp_selector_s sp_selector;
+
+/* Validates cfg, allocates the folded decoder matrices and encodes the weight
+ * tensor maps.  Synchronous (uses the legacy stream once). */
+SP_API sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weights* w,
+                             sp_selector** out);
+SP_API void sp_selector_destroy(sp_selector* s);
+
+/*
+ * One batch of images for selection.  Image b owns visual rows
+ * [sum_{c<b} n_vis[c], +n_vis[b]) of X (or H) and text rows likewise of E_text.
+ * Candidate groups: with group_size > 0 the candidates of an image are cut into
+ * consecutive groups of group_size (the last may be shorter); each group is an
+ * independent episode with its own mask, history, cap k_max and stop_bias, all
+ * sharing s_start / s_stop; group_size 0 = one episode per image.  Episodes are
+ * numbered image-major, group-minor.
+ */
+typedef struct {
+  int B;                 /* images, 1..SP_MAX_BATCH */
+  const int* n_vis;      /* HOST [B] visual tokens per image (N_b, 1..SP_MAX_NVIS) */
+  const int* n_txt;      /* HOST [B] text tokens per image (L_b, >= 0) */
+  const void* X;         /* DEVICE [sum N_b, D] bf16 visual tokens; ignored when H is set */
+  const void* E_text;    /* DEVICE [sum L_b, D_text] bf16 prompt embeddings; ignored when H is set */
+  const float* H;        /* DEVICE [sum N_b, D] fp32 encoded candidates, or NULL to run the
+                            text projection and encoder on X / E_text (Eq. 3) */
+  const float* stop_bias;/* DEVICE [n_episodes] fp32 added to the STOP logit */
+  int group_size;        /* candidates per episode (0: whole image) */
+  int g;                 /* visual tokens kept per non-STOP round (1..16); Eq. 11 */
+  int k_max;             /* per-episode cap, 1..SP_MAX_KMAX */
+} sp_select_in;
+
+/*
+ * Outputs.  idx row b holds image b's kept visual indices (image-local) in
+ * ascending (native) order, then -1 up to k_cap.  k_cap must be at least the
+ * largest possible count of an image: sum over its episodes of min(k_max, size).
+ * order / ep_count / margin / gap are optional per-episode traces:
+ *   order[e*k_max + i]   episode-local index taken i-th (step order)
+ *   ep_count[e]          tokens kept by episode e
+ *   margin[e*(k_max+1)+r] round r's smallest gap between consecutive values
+ *                        among the top g+1 available visual logits and STOP
+ *   gap[e*(k_max+1)+r]   round r's best available visual logit minus the raw
+ *                        STOP logit (before stop_bias): STOP wins iff
+ *                        stop_bias > gap, which calibrates stop_bias
+ *   rounds[e]            evaluated rounds of episode e
+ * Unwritten trace entries are left as they were.
+ */
+typedef struct {
+  int* idx;          /* DEVICE [B, k_cap] */
+  int k_cap;
+  int* count;        /* DEVICE [B] kept tokens per image (K_b) */
+  int* order;        /* DEVICE [n_episodes, k_max] or NULL */
+  int* ep_count;     /* DEVICE [n_episodes] or NULL */
+  float* margin;     /* DEVICE [n_episodes, k_max + 1] or NULL */
+  float* gap;        /* DEVICE [n_episodes, k_max + 1] or NULL */
+  int* rounds;       /* DEVICE [n_episodes] or NULL */
+  float* memory;     /* DEVICE [sum N_b, D] fp32 or NULL: receives the candidate memory H
+                        (the encoder output of Eq. 3, or a copy of the given H) */
+  int* err;          /* DEVICE error word (SP_DEVERR_*) or NULL */
+} sp_select_out;
+
+/* Number of episodes of a batch (host arithmetic; -1 on bad arguments). */
+SP_API int sp_num_episodes(int B, const int* n_vis, int group_size);
+/* Workspace bytes sp_select needs for this batch (0 on bad arguments). */
+SP_API size_t sp_select_workspace(const sp_selector* s, const sp_select_in* in);
+/* Algorithm 1 steps 1-4 for every image of the batch (see sp_select_in). */
+SP_API sp_status sp_select(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
+                    void* workspace, size_t workspace_bytes, sp_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* Compaction (Algorithm 1 step 5: X_S = Gather(X, S), then [X_S; text]).    */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Sequence b of the packed output is image b's kept visual rows (native order)
+ * followed by its text rows; positions restart at 0 for every sequence.
+ * T = cu_seqlens[B] is written on the device; T_cap = sum_b (min(n_vis[b], k_cap)
+ * + n_txt[b]) bounds it.
+ *   direct (vis_packed == NULL): W_vis must equal W_txt and visual rows go
+ *     straight into their packed slots (no projector, or one already applied).
+ *   projector mode (vis_packed != NULL): visual rows go to vis_packed, image-
+ *     major and contiguous (vis_cu[b] is image b's first row), and
+ *     vis_row_map[i] is the packed row that projected row i belongs to; the
+ *     visual slots of packed are left for sp_project.
+ */
+typedef struct {
+  int B;
+  const int* n_vis;      /* HOST [B] */
+  const int* n_txt;      /* HOST [B] */
+  const void* X;         /* DEVICE [sum N_b, W_vis] bf16 */
+  int W_vis;             /* multiple of 8 */
+  const void* text;      /* DEVICE [sum L_b, W_txt] bf16 (LM-width prompt embeddings) */
+  int W_txt;             /* multiple of 8 */
+  const int* idx;        /* DEVICE [B, k_cap] from sp_select */
+  int k_cap;
+  const int* count;      /* DEVICE [B] */
+} sp_compact_in;
+
+typedef struct {
+  void* packed;          /* DEVICE [T_cap, W_txt] bf16 */
+  int* cu_seqlens;       /* DEVICE [B + 1] */
+  int* pos;              /* DEVICE [T_cap] */
+  void* vis_packed;      /* DEVICE [sum_b min(n_vis[b], k_cap), W_vis] bf16, or NULL (direct) */
+  int* vis_row_map;      /* DEVICE [same rows] (projector mode) */
+  int* vis_cu;           /* DEVICE [B + 1] (projector mode) */
+  int* err;              /* DEVICE error word or NULL */
+} sp_compact_out;
+
+/* T_cap of a batch (host arithmetic; -1 on bad arguments). */
+SP_API int sp_packed_cap(int B, const int* n_vis, const int* n_txt, int k_cap);
+SP_API sp_status sp_compact(const sp_compact_in* in, const sp_compact_out* out, sp_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* Language model: projector + decoder-only prefill.                          */
+/* ------------------------------------------------------------------------ */
+
+typedef enum { SP_PROJ_NONE = 0, SP_PROJ_LINEAR = 1, SP_PROJ_MLP2_GELU = 2 } sp_proj_kind;
+
+typedef struct {
+  int n_layers;      /* 1..SP_MAX_LM_LAYERS */
+  int d;             /* model width; multiple of 128 */
+  int n_heads;       /* query heads */
+  int n_kv_heads;    /* key/value heads; divides n_heads (GQA when smaller) */
+  int head_dim;      /* 64 or 128 */
+  int ffn;           /* SwiGLU width; multiple of 128 */
+  int max_pos;       /* positions covered by the rotary table (> longest sequence) */
+  float rope_theta;
+  float rms_eps;
+  int proj_kind;     /* sp_proj_kind */
+  int proj_in;       /* visual width entering the projector */
+  int proj_hidden;   /* hidden width of SP_PROJ_MLP2_GELU */
+} sp_model_cfg;
+
+/*
+ * Weights (DEVICE, borrowed; bf16 unless stated).  Per layer:
+ *   wqkv  [(n_heads + 2 n_kv_heads) head_dim, d]  rows q | k | v
+ *   wo    [d, n_heads head_dim]
+ *   wgu   [2 ffn, d]  rows gate | up   (SwiGLU: down(silu(gate x) * up x))
+ *   wdown [d, ffn]
+ *   attn_norm / mlp_norm  fp32 [d] RMSNorm gains, or NULL (1)
+ * final_norm fp32 [d] or NULL.  Projector: proj_w1 [proj_hidden or d, proj_in],
+ * proj_w2 [d, proj_hidden] (SP_PROJ_MLP2_GELU only).
+ */
+typedef struct {
+  const void* wqkv[SP_MAX_LM_LAYERS];
+  const void* wo[SP_MAX_LM_LAYERS];
+  const void* wgu[SP_MAX_LM_LAYERS];
+  const void* wdown[SP_MAX_LM_LAYERS];
+  const float* attn_norm[SP_MAX_LM_LAYERS];
+  const float* mlp_norm[SP_MAX_LM_LAYERS];
+  const float* final_norm;
+  const void* proj_w1;
+  const void* proj_w2;
+} sp_model_weights;
+
+typedef struct sp_model_s sp_model;
+
+/* Validates cfg, uploads the rotary table (fp64 on the host, stored fp32) and
+ * encodes the weight tensor maps.  Synchronous. */
+SP_API sp_status sp_model_create(const sp_model_cfg* cfg, const sp_model_weights* w, sp_model** out);
+SP_API void sp_model_destroy(sp_model* m);
+
+/*
+ * Projector on the kept rows: packed[vis_row_map[i]] = P(vis_packed[i]) for
+ * i < vis_cu[B] (device count), P = W1 x, or W2 GELU(W1 x).  rows_cap bounds
+ * vis_cu[B].
+ */
+typedef struct {
+  int B;
+  int rows_cap;
+  const void* vis_packed;   /* DEVICE [rows_cap, proj_in] bf16 */
+  const int* vis_row_map;   /* DEVICE [rows_cap] */
+  const int* vis_cu;        /* DEVICE [B + 1] */
+  void* packed;             /* DEVICE [T_cap, d] bf16 (visual slots written) */
+  int* err;
+} sp_project_io;
+
+SP_API size_t sp_project_workspace(const sp_model* m, int rows_cap);
+SP_API sp_status sp_project(const sp_model* m, const sp_project_io* io, void* workspace,
+                     size_t workspace_bytes, sp_stream stream);
+
+/*
+ * Prefill of the packed sequences: causal attention within each sequence
+ * (cu_seqlens), rotary positions pos, pre-RMSNorm Llama-style layers, and the
+ * final RMSNorm.  hidden rows t < T = cu_seqlens[B] are written; rows >= T are
+ * untouched.  residual (optional) receives the last residual stream (fp32,
+ * before the final norm).
+ */
+typedef struct {
+  int B;
+  int T_cap;                /* bound on cu_seqlens[B] */
+  int max_seqlen_cap;       /* bound on every sequence length */
+  const void* x;            /* DEVICE [T_cap, d] bf16 packed LM input */
+  const int* cu_seqlens;    /* DEVICE [B + 1] */
+  const int* pos;           /* DEVICE [T_cap] */
+  float* hidden;            /* DEVICE [T_cap, d] fp32 output */
+  float* residual;          /* DEVICE [T_cap, d] fp32 or NULL */
+  int* err;
+} sp_prefill_io;
+
+SP_API size_t sp_prefill_workspace(const sp_model* m, int T_cap, int max_seqlen_cap);
+SP_API sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* workspace,
+                     size_t workspace_bytes, sp_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* The whole path: select -> compact -> project -> prefill.                  */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+  sp_select_in sel;          /* X and E_text required (H ignored); E_text is also the
+                                text rows of the LM input, so D_text must equal d */
+  int k_cap;                 /* row stride of idx */
+  int* idx;                  /* DEVICE [B, k_cap] */
+  int* count;                /* DEVICE [B] */
+  int* cu_seqlens;           /* DEVICE [B + 1] */
+  float* hidden;             /* DEVICE [T_cap, d] fp32 (T_cap = sp_packed_cap(...)) */
+  int* err;                  /* DEVICE error word or NULL */
+} sp_pipeline_io;
+
+SP_API size_t sp_pipeline_workspace(const sp_selector* s, const sp_model* m, const sp_pipeline_io* io);
+SP_API sp_status sp_pipeline(const sp_selector* s, const sp_model* m, const sp_pipeline_io* io,
+                      void* workspace, size_t workspace_bytes, sp_stream stream);
+
+/*
+ * The same path from HOST buffers: copies X, E_text and stop_bias (HOST, best
+ * pinned) into the workspace, runs sp_pipeline, and copies idx, count,
+ * cu_seqlens and the T_cap hidden rows back into the HOST outputs, all on
+ * `stream`.  The host buffers must stay valid until the stream reaches the end
+ * of the call.  The io's DEVICE pointer fields are ignored; host_* are used.
+ */
+typedef struct {
+  sp_select_in sel;          /* X, E_text, stop_bias are HOST pointers here */
+  int k_cap;
+  int* host_idx;             /* HOST [B, k_cap] */
+  int* host_count;           /* HOST [B] */
+  int* host_cu_seqlens;      /* HOST [B + 1] */
+  float* host_hidden;        /* HOST [T_cap, d] */
+} sp_pipeline_host_io;
+
+SP_API size_t sp_pipeline_host_workspace(const sp_selector* s, const sp_model* m,
+                                  const sp_pipeline_host_io* io);
+SP_API sp_status sp_pipeline_host(const sp_selector* s, const sp_model* m, const sp_pipeline_host_io* io,
+                           void* workspace, size_t workspace_bytes, sp_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* Per-kernel timing (CUDA events recorded around every launch).             */
+/* ------------------------------------------------------------------------ */
+
+typedef enum {
+  SP_K_GEMM = 0, SP_K_SGEMM = 1, SP_K_ATTN = 2, SP_K_NORM = 3, SP_K_SELECT = 4,
+  SP_K_RESTORE = 5, SP_K_COMPACT = 6, SP_K_MISC = 7, SP_K_COUNT = 8
+} sp_kernel_kind;
+
+/* Starts (capacity > 0) or stops (0) recording launch events; host-allocated. */
+SP_API sp_status sp_profile_begin(int capacity);
+/* Synchronises on the recorded events and returns, per sp_kernel_kind, the
+ * summed milliseconds, launch counts and algorithmic flops / bytes. */
+SP_API sp_status sp_profile_end(double* ms, long long* launches, double* flops, double* bytes);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* STEPPRUNE_H */

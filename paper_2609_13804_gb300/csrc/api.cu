@@ -1,0 +1,1070 @@
+// The C ABI of libstepprune (include/stepprune.h): argument validation,
+// workspace carving, tensor-map encoding and the sequencing of the kernels of
+// every stage on the caller's stream.  No entry point allocates device memory
+// except the *_create functions; no entry point synchronises the host except
+// *_create and sp_profile_end.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+
+namespace sp {
+
+// ------------------------------------------------------------------ errors
+
+static thread_local std::string g_last_error;
+
+static sp_status fail(sp_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+static sp_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(SP_ERR_CUDA, "%s: %s (%d)", where, cudaGetErrorString(e), (int)e);
+}
+
+#define SP_CUDA(call, where)                      \
+  do {                                            \
+    cudaError_t e__ = (call);                     \
+    if (e__ != cudaSuccess) return cuda_fail(e__, where); \
+  } while (0)
+
+static bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// ------------------------------------------------------------------ device info
+
+int device_sm_count() {
+  static int cached_dev = -1, cached = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev != cached_dev) {
+    cudaDeviceGetAttribute(&cached, cudaDevAttrMultiProcessorCount, dev);
+    cached_dev = dev;
+  }
+  return cached > 0 ? cached : 1;
+}
+
+static sp_status check_device() {
+  int dev = 0, major = 0, minor = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (major != 10 || minor != 3)
+    return fail(SP_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a only", dev,
+                major, minor);
+  return SP_OK;
+}
+
+// ------------------------------------------------------------------ tensor maps
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
+                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn(std::string* msg) {
+  static EncodeTiledFn fn = nullptr;
+  if (fn) return fn;
+  void* p = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q);
+  if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !p) {
+    if (msg) *msg = "cuTensorMapEncodeTiled is not available from the driver";
+    return nullptr;
+  }
+  fn = reinterpret_cast<EncodeTiledFn>(p);
+  return fn;
+}
+
+bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                      std::string* msg) {
+  EncodeTiledFn fn = encode_fn(msg);
+  if (!fn) return false;
+  if (rows == 0) rows = 1;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) {
+      char b[160];
+      snprintf(b, sizeof(b), "cuTensorMapEncodeTiled failed (%d) for %llux%llu box %u", (int)r,
+               (unsigned long long)rows, (unsigned long long)cols, box_rows);
+      *msg = b;
+    }
+    return false;
+  }
+  return true;
+}
+
+// ------------------------------------------------------------------ profiling
+
+namespace {
+struct Prof {
+  bool on = false;
+  int cap = 0, n = 0;
+  std::vector<cudaEvent_t> ev;
+  std::vector<int> kind;
+  std::vector<double> flops, bytes;
+};
+Prof g_prof;
+}  // namespace
+
+bool prof_enabled() { return g_prof.on; }
+
+void prof_begin_launch(cudaStream_t st) {
+  if (!g_prof.on || g_prof.n >= g_prof.cap) return;
+  cudaEventRecord(g_prof.ev[2 * g_prof.n], st);
+}
+
+void prof_end_launch(cudaStream_t st, int kind, double flops, double bytes) {
+  if (!g_prof.on || g_prof.n >= g_prof.cap) return;
+  cudaEventRecord(g_prof.ev[2 * g_prof.n + 1], st);
+  g_prof.kind[g_prof.n] = kind;
+  g_prof.flops[g_prof.n] = flops;
+  g_prof.bytes[g_prof.n] = bytes;
+  ++g_prof.n;
+}
+
+// ------------------------------------------------------------------ batches
+
+bool fill_batch_desc(BatchDesc* d, int B, const int* n_vis, const int* n_txt, int group_size,
+                     std::string* msg) {
+  if (B < 1 || B > SP_MAX_BATCH) {
+    if (msg) *msg = "B must be in 1..SP_MAX_BATCH";
+    return false;
+  }
+  if (!n_vis || !n_txt) {
+    if (msg) *msg = "n_vis / n_txt are required host arrays";
+    return false;
+  }
+  if (group_size < 0) {
+    if (msg) *msg = "group_size must be >= 0";
+    return false;
+  }
+  memset(d, 0, sizeof(*d));
+  d->B = B;
+  d->group_size = group_size;
+  for (int b = 0; b < B; ++b) {
+    if (n_vis[b] < 1 || n_vis[b] > SP_MAX_NVIS || n_txt[b] < 0) {
+      if (msg) *msg = "n_vis[b] must be in 1..SP_MAX_NVIS and n_txt[b] >= 0";
+      return false;
+    }
+    const int gs = group_size > 0 ? group_size : n_vis[b];
+    d->vis_off[b + 1] = d->vis_off[b] + n_vis[b];
+    d->txt_off[b + 1] = d->txt_off[b] + n_txt[b];
+    d->ep_off[b + 1] = d->ep_off[b] + (n_vis[b] + gs - 1) / gs;
+  }
+  return true;
+}
+
+// Bump allocator over the caller's workspace (256-byte aligned slices).
+struct Carve {
+  char* base;
+  size_t off = 0;
+  explicit Carve(void* p) : base(static_cast<char*>(p)) {}
+  template <class T>
+  T* take(size_t n) {
+    off = (off + 255) & ~size_t(255);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += n * sizeof(T);
+    return p;
+  }
+};
+
+}  // namespace sp
+
+using namespace sp;
+
+// ======================================================================= ABI
+
+struct sp_selector_s {
+  sp_selector_cfg cfg;
+  sp_selector_weights w;
+  float* Wcat1 = nullptr;  // [2h, D]  rows: W_in | Wq_p^T Wk_p / sqrt(h)
+  float* Wcat2 = nullptr;  // [3h, h]  rows: Wq_s / sqrt(h) | Wk_s | Wo_s Wv_s
+  GemmB Wp;
+  GemmB enc_qkv[SP_MAX_ENC_LAYERS], enc_o[SP_MAX_ENC_LAYERS], enc_1[SP_MAX_ENC_LAYERS],
+      enc_2[SP_MAX_ENC_LAYERS];
+};
+
+struct sp_model_s {
+  sp_model_cfg cfg;
+  sp_model_weights w;
+  float2* rope = nullptr;  // [max_pos, head_dim / 2]
+  std::vector<GemmB> qkv, o, gu, down;
+  GemmB p1, p2;
+};
+
+extern "C" {
+
+const char* sp_last_error(void) { return g_last_error.c_str(); }
+int sp_abi_version(void) { return SP_ABI_VERSION; }
+
+sp_status sp_device_error_status(int w) {
+  if (w == 0) return SP_OK;
+  if (w & SP_DEVERR_TIMEOUT) return fail(SP_ERR_TIMEOUT, "a bounded device wait ran out (error word 0x%x)", w);
+  return fail(SP_ERR_DEVICE, "device-side check failed (error word 0x%x)", w);
+}
+
+int sp_num_episodes(int B, const int* n_vis, int group_size) {
+  if (B < 1 || B > SP_MAX_BATCH || !n_vis || group_size < 0) return -1;
+  int e = 0;
+  for (int b = 0; b < B; ++b) {
+    if (n_vis[b] < 1) return -1;
+    const int gs = group_size > 0 ? group_size : n_vis[b];
+    e += (n_vis[b] + gs - 1) / gs;
+  }
+  return e;
+}
+
+int sp_packed_cap(int B, const int* n_vis, const int* n_txt, int k_cap) {
+  if (B < 1 || B > SP_MAX_BATCH || !n_vis || !n_txt || k_cap < 0) return -1;
+  long t = 0;
+  for (int b = 0; b < B; ++b) {
+    if (n_vis[b] < 1 || n_txt[b] < 0) return -1;
+    t += std::min(n_vis[b], k_cap) + n_txt[b];
+  }
+  return t > 0x7fffffff ? -1 : (int)t;
+}
+
+// ------------------------------------------------------------------ selector
+
+sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weights* w, sp_selector** out) {
+  if (!cfg || !w || !out) return fail(SP_ERR_INVALID_ARG, "sp_selector_create: NULL argument");
+  *out = nullptr;
+  sp_status st = check_device();
+  if (st != SP_OK) return st;
+  const sp_selector_cfg c = *cfg;
+  if (c.D <= 0 || c.D % 128 != 0) return fail(SP_ERR_SHAPE, "D must be a positive multiple of 128");
+  if (c.h < 128 || c.h > 1024 || c.h % 128 != 0) return fail(SP_ERR_SHAPE, "h must be a multiple of 128 in 128..1024");
+  if (c.n_enc_layers < 0 || c.n_enc_layers > SP_MAX_ENC_LAYERS) return fail(SP_ERR_SHAPE, "n_enc_layers out of range");
+  if (c.n_enc_layers > 0) {
+    if (c.D_text <= 0 || c.D_text % 64 != 0) return fail(SP_ERR_SHAPE, "D_text must be a multiple of 64");
+    if (c.enc_head_dim != 64 && c.enc_head_dim != 128) return fail(SP_ERR_SHAPE, "enc_head_dim must be 64 or 128");
+    if (c.D % c.enc_head_dim != 0) return fail(SP_ERR_SHAPE, "D must be a multiple of enc_head_dim");
+    if (c.enc_ffn <= 0 || c.enc_ffn % 128 != 0) return fail(SP_ERR_SHAPE, "enc_ffn must be a multiple of 128");
+    if (!w->W_p) return fail(SP_ERR_INVALID_ARG, "W_p is required with an encoder");
+    for (int i = 0; i < c.n_enc_layers; ++i)
+      if (!w->enc_wqkv[i] || !w->enc_wo[i] || !w->enc_w1[i] || !w->enc_w2[i])
+        return fail(SP_ERR_INVALID_ARG, "encoder layer %d weights missing", i);
+  }
+  if (!(c.ln_eps > 0.f)) return fail(SP_ERR_INVALID_ARG, "ln_eps must be > 0");
+  if (!w->s_stop || !w->s_start || !w->W_in || !w->Wq_s || !w->Wk_s || !w->Wv_s || !w->Wo_s || !w->Wq_p || !w->Wk_p)
+    return fail(SP_ERR_INVALID_ARG, "pointer-decoder weights missing");
+
+  sp_selector* s = new (std::nothrow) sp_selector_s();
+  if (!s) return fail(SP_ERR_INVALID_ARG, "out of host memory");
+  s->cfg = c;
+  s->w = *w;
+  const int h = c.h, D = c.D;
+  cudaError_t e = cudaMalloc(&s->Wcat1, (size_t)2 * h * D * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&s->Wcat2, (size_t)3 * h * h * sizeof(float));
+  const float rs = 1.0f / std::sqrt((float)h);
+  if (e == cudaSuccess) e = cudaMemcpy2D(s->Wcat1, D * sizeof(float), w->W_in, D * sizeof(float), D * sizeof(float), h, cudaMemcpyDeviceToDevice);
+  // Wq_p^T Wk_p / sqrt(h): (i, j) = sum_k Wq_p[k, i] Wk_p[k, j]
+  if (e == cudaSuccess) e = fold_matmul(w->Wq_p, 1, h, w->Wk_p, D, 1, s->Wcat1 + (size_t)h * D, D, h, D, h, rs, 0);
+  // Wq_s / sqrt(h), as Wq_s times the identity through the same fold kernel
+  std::vector<float> eye;
+  float* dI = nullptr;
+  if (e == cudaSuccess) {
+    eye.assign((size_t)h * h, 0.f);
+    for (int i = 0; i < h; ++i) eye[(size_t)i * h + i] = 1.f;
+    e = cudaMalloc(&dI, (size_t)h * h * sizeof(float));
+    if (e == cudaSuccess) e = cudaMemcpy(dI, eye.data(), eye.size() * sizeof(float), cudaMemcpyHostToDevice);
+  }
+  if (e == cudaSuccess) e = fold_matmul(w->Wq_s, h, 1, dI, h, 1, s->Wcat2, h, h, h, h, rs, 0);
+  if (e == cudaSuccess) e = cudaMemcpy(s->Wcat2 + (size_t)h * h, w->Wk_s, (size_t)h * h * sizeof(float), cudaMemcpyDeviceToDevice);
+  // Wo_s Wv_s: (i, j) = sum_k Wo_s[i, k] Wv_s[k, j]
+  if (e == cudaSuccess) e = fold_matmul(w->Wo_s, h, 1, w->Wv_s, h, 1, s->Wcat2 + (size_t)2 * h * h, h, h, h, h, 1.f, 0);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (dI) cudaFree(dI);
+  if (e != cudaSuccess) {
+    sp_selector_destroy(s);
+    return cuda_fail(e, "sp_selector_create (fold)");
+  }
+  std::string msg;
+  bool ok = true;
+  if (c.n_enc_layers > 0) {
+    ok = make_gemm_b(&s->Wp, w->W_p, D, c.D_text, &msg);
+    for (int i = 0; ok && i < c.n_enc_layers; ++i) {
+      ok = make_gemm_b(&s->enc_qkv[i], w->enc_wqkv[i], 3 * D, D, &msg) &&
+           make_gemm_b(&s->enc_o[i], w->enc_wo[i], D, D, &msg) &&
+           make_gemm_b(&s->enc_1[i], w->enc_w1[i], c.enc_ffn, D, &msg) &&
+           make_gemm_b(&s->enc_2[i], w->enc_w2[i], D, c.enc_ffn, &msg);
+    }
+  }
+  if (!ok) {
+    sp_selector_destroy(s);
+    return fail(SP_ERR_CUDA, "sp_selector_create: %s", msg.c_str());
+  }
+  *out = s;
+  return SP_OK;
+}
+
+void sp_selector_destroy(sp_selector* s) {
+  if (!s) return;
+  if (s->Wcat1) cudaFree(s->Wcat1);
+  if (s->Wcat2) cudaFree(s->Wcat2);
+  delete s;
+}
+
+namespace {
+
+struct SelPlan {
+  BatchDesc bd;
+  int E = 0, nvis = 0, ntxt = 0, T_enc = 0, max_enc = 0, rows = 0;
+  bool encoder = false;
+};
+
+sp_status plan_select(const sp_selector* s, const sp_select_in* in, SelPlan* p) {
+  if (!s || !in) return fail(SP_ERR_INVALID_ARG, "sp_select: NULL selector or input");
+  std::string msg;
+  if (!fill_batch_desc(&p->bd, in->B, in->n_vis, in->n_txt, in->group_size, &msg))
+    return fail(SP_ERR_SHAPE, "sp_select: %s", msg.c_str());
+  if (in->g < 1 || in->g > 16) return fail(SP_ERR_SHAPE, "g must be in 1..16");
+  if (in->k_max < 1 || in->k_max > SP_MAX_KMAX) return fail(SP_ERR_SHAPE, "k_max must be in 1..SP_MAX_KMAX");
+  p->E = p->bd.ep_off[in->B];
+  p->nvis = p->bd.vis_off[in->B];
+  p->ntxt = p->bd.txt_off[in->B];
+  p->rows = p->nvis + 2;
+  p->encoder = (in->H == nullptr);
+  if (p->encoder && s->cfg.n_enc_layers == 0 && !in->X)
+    return fail(SP_ERR_INVALID_ARG, "sp_select: X is required when H is NULL");
+  p->T_enc = p->nvis + p->ntxt;
+  p->max_enc = 0;
+  for (int b = 0; b < in->B; ++b) p->max_enc = std::max(p->max_enc, in->n_vis[b] + in->n_txt[b]);
+  return SP_OK;
+}
+
+size_t select_ws(const sp_selector* s, const SelPlan& p, const sp_select_out* out, Carve& cv,
+                 void** parts) {
+  const int D = s->cfg.D, h = s->cfg.h, F = s->cfg.enc_ffn;
+  float *P = nullptr, *R = nullptr, *Mall, *ZK, *XL, *QKVs;
+  void *Abf = nullptr, *QKV = nullptr, *O = nullptr, *F1 = nullptr;
+  int* enc_cu = nullptr;
+  if (p.encoder && s->cfg.n_enc_layers > 0) {
+    P = cv.take<float>((size_t)std::max(p.ntxt, 1) * D);
+    R = cv.take<float>((size_t)p.T_enc * D);
+    Abf = cv.take<uint16_t>((size_t)p.T_enc * D);
+    QKV = cv.take<uint16_t>((size_t)p.T_enc * 3 * D);
+    O = cv.take<uint16_t>((size_t)p.T_enc * D);
+    F1 = cv.take<uint16_t>((size_t)p.T_enc * F);
+    enc_cu = cv.take<int>(SP_MAX_BATCH + 1);
+  } else if (p.encoder) {
+    R = cv.take<float>((size_t)p.T_enc * D);
+  }
+  Mall = cv.take<float>((size_t)p.rows * D);
+  ZK = cv.take<float>((size_t)p.rows * 2 * h);
+  XL = cv.take<float>((size_t)p.rows * h);
+  QKVs = cv.take<float>((size_t)p.rows * 3 * h);
+  int* order = (out && out->order) ? nullptr : cv.take<int>((size_t)p.E * SP_MAX_KMAX);
+  int* epc = (out && out->ep_count) ? nullptr : cv.take<int>((size_t)p.E);
+  if (parts) {
+    parts[0] = P; parts[1] = R; parts[2] = Abf; parts[3] = QKV; parts[4] = O; parts[5] = F1;
+    parts[6] = enc_cu; parts[7] = Mall; parts[8] = ZK; parts[9] = XL; parts[10] = QKVs;
+    parts[11] = order; parts[12] = epc;
+  }
+  return cv.off;
+}
+
+// Runs the encoder stack (Eq. 3) on X / E_text into R (fp32 residual rows).
+sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPlan& p, void** parts,
+                      int* err, cudaStream_t st) {
+  const sp_selector_cfg& c = s->cfg;
+  const int D = c.D;
+  float* P = (float*)parts[0];
+  float* R = (float*)parts[1];
+  void* Abf = parts[2];
+  void* QKV = parts[3];
+  void* O = parts[4];
+  void* F1 = parts[5];
+  int* enc_cu = (int*)parts[6];
+  std::string msg;
+  if (p.ntxt > 0) {
+    CUtensorMap tE;
+    if (!encode_tmap_bf16(&tE, in->E_text, p.ntxt, c.D_text, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
+    GemmEpi ep;
+    ep.kind = EPI_F32;
+    ep.out = P;
+    ep.ldo = D;
+    SP_CUDA(gemm_bf16(tE, p.ntxt, nullptr, s->Wp, D, ep, err, st), "text projection");
+  }
+  SP_CUDA(assemble_encoder_input(p.bd, in->X, P, D, s->w.ln_text_g, s->w.ln_text_b, c.ln_eps, c.g_text, R,
+                                 p.T_enc, st), "encoder input");
+  SP_CUDA(write_enc_cu(p.bd, enc_cu, st), "encoder offsets");
+  CUtensorMap tA, tO, tF;
+  if (!encode_tmap_bf16(&tA, Abf, p.T_enc, D, 128, &msg) || !encode_tmap_bf16(&tO, O, p.T_enc, D, 128, &msg) ||
+      !encode_tmap_bf16(&tF, F1, p.T_enc, c.enc_ffn, 128, &msg))
+    return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  const int nh = D / c.enc_head_dim;
+  for (int l = 0; l < c.n_enc_layers; ++l) {
+    SP_CUDA(layernorm_f32(R, D, s->w.enc_ln1_g[l], s->w.enc_ln1_b[l], nullptr, Abf, D, p.T_enc, D, c.ln_eps, 1.f, st), "enc ln1");
+    GemmEpi e1;
+    e1.kind = EPI_BF16;
+    e1.out = QKV;
+    e1.ldo = 3 * D;
+    SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_qkv[l], 3 * D, e1, err, st), "enc qkv");
+    SP_CUDA(attention_varlen(QKV, O, enc_cu, in->B, p.max_enc, nh, nh, c.enc_head_dim, false, st), "enc attention");
+    GemmEpi e2;
+    e2.kind = EPI_F32_ACC;
+    e2.out = R;
+    e2.ldo = D;
+    SP_CUDA(gemm_bf16(tO, p.T_enc, nullptr, s->enc_o[l], D, e2, err, st), "enc o");
+    SP_CUDA(layernorm_f32(R, D, s->w.enc_ln2_g[l], s->w.enc_ln2_b[l], nullptr, Abf, D, p.T_enc, D, c.ln_eps, 1.f, st), "enc ln2");
+    GemmEpi e3;
+    e3.kind = EPI_GELU_BF16;
+    e3.out = F1;
+    e3.ldo = c.enc_ffn;
+    SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_1[l], c.enc_ffn, e3, err, st), "enc fc1");
+    SP_CUDA(gemm_bf16(tF, p.T_enc, nullptr, s->enc_2[l], D, e2, err, st), "enc fc2");
+  }
+  return SP_OK;
+}
+
+}  // namespace
+
+size_t sp_select_workspace(const sp_selector* s, const sp_select_in* in) {
+  SelPlan p;
+  if (plan_select(s, in, &p) != SP_OK) return 0;
+  Carve cv(nullptr);
+  return select_ws(s, p, nullptr, cv, nullptr) + 256;
+}
+
+static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const sp_select_out* out, void* ws,
+                             size_t ws_bytes, cudaStream_t st) {
+  SelPlan p;
+  sp_status rs = plan_select(s, in, &p);
+  if (rs != SP_OK) return rs;
+  if (!out || !out->idx || !out->count) return fail(SP_ERR_INVALID_ARG, "sp_select: idx and count are required");
+  if (!in->stop_bias) return fail(SP_ERR_INVALID_ARG, "sp_select: stop_bias is required");
+  if (p.encoder && (!in->X || (p.ntxt > 0 && s->cfg.n_enc_layers > 0 && !in->E_text)))
+    return fail(SP_ERR_INVALID_ARG, "sp_select: X / E_text required when H is NULL");
+  if ((in->X && !al16(in->X)) || (in->E_text && !al16(in->E_text)) || (in->H && !al16(in->H)))
+    return fail(SP_ERR_ALIGN, "sp_select: inputs must be 16-byte aligned");
+  int need_cap = 0;
+  for (int b = 0; b < in->B; ++b) {
+    const int n = in->n_vis[b], gs = in->group_size > 0 ? in->group_size : n;
+    int c = 0;
+    for (int s0 = 0; s0 < n; s0 += gs) c += std::min(in->k_max, std::min(gs, n - s0));
+    need_cap = std::max(need_cap, c);
+  }
+  if (out->k_cap < need_cap) return fail(SP_ERR_SHAPE, "sp_select: k_cap %d < largest possible count %d", out->k_cap, need_cap);
+  Carve cv(ws);
+  void* parts[13];
+  const size_t need = select_ws(s, p, out, cv, parts) + 256;
+  if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_select: workspace %zu < %zu bytes", ws_bytes, need);
+  if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_select: workspace must be 16-byte aligned");
+  int* err = out->err;
+  const int D = s->cfg.D, h = s->cfg.h;
+
+  if (p.encoder && s->cfg.n_enc_layers > 0) {
+    rs = run_encoder(s, in, p, parts, err, st);
+    if (rs != SP_OK) return rs;
+    SP_CUDA(gather_memory(p.bd, (float*)parts[1], nullptr, s->w.s_stop, s->w.s_start, (float*)parts[7], D, st), "memory");
+  } else if (p.encoder) {
+    // no encoder blocks: H = X (converted to fp32)
+    SP_CUDA(bf16_to_f32(in->X, (float*)parts[1], p.nvis, nullptr, D, st), "X to fp32");
+    BatchDesc flat = p.bd;
+    for (int b = 0; b <= in->B; ++b) flat.txt_off[b] = 0;
+    SP_CUDA(gather_memory(flat, (float*)parts[1], nullptr, s->w.s_stop, s->w.s_start, (float*)parts[7], D, st), "memory");
+  } else {
+    SP_CUDA(gather_memory(p.bd, nullptr, in->H, s->w.s_stop, s->w.s_start, (float*)parts[7], D, st), "memory");
+  }
+  float* Mall = (float*)parts[7];
+  if (out->memory)
+    SP_CUDA(cudaMemcpyAsync(out->memory, Mall, (size_t)p.nvis * D * sizeof(float), cudaMemcpyDeviceToDevice, st),
+            "memory copy");
+  float* ZK = (float*)parts[8];
+  float* XL = (float*)parts[9];
+  float* QKVs = (float*)parts[10];
+  // candidate precompute (fp32): [z | KT] = M [W_in; Wq_p^T Wk_p / sqrt h]^T, x = LN1(z),
+  // [QS | KS | VT] = x [Wq_s / sqrt h; Wk_s; Wo_s Wv_s]^T
+  SP_CUDA(sgemm_f32(Mall, D, s->Wcat1, D, ZK, 2 * h, p.rows, 2 * h, D, st), "precompute 1");
+  SP_CUDA(layernorm_f32(ZK, 2 * h, s->w.ln1_g, s->w.ln1_b, XL, nullptr, h, p.rows, h, s->cfg.ln_eps, 1.f, st), "ln1");
+  SP_CUDA(sgemm_f32(XL, h, s->Wcat2, h, QKVs, 3 * h, p.rows, 3 * h, h, st), "precompute 2");
+
+  SelectArgs a;
+  a.Z = ZK; a.ldz = 2 * h;
+  a.KT = ZK + h; a.ldkt = 2 * h;
+  a.QS = QKVs; a.ldqs = 3 * h;
+  a.KS = QKVs + h; a.ldks = 3 * h;
+  a.VT = QKVs + 2 * h; a.ldvt = 3 * h;
+  a.ln2_g = s->w.ln2_g; a.ln2_b = s->w.ln2_b;
+  a.ln_eps = s->cfg.ln_eps;
+  a.stop_row = p.nvis;
+  a.start_row = p.nvis + 1;
+  a.stop_bias = in->stop_bias;
+  a.h = h; a.k_max = in->k_max; a.g = in->g;
+  a.order = out->order ? out->order : (int*)parts[11];
+  a.ep_count = out->ep_count ? out->ep_count : (int*)parts[12];
+  a.margin = out->margin; a.gap = out->gap; a.rounds = out->rounds;
+  a.err = err;
+  bool keys_smem = true;
+  size_t smem = 0;
+  const int C = select_cluster_size(p.bd, h, &keys_smem, &smem);
+  SP_CUDA(select_launch(p.bd, p.E, a, C, keys_smem, smem, st), "selection");
+  SP_CUDA(restore_launch(p.bd, a.order, a.ep_count, in->k_max, out->idx, out->k_cap, out->count, err, st), "restore");
+  return SP_OK;
+}
+
+sp_status sp_select(const sp_selector* s, const sp_select_in* in, const sp_select_out* out, void* ws,
+                    size_t ws_bytes, sp_stream stream) {
+  return select_impl(s, in, out, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ compaction
+
+static sp_status compact_impl(const sp_compact_in* in, const sp_compact_out* out, cudaStream_t st) {
+  if (!in || !out) return fail(SP_ERR_INVALID_ARG, "sp_compact: NULL argument");
+  BatchDesc bd;
+  std::string msg;
+  if (!fill_batch_desc(&bd, in->B, in->n_vis, in->n_txt, 0, &msg)) return fail(SP_ERR_SHAPE, "sp_compact: %s", msg.c_str());
+  if (!in->X || !in->idx || !in->count || !out->packed || !out->cu_seqlens || !out->pos)
+    return fail(SP_ERR_INVALID_ARG, "sp_compact: X, idx, count, packed, cu_seqlens, pos are required");
+  if (bd.txt_off[in->B] > 0 && !in->text) return fail(SP_ERR_INVALID_ARG, "sp_compact: text is required");
+  if (in->W_vis <= 0 || in->W_vis % 8 || in->W_txt <= 0 || in->W_txt % 8)
+    return fail(SP_ERR_SHAPE, "sp_compact: W_vis and W_txt must be positive multiples of 8");
+  if (in->k_cap < 0) return fail(SP_ERR_SHAPE, "sp_compact: k_cap must be >= 0");
+  const bool direct = out->vis_packed == nullptr;
+  if (direct && in->W_vis != in->W_txt) return fail(SP_ERR_SHAPE, "sp_compact: direct mode needs W_vis == W_txt");
+  if (!direct && (!out->vis_row_map || !out->vis_cu)) return fail(SP_ERR_INVALID_ARG, "sp_compact: vis_row_map and vis_cu required with vis_packed");
+  if (!al16(in->X) || (in->text && !al16(in->text)) || !al16(out->packed) || (out->vis_packed && !al16(out->vis_packed)))
+    return fail(SP_ERR_ALIGN, "sp_compact: row buffers must be 16-byte aligned");
+  const int T_cap = sp_packed_cap(in->B, in->n_vis, in->n_txt, in->k_cap);
+  SP_CUDA(compact_launch(bd, in->X, in->W_vis, in->text, in->W_txt, in->idx, in->k_cap, in->count, out->packed,
+                         out->cu_seqlens, out->pos, out->vis_packed, out->vis_row_map, out->vis_cu, T_cap, out->err, st),
+          "compaction");
+  return SP_OK;
+}
+
+sp_status sp_compact(const sp_compact_in* in, const sp_compact_out* out, sp_stream stream) {
+  return compact_impl(in, out, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ model
+
+sp_status sp_model_create(const sp_model_cfg* cfg, const sp_model_weights* w, sp_model** out) {
+  if (!cfg || !w || !out) return fail(SP_ERR_INVALID_ARG, "sp_model_create: NULL argument");
+  *out = nullptr;
+  sp_status st = check_device();
+  if (st != SP_OK) return st;
+  const sp_model_cfg c = *cfg;
+  if (c.n_layers < 1 || c.n_layers > SP_MAX_LM_LAYERS) return fail(SP_ERR_SHAPE, "n_layers out of range");
+  if (c.d <= 0 || c.d % 128) return fail(SP_ERR_SHAPE, "d must be a multiple of 128");
+  if (c.head_dim != 64 && c.head_dim != 128) return fail(SP_ERR_SHAPE, "head_dim must be 64 or 128");
+  if (c.n_heads < 1 || c.n_kv_heads < 1 || c.n_heads % c.n_kv_heads) return fail(SP_ERR_SHAPE, "n_kv_heads must divide n_heads");
+  const int qkv = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim;
+  if (qkv % 256) return fail(SP_ERR_SHAPE, "(n_heads + 2 n_kv_heads) head_dim must be a multiple of 256");
+  if ((c.n_heads * c.head_dim) % 128) return fail(SP_ERR_SHAPE, "n_heads head_dim must be a multiple of 128");
+  if (c.ffn <= 0 || c.ffn % 128) return fail(SP_ERR_SHAPE, "ffn must be a multiple of 128");
+  if (c.max_pos < 1 || c.max_pos > (1 << 20)) return fail(SP_ERR_SHAPE, "max_pos out of range");
+  if (!(c.rope_theta > 0.f) || !(c.rms_eps > 0.f)) return fail(SP_ERR_INVALID_ARG, "rope_theta and rms_eps must be > 0");
+  if (c.proj_kind < SP_PROJ_NONE || c.proj_kind > SP_PROJ_MLP2_GELU) return fail(SP_ERR_INVALID_ARG, "bad proj_kind");
+  if (c.proj_kind != SP_PROJ_NONE) {
+    if (c.proj_in <= 0 || c.proj_in % 64) return fail(SP_ERR_SHAPE, "proj_in must be a multiple of 64");
+    if (!w->proj_w1) return fail(SP_ERR_INVALID_ARG, "proj_w1 required");
+    if (c.proj_kind == SP_PROJ_MLP2_GELU) {
+      if (c.proj_hidden <= 0 || c.proj_hidden % 128) return fail(SP_ERR_SHAPE, "proj_hidden must be a multiple of 128");
+      if (!w->proj_w2) return fail(SP_ERR_INVALID_ARG, "proj_w2 required");
+    }
+  }
+  for (int l = 0; l < c.n_layers; ++l)
+    if (!w->wqkv[l] || !w->wo[l] || !w->wgu[l] || !w->wdown[l]) return fail(SP_ERR_INVALID_ARG, "layer %d weights missing", l);
+
+  sp_model* m = new (std::nothrow) sp_model_s();
+  if (!m) return fail(SP_ERR_INVALID_ARG, "out of host memory");
+  m->cfg = c;
+  m->w = *w;
+  // rotary table: angle = pos * theta^(-2i/dh), in double, stored as fp32 (cos, sin)
+  const int half = c.head_dim / 2;
+  std::vector<float2> tab((size_t)c.max_pos * half);
+  for (int p = 0; p < c.max_pos; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double inv = std::pow((double)c.rope_theta, -(2.0 * i) / (double)c.head_dim);
+      const double ang = (double)p * inv;
+      tab[(size_t)p * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+    }
+  cudaError_t e = cudaMalloc(&m->rope, tab.size() * sizeof(float2));
+  if (e == cudaSuccess) e = cudaMemcpy(m->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    sp_model_destroy(m);
+    return cuda_fail(e, "sp_model_create (rope table)");
+  }
+  std::string msg;
+  bool ok = true;
+  m->qkv.resize(c.n_layers);
+  m->o.resize(c.n_layers);
+  m->gu.resize(c.n_layers);
+  m->down.resize(c.n_layers);
+  for (int l = 0; ok && l < c.n_layers; ++l) {
+    ok = make_gemm_b(&m->qkv[l], w->wqkv[l], qkv, c.d, &msg) &&
+         make_gemm_b(&m->o[l], w->wo[l], c.d, c.n_heads * c.head_dim, &msg) &&
+         make_gemm_b(&m->gu[l], w->wgu[l], 2 * c.ffn, c.d, &msg) &&
+         make_gemm_b(&m->down[l], w->wdown[l], c.d, c.ffn, &msg);
+  }
+  if (ok && c.proj_kind == SP_PROJ_LINEAR) ok = make_gemm_b(&m->p1, w->proj_w1, c.d, c.proj_in, &msg);
+  if (ok && c.proj_kind == SP_PROJ_MLP2_GELU)
+    ok = make_gemm_b(&m->p1, w->proj_w1, c.proj_hidden, c.proj_in, &msg) &&
+         make_gemm_b(&m->p2, w->proj_w2, c.d, c.proj_hidden, &msg);
+  if (!ok) {
+    sp_model_destroy(m);
+    return fail(SP_ERR_CUDA, "sp_model_create: %s", msg.c_str());
+  }
+  *out = m;
+  return SP_OK;
+}
+
+void sp_model_destroy(sp_model* m) {
+  if (!m) return;
+  if (m->rope) cudaFree(m->rope);
+  delete m;
+}
+
+// ------------------------------------------------------------------ projector
+
+static size_t project_ws(const sp_model* m, int rows_cap, Carve& cv, void** tmp) {
+  void* t = nullptr;
+  if (m->cfg.proj_kind == SP_PROJ_MLP2_GELU) t = cv.take<uint16_t>((size_t)std::max(rows_cap, 1) * m->cfg.proj_hidden);
+  if (tmp) *tmp = t;
+  return cv.off;
+}
+
+size_t sp_project_workspace(const sp_model* m, int rows_cap) {
+  if (!m || rows_cap < 0) return 0;
+  Carve cv(nullptr);
+  return project_ws(m, rows_cap, cv, nullptr) + 256;
+}
+
+static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* ws, size_t ws_bytes, cudaStream_t st) {
+  if (!m || !io) return fail(SP_ERR_INVALID_ARG, "sp_project: NULL argument");
+  const sp_model_cfg& c = m->cfg;
+  if (c.proj_kind == SP_PROJ_NONE) return SP_OK;
+  if (io->B < 1 || io->B > SP_MAX_BATCH || io->rows_cap < 0) return fail(SP_ERR_SHAPE, "sp_project: bad B / rows_cap");
+  if (!io->vis_packed || !io->vis_row_map || !io->vis_cu || !io->packed)
+    return fail(SP_ERR_INVALID_ARG, "sp_project: vis_packed, vis_row_map, vis_cu and packed are required");
+  if (!al16(io->vis_packed) || !al16(io->packed)) return fail(SP_ERR_ALIGN, "sp_project: buffers must be 16-byte aligned");
+  if (io->rows_cap == 0) return SP_OK;
+  Carve cv(ws);
+  void* tmp = nullptr;
+  const size_t need = project_ws(m, io->rows_cap, cv, &tmp) + 256;
+  if (c.proj_kind == SP_PROJ_MLP2_GELU && (!ws || ws_bytes < need))
+    return fail(SP_ERR_WORKSPACE, "sp_project: workspace %zu < %zu bytes", ws_bytes, need);
+  std::string msg;
+  CUtensorMap tV;
+  if (!encode_tmap_bf16(&tV, io->vis_packed, io->rows_cap, c.proj_in, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  const int* M_dev = io->vis_cu + io->B;
+  GemmEpi sc;
+  sc.kind = EPI_SCATTER_BF16;
+  sc.out = io->packed;
+  sc.ldo = c.d;
+  sc.row_map = io->vis_row_map;
+  if (c.proj_kind == SP_PROJ_LINEAR) {
+    SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.d, sc, io->err, st), "projector");
+    return SP_OK;
+  }
+  GemmEpi g1;
+  g1.kind = EPI_GELU_BF16;
+  g1.out = tmp;
+  g1.ldo = c.proj_hidden;
+  SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.proj_hidden, g1, io->err, st), "projector fc1");
+  CUtensorMap tT;
+  if (!encode_tmap_bf16(&tT, tmp, io->rows_cap, c.proj_hidden, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  SP_CUDA(gemm_bf16(tT, io->rows_cap, M_dev, m->p2, c.d, sc, io->err, st), "projector fc2");
+  return SP_OK;
+}
+
+sp_status sp_project(const sp_model* m, const sp_project_io* io, void* ws, size_t ws_bytes, sp_stream stream) {
+  return project_impl(m, io, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ prefill
+
+struct PrefillParts {
+  float* h32;
+  void *xb, *qkv, *ob, *act;
+};
+
+static size_t prefill_ws(const sp_model* m, int T_cap, bool own_residual, Carve& cv, PrefillParts* p) {
+  const sp_model_cfg& c = m->cfg;
+  const size_t T = (size_t)std::max(T_cap, 1);
+  PrefillParts q;
+  q.h32 = own_residual ? cv.take<float>(T * c.d) : nullptr;
+  q.xb = cv.take<uint16_t>(T * c.d);
+  q.qkv = cv.take<uint16_t>(T * (c.n_heads + 2 * c.n_kv_heads) * c.head_dim);
+  q.ob = cv.take<uint16_t>(T * c.n_heads * c.head_dim);
+  q.act = cv.take<uint16_t>(T * c.ffn);
+  if (p) *p = q;
+  return cv.off;
+}
+
+size_t sp_prefill_workspace(const sp_model* m, int T_cap, int max_seqlen_cap) {
+  if (!m || T_cap < 0 || max_seqlen_cap < 0) return 0;
+  Carve cv(nullptr);
+  return prefill_ws(m, T_cap, true, cv, nullptr) + 256;
+}
+
+static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* ws, size_t ws_bytes, cudaStream_t st) {
+  if (!m || !io) return fail(SP_ERR_INVALID_ARG, "sp_prefill: NULL argument");
+  const sp_model_cfg& c = m->cfg;
+  if (io->B < 1 || io->B > SP_MAX_BATCH || io->T_cap < 0 || io->max_seqlen_cap < 0)
+    return fail(SP_ERR_SHAPE, "sp_prefill: bad B / T_cap / max_seqlen_cap");
+  if (io->max_seqlen_cap > c.max_pos) return fail(SP_ERR_SHAPE, "sp_prefill: max_seqlen_cap %d > max_pos %d", io->max_seqlen_cap, c.max_pos);
+  if (!io->x || !io->cu_seqlens || !io->pos || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_prefill: x, cu_seqlens, pos, hidden required");
+  if (!al16(io->x) || !al16(io->hidden) || (io->residual && !al16(io->residual)))
+    return fail(SP_ERR_ALIGN, "sp_prefill: buffers must be 16-byte aligned");
+  if (io->T_cap == 0) return SP_OK;
+  Carve cv(ws);
+  PrefillParts p;
+  const size_t need = prefill_ws(m, io->T_cap, io->residual == nullptr, cv, &p) + 256;
+  if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_prefill: workspace %zu < %zu bytes", ws_bytes, need);
+  if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_prefill: workspace must be 16-byte aligned");
+  float* h32 = io->residual ? io->residual : p.h32;
+  const int T_cap = io->T_cap;
+  const int* T_dev = io->cu_seqlens + io->B;
+  const int dq = c.n_heads * c.head_dim, qkvw = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim;
+  std::string msg;
+  CUtensorMap tX, tO, tA;
+  if (!encode_tmap_bf16(&tX, p.xb, T_cap, c.d, 128, &msg) || !encode_tmap_bf16(&tO, p.ob, T_cap, dq, 128, &msg) ||
+      !encode_tmap_bf16(&tA, p.act, T_cap, c.ffn, 128, &msg))
+    return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  SP_CUDA(bf16_to_f32(io->x, h32, T_cap, T_dev, c.d, st), "embed");
+  for (int l = 0; l < c.n_layers; ++l) {
+    SP_CUDA(rmsnorm_f32_to_bf16(h32, m->w.attn_norm[l], p.xb, T_cap, T_dev, c.d, c.rms_eps, st), "attn norm");
+    GemmEpi eq;
+    eq.kind = EPI_BF16_ROPE;
+    eq.out = p.qkv;
+    eq.ldo = qkvw;
+    eq.rope = m->rope;
+    eq.pos = io->pos;
+    eq.max_pos = c.max_pos;
+    eq.head_dim = c.head_dim;
+    eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
+    SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->qkv[l], qkvw, eq, io->err, st), "qkv");
+    SP_CUDA(attention_varlen(p.qkv, p.ob, io->cu_seqlens, io->B, io->max_seqlen_cap, c.n_heads, c.n_kv_heads,
+                             c.head_dim, true, st), "attention");
+    GemmEpi er;
+    er.kind = EPI_F32_ACC;
+    er.out = h32;
+    er.ldo = c.d;
+    SP_CUDA(gemm_bf16(tO, T_cap, T_dev, m->o[l], c.d, er, io->err, st), "o");
+    SP_CUDA(rmsnorm_f32_to_bf16(h32, m->w.mlp_norm[l], p.xb, T_cap, T_dev, c.d, c.rms_eps, st), "mlp norm");
+    GemmEpi eg;
+    eg.kind = EPI_SWIGLU_BF16;
+    eg.out = p.act;
+    eg.ldo = c.ffn;
+    eg.up_off = c.ffn;
+    SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->gu[l], 2 * c.ffn, eg, io->err, st), "gate/up");
+    SP_CUDA(gemm_bf16(tA, T_cap, T_dev, m->down[l], c.d, er, io->err, st), "down");
+  }
+  SP_CUDA(rmsnorm_f32_to_f32(h32, m->w.final_norm, io->hidden, T_cap, T_dev, c.d, c.rms_eps, st), "final norm");
+  return SP_OK;
+}
+
+sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* ws, size_t ws_bytes, sp_stream stream) {
+  return prefill_impl(m, io, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ pipeline
+
+namespace {
+struct PipePlan {
+  int T_cap = 0, max_len = 0, rows_cap = 0;
+};
+
+sp_status plan_pipe(const sp_selector* s, const sp_model* m, const sp_select_in& sel, int k_cap, PipePlan* p) {
+  if (!s || !m) return fail(SP_ERR_INVALID_ARG, "sp_pipeline: NULL handle");
+  if (sel.B < 1 || sel.B > SP_MAX_BATCH || !sel.n_vis || !sel.n_txt) return fail(SP_ERR_SHAPE, "sp_pipeline: bad batch");
+  if (s->cfg.D_text != m->cfg.d) return fail(SP_ERR_SHAPE, "sp_pipeline: D_text must equal the LM width d");
+  if (m->cfg.proj_kind == SP_PROJ_NONE ? s->cfg.D != m->cfg.d : s->cfg.D != m->cfg.proj_in)
+    return fail(SP_ERR_SHAPE, "sp_pipeline: visual width does not match the projector input");
+  p->T_cap = sp_packed_cap(sel.B, sel.n_vis, sel.n_txt, k_cap);
+  if (p->T_cap < 0) return fail(SP_ERR_SHAPE, "sp_pipeline: bad sizes");
+  p->max_len = 0;
+  p->rows_cap = 0;
+  for (int b = 0; b < sel.B; ++b) {
+    p->max_len = std::max(p->max_len, std::min(sel.n_vis[b], k_cap) + sel.n_txt[b]);
+    p->rows_cap += std::min(sel.n_vis[b], k_cap);
+  }
+  if (p->max_len > m->cfg.max_pos) return fail(SP_ERR_SHAPE, "sp_pipeline: a sequence can exceed max_pos");
+  return SP_OK;
+}
+
+struct PipeParts {
+  void* packed;
+  int* pos;
+  void* vis_packed;
+  int* vis_row_map;
+  int* vis_cu;
+  void* scratch;
+  size_t scratch_bytes;
+};
+
+size_t pipe_ws(const sp_selector* s, const sp_model* m, const sp_select_in& sel, const PipePlan& pp, Carve& cv,
+               PipeParts* out) {
+  PipeParts q;
+  q.packed = cv.take<uint16_t>((size_t)std::max(pp.T_cap, 1) * m->cfg.d);
+  q.pos = cv.take<int>((size_t)std::max(pp.T_cap, 1));
+  const bool proj = m->cfg.proj_kind != SP_PROJ_NONE;
+  q.vis_packed = proj ? cv.take<uint16_t>((size_t)std::max(pp.rows_cap, 1) * s->cfg.D) : nullptr;
+  q.vis_row_map = proj ? cv.take<int>((size_t)std::max(pp.rows_cap, 1)) : nullptr;
+  q.vis_cu = proj ? cv.take<int>(SP_MAX_BATCH + 1) : nullptr;
+  SelPlan sp_;
+  sp_select_in si = sel;
+  si.H = nullptr;
+  plan_select(s, &si, &sp_);
+  Carve c1(nullptr), c2(nullptr), c3(nullptr);
+  sp_select_out so = {};
+  so.order = nullptr;
+  so.ep_count = nullptr;
+  const size_t a = select_ws(s, sp_, &so, c1, nullptr);
+  const size_t b = project_ws(m, pp.rows_cap, c2, nullptr);
+  const size_t c = prefill_ws(m, pp.T_cap, true, c3, nullptr);
+  q.scratch_bytes = std::max(a, std::max(b, c)) + 256;
+  q.scratch = cv.take<char>(q.scratch_bytes);
+  if (out) *out = q;
+  return cv.off;
+}
+}  // namespace
+
+size_t sp_pipeline_workspace(const sp_selector* s, const sp_model* m, const sp_pipeline_io* io) {
+  if (!io) return 0;
+  PipePlan pp;
+  if (plan_pipe(s, m, io->sel, io->k_cap, &pp) != SP_OK) return 0;
+  SelPlan tmp;
+  sp_select_in si = io->sel;
+  si.H = nullptr;
+  if (plan_select(s, &si, &tmp) != SP_OK) return 0;
+  Carve cv(nullptr);
+  return pipe_ws(s, m, io->sel, pp, cv, nullptr) + 256;
+}
+
+static sp_status pipeline_impl(const sp_selector* s, const sp_model* m, const sp_pipeline_io* io, void* ws,
+                               size_t ws_bytes, cudaStream_t st) {
+  if (!io) return fail(SP_ERR_INVALID_ARG, "sp_pipeline: NULL io");
+  PipePlan pp;
+  sp_status r = plan_pipe(s, m, io->sel, io->k_cap, &pp);
+  if (r != SP_OK) return r;
+  if (!io->idx || !io->count || !io->cu_seqlens || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_pipeline: idx, count, cu_seqlens, hidden required");
+  Carve cv(ws);
+  PipeParts q;
+  const size_t need = pipe_ws(s, m, io->sel, pp, cv, &q) + 256;
+  if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_pipeline: workspace %zu < %zu bytes", ws_bytes, need);
+  if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_pipeline: workspace must be 16-byte aligned");
+
+  sp_select_in si = io->sel;
+  si.H = nullptr;
+  sp_select_out so = {};
+  so.idx = io->idx;
+  so.k_cap = io->k_cap;
+  so.count = io->count;
+  so.err = io->err;
+  r = select_impl(s, &si, &so, q.scratch, q.scratch_bytes, st);
+  if (r != SP_OK) return r;
+
+  const bool proj = m->cfg.proj_kind != SP_PROJ_NONE;
+  sp_compact_in ci = {};
+  ci.B = si.B;
+  ci.n_vis = si.n_vis;
+  ci.n_txt = si.n_txt;
+  ci.X = si.X;
+  ci.W_vis = s->cfg.D;
+  ci.text = si.E_text;
+  ci.W_txt = m->cfg.d;
+  ci.idx = io->idx;
+  ci.k_cap = io->k_cap;
+  ci.count = io->count;
+  sp_compact_out co = {};
+  co.packed = q.packed;
+  co.cu_seqlens = io->cu_seqlens;
+  co.pos = q.pos;
+  co.vis_packed = q.vis_packed;
+  co.vis_row_map = q.vis_row_map;
+  co.vis_cu = q.vis_cu;
+  co.err = io->err;
+  r = compact_impl(&ci, &co, st);
+  if (r != SP_OK) return r;
+  if (proj) {
+    sp_project_io pj = {};
+    pj.B = si.B;
+    pj.rows_cap = pp.rows_cap;
+    pj.vis_packed = q.vis_packed;
+    pj.vis_row_map = q.vis_row_map;
+    pj.vis_cu = q.vis_cu;
+    pj.packed = q.packed;
+    pj.err = io->err;
+    r = project_impl(m, &pj, q.scratch, q.scratch_bytes, st);
+    if (r != SP_OK) return r;
+  }
+  sp_prefill_io pf = {};
+  pf.B = si.B;
+  pf.T_cap = pp.T_cap;
+  pf.max_seqlen_cap = pp.max_len;
+  pf.x = q.packed;
+  pf.cu_seqlens = io->cu_seqlens;
+  pf.pos = q.pos;
+  pf.hidden = io->hidden;
+  pf.residual = nullptr;
+  pf.err = io->err;
+  return prefill_impl(m, &pf, q.scratch, q.scratch_bytes, st);
+}
+
+sp_status sp_pipeline(const sp_selector* s, const sp_model* m, const sp_pipeline_io* io, void* ws, size_t ws_bytes,
+                      sp_stream stream) {
+  return pipeline_impl(s, m, io, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ pipeline from host buffers
+
+namespace {
+struct HostParts {
+  void* X;
+  void* E;
+  float* bias;
+  int* idx;
+  int* count;
+  int* cu;
+  float* hidden;
+  int* err;
+  void* inner;
+};
+
+size_t host_ws(const sp_selector* s, const sp_model* m, const sp_pipeline_host_io* io, const PipePlan& pp, Carve& cv,
+               HostParts* out, size_t* inner_bytes) {
+  const sp_select_in& sel = io->sel;
+  int nvis = 0, ntxt = 0;
+  for (int b = 0; b < sel.B; ++b) { nvis += sel.n_vis[b]; ntxt += sel.n_txt[b]; }
+  const int E = sp_num_episodes(sel.B, sel.n_vis, sel.group_size);
+  HostParts q;
+  q.X = cv.take<uint16_t>((size_t)nvis * s->cfg.D);
+  q.E = cv.take<uint16_t>((size_t)std::max(ntxt, 1) * s->cfg.D_text);
+  q.bias = cv.take<float>((size_t)std::max(E, 1));
+  q.idx = cv.take<int>((size_t)sel.B * io->k_cap);
+  q.count = cv.take<int>(sel.B);
+  q.cu = cv.take<int>(sel.B + 1);
+  q.hidden = cv.take<float>((size_t)std::max(pp.T_cap, 1) * m->cfg.d);
+  q.err = cv.take<int>(4);
+  Carve c2(nullptr);
+  const size_t ib = pipe_ws(s, m, sel, pp, c2, nullptr) + 256;
+  q.inner = cv.take<char>(ib);
+  if (out) *out = q;
+  if (inner_bytes) *inner_bytes = ib;
+  return cv.off;
+}
+}  // namespace
+
+size_t sp_pipeline_host_workspace(const sp_selector* s, const sp_model* m, const sp_pipeline_host_io* io) {
+  if (!io) return 0;
+  PipePlan pp;
+  if (plan_pipe(s, m, io->sel, io->k_cap, &pp) != SP_OK) return 0;
+  if (sp_num_episodes(io->sel.B, io->sel.n_vis, io->sel.group_size) < 0) return 0;
+  Carve cv(nullptr);
+  return host_ws(s, m, io, pp, cv, nullptr, nullptr) + 256;
+}
+
+sp_status sp_pipeline_host(const sp_selector* s, const sp_model* m, const sp_pipeline_host_io* io, void* ws,
+                           size_t ws_bytes, sp_stream stream) {
+  cudaStream_t st = (cudaStream_t)stream;
+  if (!io) return fail(SP_ERR_INVALID_ARG, "sp_pipeline_host: NULL io");
+  PipePlan pp;
+  sp_status r = plan_pipe(s, m, io->sel, io->k_cap, &pp);
+  if (r != SP_OK) return r;
+  const sp_select_in& sel = io->sel;
+  if (!sel.X || !sel.stop_bias || !io->host_idx || !io->host_count || !io->host_cu_seqlens || !io->host_hidden)
+    return fail(SP_ERR_INVALID_ARG, "sp_pipeline_host: host buffers missing");
+  const int E = sp_num_episodes(sel.B, sel.n_vis, sel.group_size);
+  if (E < 0) return fail(SP_ERR_SHAPE, "sp_pipeline_host: bad batch");
+  Carve cv(ws);
+  HostParts q;
+  size_t inner = 0;
+  const size_t need = host_ws(s, m, io, pp, cv, &q, &inner) + 256;
+  if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_pipeline_host: workspace %zu < %zu bytes", ws_bytes, need);
+  int nvis = 0, ntxt = 0;
+  for (int b = 0; b < sel.B; ++b) { nvis += sel.n_vis[b]; ntxt += sel.n_txt[b]; }
+  SP_CUDA(cudaMemcpyAsync(q.X, sel.X, (size_t)nvis * s->cfg.D * 2, cudaMemcpyHostToDevice, st), "copy X");
+  if (ntxt > 0) SP_CUDA(cudaMemcpyAsync(q.E, sel.E_text, (size_t)ntxt * s->cfg.D_text * 2, cudaMemcpyHostToDevice, st), "copy E");
+  SP_CUDA(cudaMemcpyAsync(q.bias, sel.stop_bias, (size_t)E * 4, cudaMemcpyHostToDevice, st), "copy stop_bias");
+  SP_CUDA(cudaMemsetAsync(q.err, 0, 16, st), "clear error word");
+  sp_pipeline_io dio = {};
+  dio.sel = sel;
+  dio.sel.X = q.X;
+  dio.sel.E_text = q.E;
+  dio.sel.stop_bias = q.bias;
+  dio.sel.H = nullptr;
+  dio.k_cap = io->k_cap;
+  dio.idx = q.idx;
+  dio.count = q.count;
+  dio.cu_seqlens = q.cu;
+  dio.hidden = q.hidden;
+  dio.err = q.err;
+  r = pipeline_impl(s, m, &dio, q.inner, inner, st);
+  if (r != SP_OK) return r;
+  SP_CUDA(cudaMemcpyAsync(io->host_idx, q.idx, (size_t)sel.B * io->k_cap * 4, cudaMemcpyDeviceToHost, st), "copy idx");
+  SP_CUDA(cudaMemcpyAsync(io->host_count, q.count, (size_t)sel.B * 4, cudaMemcpyDeviceToHost, st), "copy count");
+  SP_CUDA(cudaMemcpyAsync(io->host_cu_seqlens, q.cu, (size_t)(sel.B + 1) * 4, cudaMemcpyDeviceToHost, st), "copy cu");
+  SP_CUDA(cudaMemcpyAsync(io->host_hidden, q.hidden, (size_t)pp.T_cap * m->cfg.d * 4, cudaMemcpyDeviceToHost, st), "copy hidden");
+  return SP_OK;
+}
+
+// ------------------------------------------------------------------ profiling
+
+sp_status sp_profile_begin(int capacity) {
+  for (cudaEvent_t e : g_prof.ev) cudaEventDestroy(e);
+  g_prof = Prof();
+  if (capacity <= 0) return SP_OK;
+  g_prof.ev.resize((size_t)2 * capacity);
+  for (auto& e : g_prof.ev) SP_CUDA(cudaEventCreate(&e), "cudaEventCreate");
+  g_prof.kind.assign(capacity, 0);
+  g_prof.flops.assign(capacity, 0.0);
+  g_prof.bytes.assign(capacity, 0.0);
+  g_prof.cap = capacity;
+  g_prof.n = 0;
+  g_prof.on = true;
+  return SP_OK;
+}
+
+sp_status sp_profile_end(double* ms, long long* launches, double* flops, double* bytes) {
+  if (!g_prof.on) return fail(SP_ERR_INVALID_ARG, "sp_profile_end: profiling is not active");
+  for (int k = 0; k < SP_K_COUNT; ++k) {
+    if (ms) ms[k] = 0.0;
+    if (launches) launches[k] = 0;
+    if (flops) flops[k] = 0.0;
+    if (bytes) bytes[k] = 0.0;
+  }
+  sp_status st = SP_OK;
+  if (g_prof.n > 0) {
+    cudaError_t e = cudaEventSynchronize(g_prof.ev[2 * g_prof.n - 1]);
+    if (e != cudaSuccess) st = cuda_fail(e, "sp_profile_end");
+  }
+  for (int i = 0; st == SP_OK && i < g_prof.n; ++i) {
+    float t = 0.f;
+    cudaEventElapsedTime(&t, g_prof.ev[2 * i], g_prof.ev[2 * i + 1]);
+    const int k = g_prof.kind[i];
+    if (ms) ms[k] += t;
+    if (launches) launches[k] += 1;
+    if (flops) flops[k] += g_prof.flops[i];
+    if (bytes) bytes[k] += g_prof.bytes[i];
+  }
+  for (cudaEvent_t e : g_prof.ev) cudaEventDestroy(e);
+  g_prof = Prof();
+  return st;
+}
+
+}  // extern "C"

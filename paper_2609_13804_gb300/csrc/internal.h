@@ -1,0 +1,137 @@
+// Host-side interfaces between the translation units of libstepprune.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "stepprune.h"
+
+namespace sp {
+
+// Per-image offsets known on the host, passed to kernels by value.
+struct BatchDesc {
+  int B;
+  int group_size;                 // candidates per episode (resolved: > 0 only when grouping)
+  int vis_off[SP_MAX_BATCH + 1];  // prefix of n_vis
+  int txt_off[SP_MAX_BATCH + 1];  // prefix of n_txt
+  int ep_off[SP_MAX_BATCH + 1];   // prefix of episodes per image
+};
+
+bool fill_batch_desc(BatchDesc* d, int B, const int* n_vis, const int* n_txt, int group_size,
+                     std::string* msg);
+
+int device_sm_count();
+
+// ------------------------------------------------------------- profiling
+void prof_begin_launch(cudaStream_t st);
+void prof_end_launch(cudaStream_t st, int kind, double flops, double bytes);
+bool prof_enabled();
+
+// ------------------------------------------------------------- tensor maps
+bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
+                      uint32_t box_rows, std::string* msg);
+
+// ------------------------------------------------------------- tcgen05 GEMM
+enum EpiKind {
+  EPI_BF16 = 0,         // out bf16 = acc
+  EPI_BF16_ROPE = 1,    // out bf16 = acc with rotate-half RoPE on columns < rope_cols
+  EPI_F32 = 2,          // out fp32 = acc
+  EPI_F32_ACC = 3,      // out fp32 += acc (residual add)
+  EPI_GELU_BF16 = 4,    // out bf16 = gelu(acc)
+  EPI_SWIGLU_BF16 = 5,  // out bf16 [.., N/2] = silu(gate) * up
+  EPI_SCATTER_BF16 = 6  // out bf16 row row_map[r] = acc
+};
+
+struct GemmEpi {
+  int kind = EPI_BF16;
+  void* out = nullptr;
+  int ldo = 0;                       // elements
+  const int* row_map = nullptr;      // EPI_SCATTER_BF16
+  const float2* rope = nullptr;      // [max_pos, head_dim / 2] (cos, sin)
+  const int* pos = nullptr;          // [rows]
+  int max_pos = 0;
+  int head_dim = 0;
+  int rope_cols = 0;
+  int up_off = 0;                    // EPI_SWIGLU_BF16: row of B where the 'up' half starts
+};
+
+// Weight operand: the B tensor maps for both tile widths.
+struct GemmB {
+  CUtensorMap map128;  // box rows 64  (BN = 128 -> two boxes of 64)
+  CUtensorMap map256;  // box rows 128 (BN = 256 -> two boxes of 128)
+  int N = 0;           // rows of B
+  int K = 0;
+};
+
+bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg);
+
+// C[M, N] = A[M, K] B[N, K]^T with the given epilogue.  A's tensor map has box
+// rows 128.  M_dev (device int, may be NULL) bounds the rows actually computed;
+// M_cap bounds it on the host.  N_out is the accumulator width (N of B, or the
+// tile columns for SWIGLU: 2 F).
+cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B,
+                      int N_acc, const GemmEpi& e, int* err, cudaStream_t st);
+
+// ------------------------------------------------------------- fp32 SIMT GEMM
+// C[M, N] = A[M, K] B[N, K]^T, fp32, row-major with leading dims.
+cudaError_t sgemm_f32(const float* A, int lda, const float* B, int ldb, float* C, int ldc, int M,
+                      int N, int K, cudaStream_t st);
+// C[i, j] = scale * sum_k A(i, k) B(k, j), fp64 accumulation, arbitrary strides (set-up only).
+cudaError_t fold_matmul(const float* A, long sai, long sak, const float* B, long sbk, long sbj,
+                        float* C, int ldc, int I, int J, int K, float scale, cudaStream_t st);
+
+// ------------------------------------------------------------- norms and small kernels
+// rows from row_count (device, may be NULL) bounded by rows_cap.
+cudaError_t rmsnorm_f32_to_bf16(const float* x, const float* gain, void* out, int rows_cap,
+                                const int* row_count, int d, float eps, cudaStream_t st);
+cudaError_t rmsnorm_f32_to_f32(const float* x, const float* gain, float* out, int rows_cap,
+                               const int* row_count, int d, float eps, cudaStream_t st);
+cudaError_t layernorm_f32(const float* x, int ldx, const float* gain, const float* bias, float* out_f32,
+                          void* out_bf16, int ldo, int rows, int d, float eps, float scale,
+                          cudaStream_t st);
+cudaError_t bf16_to_f32(const void* x, float* out, int rows_cap, const int* row_count, int d,
+                        cudaStream_t st);
+cudaError_t assemble_encoder_input(const BatchDesc& bd, const void* X, const float* P, int D,
+                                   const float* ln_g, const float* ln_b, float eps, float g_text,
+                                   float* R, int rows, cudaStream_t st);
+cudaError_t gather_memory(const BatchDesc& bd, const float* R, const float* H, const float* s_stop,
+                          const float* s_start, float* Mall, int D, cudaStream_t st);
+cudaError_t write_enc_cu(const BatchDesc& bd, int* cu, cudaStream_t st);
+
+// ------------------------------------------------------------- attention
+// Varlen attention over packed qkv [T, (Hq + 2 Hkv) dh] bf16 -> out [T, Hq dh] bf16.
+cudaError_t attention_varlen(const void* qkv, void* out, const int* cu_seqlens, int B,
+                             int max_seqlen_cap, int Hq, int Hkv, int dh, bool causal,
+                             cudaStream_t st);
+
+// ------------------------------------------------------------- selection
+struct SelectArgs {
+  const float* Z;  int ldz;     // decoder tokens y = W_in m
+  const float* KT; int ldkt;    // folded pointer keys
+  const float* QS; int ldqs;    // folded self-attention queries (1/sqrt h inside)
+  const float* KS; int ldks;    // self-attention keys
+  const float* VT; int ldvt;    // folded values Wo_s Wv_s x
+  const float* ln2_g; const float* ln2_b;
+  float ln_eps;
+  int stop_row, start_row;
+  const float* stop_bias;
+  int h, k_max, g;
+  int* order; int* ep_count; float* margin; float* gap; int* rounds;
+  int* err;
+};
+
+int select_cluster_size(const BatchDesc& bd, int h, bool* keys_in_smem, size_t* smem_bytes);
+cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs& a,
+                          int cluster, bool keys_in_smem, size_t smem_bytes, cudaStream_t st);
+cudaError_t restore_launch(const BatchDesc& bd, const int* order, const int* ep_count, int k_max,
+                           int* idx, int k_cap, int* count, int* err, cudaStream_t st);
+
+// ------------------------------------------------------------- compaction
+cudaError_t compact_launch(const BatchDesc& bd, const void* X, int W_vis, const void* text, int W_txt,
+                           const int* idx, int k_cap, const int* count, void* packed, int* cu,
+                           int* pos, void* vis_packed, int* vis_row_map, int* vis_cu, int T_cap,
+                           int* err, cudaStream_t st);
+
+}  // namespace sp

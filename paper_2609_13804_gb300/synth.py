@@ -351,3 +351,64 @@ def target_counts(w: Workload, n_episodes: Optional[int] = None) -> np.ndarray:
             k[j] -= 1
         i += 1
     return k
+
+
+# ----------------------------------------------------------------------------
+# STOP-bias calibration of random-init selectors
+# ----------------------------------------------------------------------------
+
+def _realisable(gaps: np.ndarray):
+    """Round counts a scalar STOP bias can produce for one episode, from its gap
+    trace (best available visual logit minus raw STOP logit, recorded with STOP
+    disabled): stopping after K rounds needs a bias above gap[K] and at or below
+    every earlier gap, i.e. gap[K] must be a new running minimum."""
+    R = len(gaps)
+    out = [(0, float(gaps[0]) + 1.0 if R else 0.0)]
+    run_min = np.inf
+    for t in range(R):
+        if t > 0 and gaps[t] < run_min:
+            lo = float(gaps[t])
+            bias = run_min - 1.0 if not np.isfinite(lo) else 0.5 * (lo + run_min)
+            out.append((t, float(bias)))
+        run_min = min(run_min, float(gaps[t]))
+    if R:
+        out.append((R, float(run_min) - 1.0 if np.isfinite(run_min) else -1e30))
+    return out
+
+
+def stop_biases(gap_traces, targets, *, g: int, k_max: int, n_cand, mean_target: Optional[float] = None):
+    """Per-episode STOP biases whose kept counts are the realisable counts nearest
+    to `targets` (tokens), then nudged so their mean approaches `mean_target`.
+
+    gap_traces[e]: that episode's gap trace with STOP disabled; n_cand[e]: its
+    candidate count.  Returns (biases float32, expected kept counts)."""
+    opts = []
+    for e, gaps in enumerate(gap_traces):
+        gaps = np.asarray(gaps, np.float64)
+        gaps = gaps[~np.isnan(gaps)]
+        cand = []
+        for rounds, bias in _realisable(gaps):
+            cand.append((min(rounds * g, k_max, int(n_cand[e])), bias))
+        opts.append(cand)
+    pick = []
+    for e, cand in enumerate(opts):
+        pick.append(int(np.argmin([abs(k - targets[e]) for k, _ in cand])))
+    if mean_target is not None:
+        want = mean_target * len(opts)
+        for _ in range(20 * len(opts)):
+            tot = sum(opts[e][pick[e]][0] for e in range(len(opts)))
+            best = None
+            for e, cand in enumerate(opts):
+                for step in (-1, 1):
+                    j = pick[e] + step
+                    if 0 <= j < len(cand):
+                        nt = tot - cand[pick[e]][0] + cand[j][0]
+                        gain = abs(tot - want) - abs(nt - want)
+                        if gain > 0 and (best is None or gain > best[0]):
+                            best = (gain, e, j)
+            if best is None:
+                break
+            pick[best[1]] = best[2]
+    biases = np.array([opts[e][pick[e]][1] for e in range(len(opts))], np.float32)
+    counts = np.array([opts[e][pick[e]][0] for e in range(len(opts))], np.int64)
+    return biases, counts

@@ -1,0 +1,306 @@
+"""GPU parity: every stage of the path through the C ABI against the CPU oracle
+on the same seeded inputs (stage-local: each stage is fed seeded inputs, never
+another stage's GPU output)."""
+import numpy as np
+import pytest
+
+import _parity as PT
+from oracle import core as O
+from paper_2609_13804_gb300 import synth as S
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def B():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2609_13804_gb300 import binding
+    binding.lib()
+    return binding
+
+
+def np_(t):
+    if t.dtype == torch.bfloat16:
+        return t.float().cpu().numpy()
+    return t.cpu().numpy()
+
+
+# ------------------------------------------------------------------ selection (Eq. 4, Eq. 11, Alg. 1)
+
+def _run_select_case(B, w, *, scale=1.0, ln_affine=True, targets=None, seed_bias=0, mean_target=None):
+    s = w.selector
+    sel = S.make_selector_weights(w, ln_affine=ln_affine)
+    if scale != 1.0:
+        PT.scale_decoder(sel, scale)
+    H = S.make_memory(w)
+    eps_list = PT.episodes(w.n_vis, w.group_size)
+    if targets is None:
+        t = S.uniform_int(w.seed + seed_bias, "targets", 0, w.k_max + 1, len(eps_list))
+    else:
+        t = targets
+    biases = PT.calibrate_biases(H, w.n_vis, sel, k_max=w.k_max, g=w.g, group_size=w.group_size, targets=t,
+                                 mean_target=mean_target)
+    shape = S.SelectorShape(D=s.D, D_text=s.D_text, h=s.h, n_enc_layers=0)
+    selector = B.Selector(shape, sel, DEV)
+    out = B.sp_select(selector, w.n_vis, w.n_txt, H=B.dev_f32(H, DEV), stop_bias=B.dev_f32(biases, DEV),
+                      group_size=w.group_size, g=w.g, k_max=w.k_max, memory=True)
+    torch.cuda.synchronize()
+    assert int(out["err"].item()) == 0
+    gpu = {k: np_(out[k]) for k in ("order", "ep_count", "rounds", "margin", "gap", "idx", "count")}
+    np.testing.assert_array_equal(np_(out["memory"]), H)
+    images = PT.oracle_select(H, w.n_vis, sel, k_max=w.k_max, g=w.g, group_size=w.group_size, biases=biases)
+    report = []
+    near = PT.compare_selection(gpu, images, g=w.g, report=report)
+    for r in report:
+        print("near-tie:", r)
+    # invariants that hold whatever the ties did
+    for b, n in enumerate(w.n_vis):
+        k = int(gpu["count"][b])
+        row = gpu["idx"][b][:k]
+        assert np.all(np.diff(row) > 0) and (k == 0 or (row[0] >= 0 and row[-1] < n))
+    selector.close()
+    return gpu, images, near
+
+
+def test_select_tiny_ragged(B):
+    w = S.tiny_workload(21, [37, 5, 130, 1, 64], [3, 0, 2, 1, 4], D=128, h=128, k_max=12)
+    _run_select_case(B, w, scale=4.0)
+
+
+def test_select_tiny_stop_extremes(B):
+    w = S.tiny_workload(22, [9, 20, 3], [1, 1, 1], D=128, h=128, k_max=8)
+    gpu, images, _ = _run_select_case(B, w, scale=4.0, targets=[0, 8, 3])
+    assert int(gpu["count"][0]) == 0
+    assert int(gpu["count"][1]) == 8 and int(gpu["rounds"][1]) == 8  # cap: no extra round
+    assert int(gpu["count"][2]) == 3 and int(gpu["rounds"][2]) == 4  # exhausted: only STOP left
+
+
+def test_select_groups_g5(B):
+    w = S.tiny_workload(23, [300, 77, 128], [2, 2, 2], D=128, h=128, k_max=20, group_size=128, g=5)
+    _run_select_case(B, w, scale=4.0)
+
+
+def test_select_llava15_576(B):
+    """576 candidates, D=1024, h=256, cap 192 (the single-image workload)."""
+    w = S.llava15_1layer()
+    _run_select_case(B, w, targets=[64])
+
+
+def test_select_llava15_b16_full(B):
+    """16 x 576 candidates, D=1024, h=512, cap 192, per-image targets 16..192 (mean 64)."""
+    w = S.llava15_7b_b16()
+    gpu, images, near = _run_select_case(B, w, targets=S.target_counts(w), mean_target=w.target_mean_k)
+    counts = gpu["count"].astype(int)
+    print("kept counts", counts.tolist(), "mean", counts.mean(), "near-tie episodes", near)
+
+
+def test_select_anyres_groups(B):
+    """8 x 2880 candidates in groups of 576, g=5, per-group cap 128."""
+    w = S.llavanext_anyres_b8()
+    _run_select_case(B, w, targets=S.uniform_int(w.seed, "t", 16, 129, 40))
+
+
+def test_select_qwen_varres_cluster16(B):
+    """Variable image sizes, D=3584, groups of 1024 (16-CTA clusters hold the keys)."""
+    w = S.qwen25vl_varres_b8()
+    E = len(PT.episodes(w.n_vis, w.group_size))
+    t = [max(1, int(0.11 * n)) for (_, _, n) in PT.episodes(w.n_vis, w.group_size)]
+    _run_select_case(B, w, targets=t)
+
+
+def test_select_internvl_single_episode(B):
+    """One episode over 3328 candidates with cap 1024 and g=5 (keys streamed from L2)."""
+    w = S.internvl3_tiles_b4(mean_k=128)
+    w.n_vis = w.n_vis[:2]
+    w.n_txt = w.n_txt[:2]
+    _run_select_case(B, w, targets=[128, 512])
+
+
+# ------------------------------------------------------------------ cross-modal encoder (Eq. 3)
+
+@pytest.mark.parametrize("case", ["tiny", "llava15"])
+def test_encoder_memory(B, case):
+    if case == "tiny":
+        w = S.tiny_workload(31, [40, 130], [7, 0], D=128, D_text=128, h=128, enc_head_dim=64)
+    else:
+        w = S.llava15_1layer()
+    s = w.selector
+    sel = S.make_selector_weights(w, ln_affine=True)
+    inp = S.make_inputs(w)
+    selector = B.Selector(s, sel, DEV)
+    E = PT.episodes(w.n_vis, w.group_size)
+    out = B.sp_select(selector, w.n_vis, w.n_txt, X=B.dev_bf16(inp["X"], DEV), E_text=B.dev_bf16(inp["E_text"], DEV),
+                      stop_bias=B.dev_f32(np.zeros(len(E)), DEV), group_size=0, g=1, k_max=4, memory=True)
+    torch.cuda.synchronize()
+    got = np_(out["memory"])
+    v0 = t0 = 0
+    for b in range(w.B):
+        Et = O.text_projection(inp["E_text"][t0:t0 + w.n_txt[b]], sel, s.ln_eps, s.g_text)
+        ref = O.encoder(inp["X"][v0:v0 + w.n_vis[b]], Et, sel, s.enc_heads, s.ln_eps)
+        g_ = got[v0:v0 + w.n_vis[b]]
+        rel = np.abs(g_ - ref).max() / np.sqrt((ref ** 2).mean())
+        assert rel <= 1e-2, (b, rel)
+        v0 += w.n_vis[b]
+        t0 += w.n_txt[b]
+    selector.close()
+
+
+# ------------------------------------------------------------------ compaction (Alg. 1 step 5)
+
+@pytest.mark.parametrize("projector_mode", [False, True])
+def test_compaction_bit_exact(B, projector_mode):
+    n_vis, n_txt = [576, 7, 1, 300], [48, 0, 5, 13]
+    W = 1024
+    X = S.bf16_round(S.normal(41, "X", (sum(n_vis), W)))
+    text = S.bf16_round(S.normal(41, "T", (sum(n_txt), W)))
+    k_cap = 200
+    rng = np.random.default_rng(41)
+    idx_list = [np.sort(rng.choice(576, 200, replace=False)), np.arange(7), np.zeros(0, int),
+                np.sort(rng.choice(300, 17, replace=False))]
+    idx = np.full((4, k_cap), -1, np.int32)
+    for b, l in enumerate(idx_list):
+        idx[b, :len(l)] = l
+    count = np.array([len(l) for l in idx_list], np.int32)
+    out = B.sp_compact(n_vis, n_txt, X=B.dev_bf16(X, DEV), text=B.dev_bf16(text, DEV), idx=torch.from_numpy(idx).to(DEV),
+                       count=torch.from_numpy(count).to(DEV), k_cap=k_cap, projector_mode=projector_mode)
+    torch.cuda.synchronize()
+    assert int(out["err"].item()) == 0
+    packed, cu, pos = O.compact(X, n_vis, idx_list, text, n_txt)
+    T = int(cu[-1])
+    np.testing.assert_array_equal(np_(out["cu_seqlens"]), cu)
+    np.testing.assert_array_equal(np_(out["pos"])[:T], pos)
+    got = np_(out["packed"])[:T]
+    if not projector_mode:
+        np.testing.assert_array_equal(got, packed)
+    else:
+        vis_rows = np.concatenate([X[sum(n_vis[:b]):][l] for b, l in enumerate(idx_list)])
+        R = len(vis_rows)
+        np.testing.assert_array_equal(np_(out["vis_packed"])[:R], vis_rows)
+        rmap = np_(out["vis_row_map"])[:R]
+        np.testing.assert_array_equal(packed[rmap], vis_rows)
+        text_rows = np.setdiff1d(np.arange(T), rmap)
+        np.testing.assert_array_equal(got[text_rows], packed[text_rows])
+        np.testing.assert_array_equal(np_(out["vis_cu"]), np.concatenate([[0], np.cumsum(count)]))
+
+
+# ------------------------------------------------------------------ projector
+
+@pytest.mark.parametrize("kind", ["linear", "mlp2"])
+def test_projector_scatter(B, kind):
+    w = S.tiny_workload(51, [300], [1], D=1024, d=1024, n_heads=8, n_kv_heads=8, head_dim=128, ffn=1024,
+                        n_layers=1, proj_kind=kind)
+    w.model.proj_hidden = 2048
+    head = S.make_model_head(w)
+    L = S.make_layer_weights(w, 0)
+    model = B.Model(w.model, [L], head, DEV, max_pos=512)
+    rows = 300
+    vis = S.bf16_round(S.normal(51, "vis", (rows, 1024)))
+    T = rows + 50
+    rmap = np.random.default_rng(51).permutation(T)[:rows].astype(np.int32)
+    packed = torch.zeros((T, 1024), dtype=torch.bfloat16, device=DEV)
+    vis_cu = torch.tensor([0, rows], dtype=torch.int32, device=DEV)
+    err = B.sp_project(model, vis_packed=B.dev_bf16(vis, DEV), vis_row_map=torch.from_numpy(rmap).to(DEV),
+                       vis_cu=vis_cu, packed=packed, rows_cap=rows, B=1)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    ref = O.projector(vis, head)
+    got = np_(packed)[rmap]
+    tol = 1e-2 * np.abs(ref).max()
+    assert np.abs(got - ref).max() <= tol, np.abs(got - ref).max()
+    untouched = np.setdiff1d(np.arange(T), rmap)
+    assert np.all(np_(packed)[untouched] == 0)
+    model.close()
+
+
+# ------------------------------------------------------------------ prefill
+
+def _prefill_case(B, w, lens, n_layers, seed_name="packed", affine=True):
+    layers = [S.make_layer_weights(w, l, norm_affine=affine) for l in range(n_layers)]
+    head = S.make_model_head(w, norm_affine=affine)
+    model = B.Model(w.model, layers, head, DEV, max_pos=max(lens) + 8)
+    T = int(sum(lens))
+    x = S.bf16_round(S.normal(w.seed, seed_name, (T, w.model.d), 0.5))
+    cu, pos = PT.lens_cu_pos(lens)
+    out = B.sp_prefill(model, x=B.dev_bf16(x, DEV), cu_seqlens=torch.from_numpy(cu.astype(np.int32)).to(DEV),
+                       pos=torch.from_numpy(pos.astype(np.int32)).to(DEV), B=len(lens), T_cap=T,
+                       max_seqlen_cap=max(lens))
+    torch.cuda.synchronize()
+    assert int(out["err"].item()) == 0
+    ref = O.prefill(x, layers, w.model, cu, pos, head["final_norm"])
+    r = PT.hidden_close(np_(out["hidden"])[:T], ref, w.name)
+    print("prefill", w.name, "max-abs %.3e mean-rel %.3e" % r)
+    model.close()
+
+
+def test_prefill_tiny_gqa_ragged(B):
+    w = S.tiny_workload(61, [1], [1], d=128, n_heads=2, n_kv_heads=1, head_dim=64, ffn=256, n_layers=2)
+    _prefill_case(B, w, [5, 130, 1, 64], 2)
+
+
+def test_prefill_llava15_1layer(B):
+    w = S.llava15_1layer()
+    _prefill_case(B, w, [96, 33, 200], 1)
+
+
+def test_prefill_llama7b_dims_2layers(B):
+    w = S.llava15_7b_b16()
+    _prefill_case(B, w, [112, 240, 64, 17], 2)
+
+
+def test_prefill_qwen_gqa_dims(B):
+    w = S.qwen25vl_varres_b8()
+    _prefill_case(B, w, [75, 300], 1)
+
+
+# ------------------------------------------------------------------ whole path
+
+def test_pipeline_end_to_end_without_encoder(B):
+    """Selection straight on the visual tokens (no encoder blocks) so that the
+    selection is exact end to end; then compaction, projector and prefill."""
+    w = S.tiny_workload(71, [200, 64, 130], [9, 3, 0], D=128, D_text=256, h=128, d=256, n_heads=4,
+                        n_kv_heads=2, head_dim=64, ffn=256, n_layers=2, k_max=40, proj_kind="mlp2")
+    w.model.proj_hidden = 256
+    s = w.selector
+    sel = S.make_selector_weights(w, ln_affine=True)
+    PT.scale_decoder(sel, 4.0)
+    sel["enc"] = []
+    inp = S.make_inputs(w)
+    X, E = inp["X"], inp["E_text"]
+    biases = PT.calibrate_biases(X, w.n_vis, sel, k_max=w.k_max, g=1, group_size=0, targets=[17, 40, 5])
+    layers = [S.make_layer_weights(w, l, norm_affine=True) for l in range(2)]
+    head = S.make_model_head(w, norm_affine=True)
+    shape = S.SelectorShape(D=s.D, D_text=s.D_text, h=s.h, n_enc_layers=0)
+    selector = B.Selector(shape, sel, DEV)
+    model = B.Model(w.model, layers, head, DEV, max_pos=512)
+    pipe = B.Pipeline(selector, model, w.n_vis, w.n_txt, group_size=0, g=1, k_max=w.k_max)
+    Xd, Ed, bd = B.dev_bf16(X, DEV), B.dev_bf16(E, DEV), B.dev_f32(biases, DEV)
+    pipe(Xd, Ed, bd)
+    torch.cuda.synchronize()
+    assert int(pipe.err.item()) == 0
+    ref = O.run_pipeline(X, E, w.n_vis, w.n_txt, sel, shape, head, layers, w.model, k_max=w.k_max, g=1,
+                         group_size=0, stop_bias=biases)
+    counts = np_(pipe.count)
+    for b in range(w.B):
+        assert list(np_(pipe.idx)[b][:counts[b]]) == list(ref["idx"][b])
+    cu = np_(pipe.cu)
+    np.testing.assert_array_equal(cu, ref["cu_seqlens"])
+    T = int(cu[-1])
+    PT.hidden_close(np_(pipe.hidden)[:T], ref["hidden"], "pipeline")
+    # the same call from host buffers gives the same bytes
+    Xh, Eh = Xd.cpu().pin_memory(), Ed.cpu().pin_memory()
+    bh = bd.cpu().pin_memory()
+    oi = torch.empty_like(pipe.idx, device="cpu").pin_memory()
+    oc = torch.empty_like(pipe.count, device="cpu").pin_memory()
+    ocu = torch.empty_like(pipe.cu, device="cpu").pin_memory()
+    oh = torch.empty_like(pipe.hidden, device="cpu").pin_memory()
+    pipe.host(Xh, Eh, bh, oi, oc, ocu, oh)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(oi.numpy(), np_(pipe.idx))
+    np.testing.assert_array_equal(ocu.numpy(), cu)
+    np.testing.assert_array_equal(oh.numpy()[:T], np_(pipe.hidden)[:T])
+    selector.close()
+    model.close()
