@@ -1,0 +1,404 @@
+"""Benchmark of the StepPrune inference path on the LLaVA-1.5-7B-shaped batch.
+
+One step = one sp_pipeline call over a batch of 16 images x 576 visual tokens
+(+ 48 text tokens each): text projection and the 2-block cross-modal encoder,
+candidate precompute, the sequential selection loop, restore, compaction, the
+2-layer GELU projector on the kept rows and the 32-layer Llama-7B-dims prefill
+over the packed prefix.  Random-init weights and seeded synthetic inputs; STOP
+biases tuned so the kept counts span 16..192 with mean about 64.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  `value` is ms per batch over the whole job
+(lower is better); with N ranks each rank runs its own batch (weak scaling).
+`--impl reference` times the CPU oracle on a bounded sample of the same
+workload instead.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_13804_gb300 import synth as S  # noqa: E402
+
+METRIC = "pruned-prefill ms/batch"
+UNIT = "ms/batch"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16": d["bf16_tflops"], "bf16_sus": d["bf16_tflops_sustained"],
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sus": 1700.0, "source": "fallback"}
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- set-up
+
+def device_layer_weights(m, l, dev, gen, torch):
+    qkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
+
+    def rnd(shape):
+        return (torch.randn(shape, device=dev, generator=gen, dtype=torch.float32) * 0.02).to(torch.bfloat16)
+
+    return {"Wqkv": rnd((qkv, m.d)), "Wo": rnd((m.d, m.n_heads * m.head_dim)), "Wgu": rnd((2 * m.ffn, m.d)),
+            "Wdown": rnd((m.d, m.ffn)), "attn_norm": torch.ones(m.d, device=dev),
+            "mlp_norm": torch.ones(m.d, device=dev)}
+
+
+def gemm_flops(w, T, K_sum, T_enc, n_txt_sum):
+    """Algorithmic flops of every dense contraction of one step (2 per MAC)."""
+    s, m = w.selector, w.model
+    enc = s.n_enc_layers * 2.0 * T_enc * (3 * s.D * s.D + s.D * s.D + 2 * s.D * s.enc_ffn)
+    text = 2.0 * n_txt_sum * s.D_text * s.D
+    proj = 2.0 * K_sum * (m.proj_in * m.proj_hidden + m.proj_hidden * m.d) if m.proj_kind == "mlp2" else \
+        (2.0 * K_sum * m.proj_in * m.d if m.proj_kind == "linear" else 0.0)
+    qkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
+    lm = m.n_layers * 2.0 * T * (m.d * qkv + m.n_heads * m.head_dim * m.d + 2 * m.d * m.ffn + m.ffn * m.d)
+    return enc + text + proj + lm
+
+
+_SAMPLE_CACHE = {}
+
+
+def cpu_oracle_sample(w, n_images=1, n_layers=1):
+    """Times the oracle on a bounded sample of the workload and scales it to one
+    batch: per image the encoder + selection, the projector on its kept rows and
+    n_layers of the 32 decoder layers (weights are drawn once, outside the timing)."""
+    from oracle import core as O
+    s, m = w.selector, w.model
+    key = (w.name, n_layers)
+    if key not in _SAMPLE_CACHE:
+        _SAMPLE_CACHE[key] = (S.make_selector_weights(w), S.make_model_head(w), S.make_inputs(w),
+                              [S.make_layer_weights(w, l) for l in range(n_layers)])
+    sel, head, inp, layers = _SAMPLE_CACHE[key]
+    n_heads = s.D // s.enc_head_dim
+    t_sel = t_proj = t_lm = 0.0
+    for b in range(n_images):
+        v0, t0 = b * w.n_vis[0], b * w.n_txt[0]
+        X = inp["X"][v0:v0 + w.n_vis[b]]
+        E = inp["E_text"][t0:t0 + w.n_txt[b]]
+        t = time.perf_counter()
+        Et = O.text_projection(E, sel, s.ln_eps, s.g_text)
+        H = O.encoder(X, Et, sel, n_heads, s.ln_eps)
+        r = O.select_episode(H, sel, k_max=w.k_max, g=w.g, stop_bias=0.0, eps=s.ln_eps)
+        idx = O.restore(r["order"])
+        if len(idx) < int(w.target_mean_k):  # time a mean-sized prefix whatever this bias kept
+            idx = np.arange(int(w.target_mean_k))
+        t_sel += time.perf_counter() - t
+        t = time.perf_counter()
+        vis = O.projector(X[idx], head)
+        t_proj += time.perf_counter() - t
+        x = np.concatenate([vis, E])
+        cu, pos = np.array([0, len(x)]), np.arange(len(x))
+        t = time.perf_counter()
+        for L in layers:
+            x = O.prefill_layer(x, L, m, cu, pos)
+        t_lm += time.perf_counter() - t
+    per_image_ms = 1e3 * (t_sel + t_proj + t_lm * m.n_layers / n_layers) / n_images
+    return per_image_ms * w.B, t_sel + t_proj + t_lm
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = S.llava15_7b_b16()
+    samples = []
+    wall = 0.0
+    for i in range(args.warmup + args.steps):
+        v, secs = cpu_oracle_sample(w)
+        wall += secs
+        if i >= args.warmup:
+            samples.append(v)
+    value = statistics.median(samples)
+    sample = ("per step: 1 of 16 images through text projection + 2-block encoder + selection, projector on "
+              "its kept rows, 1 of 32 decoder layers; scaled to 16 images x 32 layers")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": value, "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "images": w.B, "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
+                       "layers": w.model.n_layers},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args):
+    import torch
+    from paper_2609_13804_gb300 import binding as B
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    def barrier():
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    w = S.llava15_7b_b16(seed=1002 + rank)
+    s, m = w.selector, w.model
+    sel_w = S.make_selector_weights(w)
+    selector = B.Selector(s, sel_w, dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(w.seed)
+    layers = [device_layer_weights(m, l, dev, gen, torch) for l in range(m.n_layers)]
+    head = {"final_norm": torch.ones(m.d, device=dev),
+            "proj_W1": (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16),
+            "proj_W2": (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)}
+    model = B.Model(m, layers, head, dev, max_pos=1024)
+    inp = S.make_inputs(w)
+    X = B.dev_bf16(inp["X"], dev)
+    E = B.dev_bf16(inp["E_text"], dev)
+    n_ep = len(w.episodes())
+
+    # STOP biases: gap traces with STOP disabled, then the realisable counts
+    # nearest the per-image targets (16..192, mean 64)
+    cal = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=B.dev_f32(np.full(n_ep, -1e30), dev),
+                      group_size=w.group_size, g=w.g, k_max=w.k_max)
+    torch.cuda.synchronize()
+    gaps = cal["gap"].cpu().numpy()
+    rounds = cal["rounds"].cpu().numpy()
+    traces = [gaps[e, :rounds[e]] for e in range(n_ep)]
+    biases, expect = S.stop_biases(traces, S.target_counts(w), g=w.g, k_max=w.k_max,
+                                   n_cand=[n for (_, _, n) in w.episodes()], mean_target=w.target_mean_k)
+    bias = B.dev_f32(biases, dev)
+
+    pipe = B.Pipeline(selector, model, w.n_vis, w.n_txt, group_size=w.group_size, g=w.g, k_max=w.k_max)
+    for _ in range(args.warmup):
+        pipe(X, E, bias)
+    torch.cuda.synchronize()
+    counts = pipe.count.cpu().numpy().astype(int)
+    K_sum = int(counts.sum())
+    T = int(pipe.cu[-1].item())
+    T_enc = sum(w.n_vis) + sum(w.n_txt)
+    flops = gemm_flops(w, T, K_sum, T_enc, sum(w.n_txt))
+
+    # ---- timed region: K steps, per-launch events inside
+    st = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    B.sp_profile_begin(args.steps * 2000)
+    with Clocks(local) as clk:
+        barrier()
+        ev0.record(st)
+        for _ in range(args.steps):
+            pipe(X, E, bias)
+        ev1.record(st)
+        barrier()
+    prof = B.sp_profile_end()
+    ms_step = ev0.elapsed_time(ev1) / args.steps
+    if dist:
+        t = torch.tensor([ms_step], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_step = float(t.item())
+    value = ms_step / world
+    launches = sum(v["launches"] for v in prof.values()) // args.steps
+    gemm_ms = prof["gemm"]["ms"] / args.steps
+    pk = peaks()
+    achieved = flops / (gemm_ms * 1e-3) / 1e12
+
+    # ---- side measurements (outside the timed region)
+    def timed(fn, reps=5):
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        fn()
+        torch.cuda.synchronize()
+        a.record()
+        for _ in range(reps):
+            fn()
+        b_.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b_) / reps
+
+    sel_ws = None
+
+    def do_select():
+        nonlocal sel_ws
+        r = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bias, group_size=w.group_size,
+                        g=w.g, k_max=w.k_max, traces=False, ws=sel_ws)
+        sel_ws = r["_ws"]
+        return r
+
+    sel_out = do_select()
+    select_ms = timed(do_select)
+    k_cap = pipe.k_cap
+    comp = {}
+
+    def do_compact(idx, count, kc):
+        comp["o"] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
+                                 projector_mode=True)
+
+    compact_ms = timed(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap))
+    comp_bytes = 2.0 * (K_sum * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
+
+    def prefill_stage(idx, count, kc):
+        do_compact(idx, count, kc)
+        o = comp["o"]
+        B.sp_project(model, vis_packed=o["vis_packed"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
+                     packed=o["packed"], rows_cap=o["rows_cap"], B=w.B)
+        lens_cap = max(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
+        B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=w.B, T_cap=o["T_cap"],
+                     max_seqlen_cap=lens_cap)
+
+    pruned_ms = timed(lambda: prefill_stage(sel_out["idx"], sel_out["count"], k_cap), reps=3)
+    full_idx = torch.arange(576, dtype=torch.int32, device=dev).repeat(w.B, 1).contiguous()
+    full_cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
+    full_ms = timed(lambda: prefill_stage(full_idx, full_cnt, 576), reps=3)
+
+    # ---- end to end from host buffers (copies inside the timed region)
+    Xh = X.cpu().pin_memory()
+    Eh = E.cpu().pin_memory()
+    bh = bias.cpu().pin_memory()
+    oi = torch.empty(pipe.idx.shape, dtype=torch.int32).pin_memory()
+    oc = torch.empty(pipe.count.shape, dtype=torch.int32).pin_memory()
+    ocu = torch.empty(pipe.cu.shape, dtype=torch.int32).pin_memory()
+    oh = torch.empty(pipe.hidden.shape, dtype=torch.float32).pin_memory()
+    pipe.host(Xh, Eh, bh, oi, oc, ocu, oh)
+    torch.cuda.synchronize()
+    e2e_steps = max(2, min(args.steps, 5))
+    barrier()
+    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(e2e_steps):
+        pipe.host(Xh, Eh, bh, oi, oc, ocu, oh)
+    b_.record()
+    barrier()
+    e2e_ms = a.elapsed_time(b_) / e2e_steps
+    if dist:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    h2d = Xh.numel() * 2 + Eh.numel() * 2 + bh.numel() * 4
+    d2h = oi.numel() * 4 + oc.numel() * 4 + ocu.numel() * 4 + oh.numel() * 4
+
+    if rank == 0:
+        cpu_line = None
+        if world == 1 and not args.no_cpu:
+            v, secs = cpu_oracle_sample(w)
+            cpu_line = {"value": v, "unit": UNIT, "cores": cores(), "kind": "oracle",
+                        "sample": "1 of 16 images (encoder + selection, projector, 1 of 32 layers), scaled to "
+                                  f"16 images x 32 layers; {secs:.1f} s of CPU work"}
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "images": w.B, "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
+                       "layers": m.n_layers, "d": m.d, "selector_h": s.h, "k_max": w.k_max,
+                       "mean_kept": float(counts.mean()), "packed_tokens": T,
+                       "l2": "inputs larger than L2: 13.5 GB of weights streamed every step"},
+            "roofline": {"kernel": "gemm_tc (tcgen05)", "bound": "tensor", "achieved": achieved,
+                         "peak": pk["bf16_sus"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sus"],
+                         "peak_source": pk["source"] + " bf16 sustained", "traffic": None,
+                         "gemm_ms_per_step": gemm_ms, "gemm_flops_per_step": flops},
+            "cpu_baseline": cpu_line,
+            "e2e": {"value": e2e_ms / world, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches,
+            "clocks": clk.summary(),
+            "stages_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()},
+            "select_us_per_image": 1e3 * select_ms / w.B,
+            "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,
+            "pruned_prefill_ms": pruned_ms,
+            "full_prefix_prefill_ms": full_ms,
+            "speedup_prefill": full_ms / pruned_ms,
+            "speedup_with_selection": full_ms / (pruned_ms + select_ms),
+            "token_ratio": (sum(w.n_vis) + sum(w.n_txt)) / T,
+            "kept_counts": counts.tolist(),
+        }
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -27,6 +27,7 @@ Parity status of each function:
                                         special case, Eq. 1; invariants of Alg. 1 and Eq. 11)
   restore / compact                     pinned (hand-worked golden fixture; invariants)
   rope                                  pinned (rotation closed form, relative-position property)
+  round_bf16                            pinned (torch's float32 -> bfloat16 conversion)
   projector, prefill_layer, prefill     pinned through their parts plus special cases
                                         (zero output weights -> identity; uniform attention);
                                         the composition of a whole random-weight LM is
@@ -46,6 +47,26 @@ NEG_INF = -np.inf
 
 def _f(x) -> np.ndarray:
     return np.asarray(x, dtype=F64)
+
+
+def round_bf16(x) -> np.ndarray:
+    """Round to the nearest bfloat16 (ties to even), returned as fp64.
+
+    bfloat16 keeps the top 16 bits of the IEEE fp32 pattern: the value is first
+    rounded to fp32, then the low 16 bits are rounded away (ties to even)."""
+    u = np.ascontiguousarray(_f(x).astype(np.float32)).view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
+    return r.astype(np.uint32).view(np.float32).astype(F64)
+
+
+def _store(x, store: Optional[str]) -> np.ndarray:
+    """Storage rounding of an activation between two ops: none (fp64 throughout)
+    or 'bf16' (what a bf16 model keeps in memory between its kernels)."""
+    if store is None:
+        return _f(x)
+    if store == "bf16":
+        return round_bf16(x)
+    raise ValueError(store)
 
 
 # ----------------------------------------------------------------------------
@@ -369,17 +390,19 @@ def compact(X, n_vis: Sequence[int], idx_list: Sequence[Sequence[int]], text, n_
     return packed, cu, pos
 
 
-def projector(rows, head: Dict) -> np.ndarray:
+def projector(rows, head: Dict, store: Optional[str] = None) -> np.ndarray:
     """Frozen multimodal projector applied to the kept visual rows after the
-    restore (Sec. 3.3): linear W1 x, or the two-layer W2 GELU(W1 x)."""
+    restore (Sec. 3.3): linear W1 x, or the two-layer W2 GELU(W1 x).  With
+    store='bf16' the hidden activation and the output are stored as bf16."""
     kind = head["proj_kind"]
     rows = _f(rows)
     if kind == "none":
         return rows
     if kind == "linear":
-        return rows @ _f(head["proj_W1"]).T
+        return _store(rows @ _f(head["proj_W1"]).T, store)
     if kind == "mlp2":
-        return gelu(rows @ _f(head["proj_W1"]).T) @ _f(head["proj_W2"]).T
+        a = _store(gelu(rows @ _f(head["proj_W1"]).T), store)
+        return _store(a @ _f(head["proj_W2"]).T, store)
     raise ValueError(kind)
 
 
@@ -395,27 +418,30 @@ def rope(x, pos, n_heads: int, head_dim: int, theta: float) -> np.ndarray:
     return np.concatenate([a * c - b * s, b * c + a * s], axis=-1).reshape(x.shape[0], -1)
 
 
-def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos) -> np.ndarray:
+def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = None) -> np.ndarray:
     """One pre-norm decoder layer of the frozen LM over the packed sequences:
     h += Wo Attn(RoPE(Wq x), RoPE(Wk x), Wv x), x = RMSNorm(h);
     h += Wdown (SiLU(Wg x') * Wu x'), x' = RMSNorm(h).  Attention is causal and
-    never crosses a sequence boundary."""
+    never crosses a sequence boundary.  The residual stream h stays fp64; with
+    store='bf16' the activations a bf16 model keeps between ops (normalised
+    inputs, rotated q / k, v, attention output, SwiGLU output) are rounded to
+    bf16 where they are stored."""
     h = _f(h).copy()
     Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
-    x = rms_norm(h, m.rms_eps, L.get("attn_norm"))
+    x = _store(rms_norm(h, m.rms_eps, L.get("attn_norm")), store)
     qkv = x @ _f(L["Wqkv"]).T
-    q = rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta)
-    k = rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta)
-    v = qkv[:, (Hq + Hkv) * dh:]
+    q = _store(rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta), store)
+    k = _store(rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta), store)
+    v = _store(qkv[:, (Hq + Hkv) * dh:], store)
     o = np.zeros((h.shape[0], Hq * dh), dtype=F64)
     for b in range(len(cu) - 1):
         s, e = int(cu[b]), int(cu[b + 1])
         if e > s:
             o[s:e] = attention(q[s:e], k[s:e], v[s:e], Hq, Hkv, causal=True)
-    h = h + o @ _f(L["Wo"]).T
-    x2 = rms_norm(h, m.rms_eps, L.get("mlp_norm"))
+    h = h + _store(o, store) @ _f(L["Wo"]).T
+    x2 = _store(rms_norm(h, m.rms_eps, L.get("mlp_norm")), store)
     gu = x2 @ _f(L["Wgu"]).T
-    h = h + (silu(gu[:, :F]) * gu[:, F:]) @ _f(L["Wdown"]).T
+    h = h + _store(silu(gu[:, :F]) * gu[:, F:], store) @ _f(L["Wdown"]).T
     return h
 
 
@@ -425,10 +451,10 @@ def final_norm(h, m, gain=None) -> np.ndarray:
     return rms_norm(h, m.rms_eps, gain)
 
 
-def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None) -> np.ndarray:
+def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None, store: Optional[str] = None) -> np.ndarray:
     h = _f(x)
     for L in layers:
-        h = prefill_layer(h, L, m, cu, pos)
+        h = prefill_layer(h, L, m, cu, pos, store)
     return final_norm(h, m, final_gain)
 
 
@@ -438,7 +464,7 @@ def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None) -> np.ndarra
 
 def run_pipeline(X, E_text, n_vis, n_txt, sel: Dict, sel_shape, head: Dict, layers, model_shape,
                  *, k_max: int, g: int, group_size: int, stop_bias: Sequence[float],
-                 mode: str = "incremental") -> Dict:
+                 mode: str = "incremental", store: Optional[str] = None) -> Dict:
     """Selector encoder -> selection -> restore -> gather -> projector -> prefill."""
     X, E_text = _f(X), _f(E_text)
     n_heads = sel_shape.D // sel_shape.enc_head_dim
@@ -462,7 +488,7 @@ def run_pipeline(X, E_text, n_vis, n_txt, sel: Dict, sel_shape, head: Dict, laye
     v0 = 0
     vis_proj = []
     for b in range(len(n_vis)):
-        vis_proj.append(projector(X[v0:v0 + n_vis[b]][idx_list[b]], head))
+        vis_proj.append(projector(X[v0:v0 + n_vis[b]][idx_list[b]], head, store))
         v0 += n_vis[b]
     packed_rows, lens = [], []
     t0 = 0
@@ -473,6 +499,6 @@ def run_pipeline(X, E_text, n_vis, n_txt, sel: Dict, sel_shape, head: Dict, laye
     x = np.concatenate(packed_rows, axis=0)
     cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
     pos = np.concatenate([np.arange(n) for n in lens])
-    hidden = prefill(x, layers, model_shape, cu, pos, head.get("final_norm"))
+    hidden = prefill(x, layers, model_shape, cu, pos, head.get("final_norm"), store)
     return {"H": H_all, "idx": idx_list, "images": eps_per_img, "x": x, "cu_seqlens": cu,
             "pos": pos, "hidden": hidden}

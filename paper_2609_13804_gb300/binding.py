@@ -363,7 +363,7 @@ class Model:
             self._keep.append(t)
             return ptr(t)
 
-        if device_weights is not None:  # already on the device (bench: generated there)
+        if device_weights is not None:  # already on the device
             layers = device_weights["layers"]
             head = device_weights["head"]
         for l, L in enumerate(layers):

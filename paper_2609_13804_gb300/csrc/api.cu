@@ -346,8 +346,6 @@ sp_status plan_select(const sp_selector* s, const sp_select_in* in, SelPlan* p) 
   p->ntxt = p->bd.txt_off[in->B];
   p->rows = p->nvis + 2;
   p->encoder = (in->H == nullptr);
-  if (p->encoder && s->cfg.n_enc_layers == 0 && !in->X)
-    return fail(SP_ERR_INVALID_ARG, "sp_select: X is required when H is NULL");
   p->T_enc = p->nvis + p->ntxt;
   p->max_enc = 0;
   for (int b = 0; b < in->B; ++b) p->max_enc = std::max(p->max_enc, in->n_vis[b] + in->n_txt[b]);

@@ -8,7 +8,9 @@ Comparison rules:
     Per-round STOP gaps and margins agree to 2e-4 before that round.
   * compaction: packed rows, cu_seqlens and positions bit-exact.
   * prefill hidden states (after the final RMSNorm): max-abs <= 3e-2 and
-    mean |diff| / mean |ref| <= 1e-2.
+    mean |diff| / mean |ref| <= 1e-2 against the oracle with bf16 storage of
+    the activations a bf16 model keeps between ops; against the pure fp64
+    oracle the mean-rel bound still holds and max-abs is reported.
 """
 import math
 
@@ -110,6 +112,16 @@ def hidden_close(gpu, ref, what=""):
     max_abs = float(d.max()) if d.size else 0.0
     mean_rel = float(d.mean() / max(np.abs(ref).mean(), 1e-30)) if d.size else 0.0
     assert max_abs <= HID_MAX_ABS and mean_rel <= HID_MEAN_REL, f"{what}: max-abs {max_abs:.3e} mean-rel {mean_rel:.3e}"
+    return max_abs, mean_rel
+
+
+def mean_rel_only(gpu, ref, what=""):
+    gpu = np.asarray(gpu, np.float64)
+    ref = np.asarray(ref, np.float64)
+    d = np.abs(gpu - ref)
+    max_abs = float(d.max()) if d.size else 0.0
+    mean_rel = float(d.mean() / max(np.abs(ref).mean(), 1e-30)) if d.size else 0.0
+    assert mean_rel <= HID_MEAN_REL, f"{what} vs fp64: mean-rel {mean_rel:.3e}"
     return max_abs, mean_rel
 
 

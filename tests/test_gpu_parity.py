@@ -230,14 +230,17 @@ def _prefill_case(B, w, lens, n_layers, seed_name="packed", affine=True):
                        max_seqlen_cap=max(lens))
     torch.cuda.synchronize()
     assert int(out["err"].item()) == 0
-    ref = O.prefill(x, layers, w.model, cu, pos, head["final_norm"])
-    r = PT.hidden_close(np_(out["hidden"])[:T], ref, w.name)
-    print("prefill", w.name, "max-abs %.3e mean-rel %.3e" % r)
+    got = np_(out["hidden"])[:T]
+    ref = O.prefill(x, layers, w.model, cu, pos, head["final_norm"], store="bf16")
+    r = PT.hidden_close(got, ref, w.name)
+    r64 = PT.mean_rel_only(got, O.prefill(x, layers, w.model, cu, pos, head["final_norm"]), w.name)
+    print("prefill", w.name, "vs bf16-storage oracle: max-abs %.3e mean-rel %.3e" % r,
+          "| vs fp64 oracle: max-abs %.3e mean-rel %.3e" % r64)
     model.close()
 
 
 def test_prefill_tiny_gqa_ragged(B):
-    w = S.tiny_workload(61, [1], [1], d=128, n_heads=2, n_kv_heads=1, head_dim=64, ffn=256, n_layers=2)
+    w = S.tiny_workload(61, [1], [1], D=128, d=128, n_heads=2, n_kv_heads=1, head_dim=64, ffn=256, n_layers=2)
     _prefill_case(B, w, [5, 130, 1, 64], 2)
 
 
@@ -282,7 +285,7 @@ def test_pipeline_end_to_end_without_encoder(B):
     torch.cuda.synchronize()
     assert int(pipe.err.item()) == 0
     ref = O.run_pipeline(X, E, w.n_vis, w.n_txt, sel, shape, head, layers, w.model, k_max=w.k_max, g=1,
-                         group_size=0, stop_bias=biases)
+                         group_size=0, stop_bias=biases, store="bf16")
     counts = np_(pipe.count)
     for b in range(w.B):
         assert list(np_(pipe.idx)[b][:counts[b]]) == list(ref["idx"][b])
@@ -303,4 +306,43 @@ def test_pipeline_end_to_end_without_encoder(B):
     np.testing.assert_array_equal(ocu.numpy(), cu)
     np.testing.assert_array_equal(oh.numpy()[:T], np_(pipe.hidden)[:T])
     selector.close()
+    model.close()
+
+
+def test_prefill_llava15_b16_32layers_sampled(B):
+    """The benchmark's prefill launch: 32 Llama-7B-dims layers over 16 packed
+    sequences (kept counts 16..192 + 48 text tokens).  The oracle evaluates two
+    of the sequences (the shortest and the longest); attention never crosses a
+    sequence, so their rows are exact to compare."""
+    w = S.llava15_7b_b16()
+    m = w.model
+    k = S.target_counts(w)
+    lens = [int(x) + 48 for x in k]
+    T = sum(lens)
+    cu, pos = PT.lens_cu_pos(lens)
+    x = S.bf16_round(S.normal(w.seed, "packed32", (T, m.d), 0.5))
+    picks = [int(np.argmin(lens)), int(np.argmax(lens))]
+    hs = {b: x[cu[b]:cu[b + 1]].astype(np.float64) for b in picks}
+    dev_layers = []
+    for l in range(m.n_layers):
+        L = S.make_layer_weights(w, l)
+        dev_layers.append({k_: B.dev_bf16(L[k_], DEV) for k_ in ("Wqkv", "Wo", "Wgu", "Wdown")})
+        dev_layers[-1]["attn_norm"] = torch.ones(m.d, device=DEV)
+        dev_layers[-1]["mlp_norm"] = torch.ones(m.d, device=DEV)
+        for b in picks:
+            n = lens[b]
+            hs[b] = O.prefill_layer(hs[b], L, m, [0, n], np.arange(n), store="bf16")
+        del L
+    head = {"final_norm": torch.ones(m.d, device=DEV), "proj_W1": None, "proj_W2": None}
+    model = B.Model(m, None, None, DEV, max_pos=512, device_weights={"layers": dev_layers, "head": head})
+    out = B.sp_prefill(model, x=B.dev_bf16(x, DEV), cu_seqlens=torch.from_numpy(cu.astype(np.int32)).to(DEV),
+                       pos=torch.from_numpy(pos.astype(np.int32)).to(DEV), B=len(lens), T_cap=T,
+                       max_seqlen_cap=max(lens))
+    torch.cuda.synchronize()
+    assert int(out["err"].item()) == 0
+    got = np_(out["hidden"])
+    for b in picks:
+        ref = O.final_norm(hs[b], m)
+        r = PT.hidden_close(got[cu[b]:cu[b + 1]], ref, f"sequence {b}")
+        print(f"32-layer prefill, sequence {b} (len {lens[b]}): max-abs %.3e mean-rel %.3e" % r)
     model.close()

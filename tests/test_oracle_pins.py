@@ -378,3 +378,17 @@ def test_projector_forms():
         ref[2].weight.copy_(t64(W2))
         want = ref(t64(x)).numpy()
     np.testing.assert_allclose(O.projector(x, head), want, atol=1e-12)
+
+
+def test_bf16_storage_rounding_matches_torch():
+    x = np.concatenate([S.normal(16, "x", (4000,)) * 10 ** k for k in range(-6, 6)]).astype(np.float64)
+    x = np.concatenate([x, [0.0, -0.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, 65504.0, 1e-40]])
+    ref = torch.tensor(x, dtype=torch.float64).to(torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_bf16(x), ref)
+    # storage rounding only moves values by at most half a bf16 ulp
+    w, L = _tiny_lm(17)
+    xin = S.normal(17, "x", (9, 32)).astype(np.float64)
+    cu, pos = [0, 9], np.arange(9)
+    a = O.prefill_layer(xin, L, w.model, cu, pos)
+    b = O.prefill_layer(xin, L, w.model, cu, pos, store="bf16")
+    assert 0 < np.abs(a - b).max() < 0.05 * np.abs(a).max()
