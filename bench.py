@@ -244,6 +244,11 @@ def run_ours(args):
     for _ in range(args.warmup):
         pipe(X, E, bias)
     torch.cuda.synchronize()
+    if args.launch_list:
+        # one more step and nothing else: the last step's launches are the list to read
+        pipe(X, E, bias)
+        torch.cuda.synchronize()
+        return
     counts = pipe.count.cpu().numpy().astype(int)
     K_sum = int(counts.sum())
     T = int(pipe.cu[-1].item())
@@ -391,6 +396,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--launch-list", action="store_true",
+                    help="set up, warm up and run one more step only (for an ncu launch list)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -1,0 +1,82 @@
+"""Small, self-contained invocations of one stage of the path, sized for
+`ncu --set full` captures (a few GB on the device at most, a handful of
+launches).  Shapes are those of the 16-image LLaVA-1.5-7B-shaped batch.
+
+    python -m paper_2609_13804_gb300.profile_case gemm       # 1 decoder layer, T = 1791 (4 GEMMs)
+    python -m paper_2609_13804_gb300.profile_case select     # selection from a given memory H
+    python -m paper_2609_13804_gb300.profile_case compact    # compaction of the batch
+    python -m paper_2609_13804_gb300.profile_case attention  # 1 decoder layer, like gemm
+
+Each case runs its stage twice (the second launch set is the one to capture
+with `-s`).
+"""
+import dataclasses
+import sys
+
+import numpy as np
+
+
+def main(case: str):
+    import torch
+
+    from paper_2609_13804_gb300 import binding as B
+    from paper_2609_13804_gb300 import synth as S
+
+    dev = torch.device("cuda", 0)
+    w = S.llava15_7b_b16()
+    counts = S.target_counts(w)
+    if case in ("gemm", "attention"):
+        m = dataclasses.replace(w.model, proj_kind="none", proj_in=w.model.d)
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(1)
+
+        def rnd(shape):
+            return (torch.randn(shape, device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+
+        qkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
+        L = {"Wqkv": rnd((qkv, m.d)), "Wo": rnd((m.d, m.n_heads * m.head_dim)), "Wgu": rnd((2 * m.ffn, m.d)),
+             "Wdown": rnd((m.d, m.ffn)), "attn_norm": torch.ones(m.d, device=dev),
+             "mlp_norm": torch.ones(m.d, device=dev)}
+        head = {"final_norm": torch.ones(m.d, device=dev), "proj_W1": None, "proj_W2": None}
+        model = B.Model(m, None, None, dev, max_pos=512, device_weights={"layers": [L], "head": head})
+        lens = [int(k) + 48 for k in counts]
+        T = sum(lens)
+        cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
+        pos = torch.tensor(np.concatenate([np.arange(n) for n in lens]), dtype=torch.int32, device=dev)
+        x = (torch.randn((T, m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+        ws = None
+        for _ in range(2):
+            out = B.sp_prefill(model, x=x, cu_seqlens=cu, pos=pos, B=len(lens), T_cap=T, max_seqlen_cap=max(lens),
+                               ws=ws)
+            ws = out["_ws"]
+        torch.cuda.synchronize()
+    elif case == "select":
+        s = S.SelectorShape(D=w.selector.D, D_text=w.selector.D_text, h=w.selector.h, n_enc_layers=0)
+        sel = S.make_selector_weights(w)
+        H = S.make_memory(w)
+        selector = B.Selector(s, sel, dev)
+        Hd = B.dev_f32(H, dev)
+        bias = B.dev_f32(np.full(w.B, -1e30), dev)   # every episode runs to its cap of 192
+        ws = None
+        for _ in range(2):
+            r = B.sp_select(selector, w.n_vis, w.n_txt, H=Hd, stop_bias=bias, k_max=w.k_max, traces=False, ws=ws)
+            ws = r["_ws"]
+        torch.cuda.synchronize()
+    elif case == "compact":
+        X = B.dev_bf16(S.bf16_round(S.normal(w.seed, "X", (sum(w.n_vis), 1024))), dev)
+        E = B.dev_bf16(S.bf16_round(S.normal(w.seed, "E", (sum(w.n_txt), 4096), 0.02)), dev)
+        k_cap = 192
+        idx = torch.full((w.B, k_cap), -1, dtype=torch.int32, device=dev)
+        for b, k in enumerate(counts):
+            idx[b, :k] = torch.arange(0, 576, 576 // max(int(k), 1), device=dev)[:k].to(torch.int32)
+        cnt = torch.tensor(counts, dtype=torch.int32, device=dev)
+        for _ in range(2):
+            B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=cnt, k_cap=k_cap, projector_mode=True)
+        torch.cuda.synchronize()
+    else:
+        raise SystemExit(f"unknown case {case}")
+    print("ok", case)
+
+
+if __name__ == "__main__":
+    main(sys.argv[1] if len(sys.argv) > 1 else "gemm")

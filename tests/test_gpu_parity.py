@@ -314,8 +314,9 @@ def test_prefill_llava15_b16_32layers_sampled(B):
     sequences (kept counts 16..192 + 48 text tokens).  The oracle evaluates two
     of the sequences (the shortest and the longest); attention never crosses a
     sequence, so their rows are exact to compare."""
+    import dataclasses
     w = S.llava15_7b_b16()
-    m = w.model
+    m = dataclasses.replace(w.model, proj_kind="none", proj_in=w.model.d)
     k = S.target_counts(w)
     lens = [int(x) + 48 for x in k]
     T = sum(lens)
