@@ -44,9 +44,16 @@ def main(case: str):
         cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
         pos = torch.tensor(np.concatenate([np.arange(n) for n in lens]), dtype=torch.int32, device=dev)
         x = (torch.randn((T, m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+        # the caps of the pipeline (k_cap 192 per image) so tile widths match the benchmark's launches
+        T_cap = sum(min(n, w.k_max) + t for n, t in zip(w.n_vis, w.n_txt))
+        len_cap = max(min(n, w.k_max) + t for n, t in zip(w.n_vis, w.n_txt))
+        xc = torch.zeros((T_cap, m.d), dtype=torch.bfloat16, device=dev)
+        xc[:T] = x
+        pc = torch.zeros(T_cap, dtype=torch.int32, device=dev)
+        pc[:T] = pos
         ws = None
         for _ in range(2):
-            out = B.sp_prefill(model, x=x, cu_seqlens=cu, pos=pos, B=len(lens), T_cap=T, max_seqlen_cap=max(lens),
+            out = B.sp_prefill(model, x=xc, cu_seqlens=cu, pos=pc, B=len(lens), T_cap=T_cap, max_seqlen_cap=len_cap,
                                ws=ws)
             ws = out["_ws"]
         torch.cuda.synchronize()
