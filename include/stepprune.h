@@ -206,6 +206,26 @@ SP_API size_t sp_select_workspace(const sp_selector* s, const sp_select_in* in);
 SP_API sp_status sp_select(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
                     void* workspace, size_t workspace_bytes, sp_stream stream);
 
+/*
+ * sp_select without a caller workspace.  The paper has no counterpart: this is
+ * for callers that cannot allocate device memory (a plug-in whose host
+ * application owns all device memory, a plain-C caller with no allocator, a
+ * path that may not pay for cudaMalloc).  It runs the same selection as
+ * sp_select; its scratch is one static device array of
+ * SP_SELECT_NOALLOC_SCRATCH_BYTES that every GPU loading the library holds
+ * until exit.  Inputs and outputs are still the caller's.
+ *   - A batch whose sp_select_workspace() exceeds that size is rejected with
+ *     SP_ERR_WORKSPACE before any launch.
+ *   - It calls no cudaMalloc / cudaFree and no allocating library routine.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls share the array and it keeps the last call's contents: calls
+ *     whose GPU work overlaps (several streams or threads) race; serialise them.
+ */
+#define SP_SELECT_NOALLOC_SCRATCH_BYTES (64u << 20)
+SP_API sp_status sp_select_noalloc(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
+                                   sp_stream stream);
+
 /* ------------------------------------------------------------------------ */
 /* Compaction (Algorithm 1 step 5: X_S = Gather(X, S), then [X_S; text]).    */
 /* ------------------------------------------------------------------------ */

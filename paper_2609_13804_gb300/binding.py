@@ -32,8 +32,9 @@ EXPORTS = [
     "sp_num_episodes", "sp_select_workspace", "sp_select", "sp_packed_cap", "sp_compact", "sp_model_create",
     "sp_model_destroy", "sp_project_workspace", "sp_project", "sp_prefill_workspace", "sp_prefill",
     "sp_pipeline_workspace", "sp_pipeline", "sp_pipeline_host_workspace", "sp_pipeline_host",
-    "sp_profile_begin", "sp_profile_end",
+    "sp_profile_begin", "sp_profile_end", "sp_select_noalloc",
 ]
+SP_SELECT_NOALLOC_SCRATCH_BYTES = 64 << 20
 
 P = C.c_void_p
 FP = C.POINTER(C.c_float)
@@ -140,6 +141,7 @@ def lib():
         "sp_pipeline": (C.c_int, [P, P, C.POINTER(sp_pipeline_io), P, C.c_size_t, P]),
         "sp_pipeline_host_workspace": (C.c_size_t, [P, P, C.POINTER(sp_pipeline_host_io)]),
         "sp_pipeline_host": (C.c_int, [P, P, C.POINTER(sp_pipeline_host_io), P, C.c_size_t, P]),
+        "sp_select_noalloc": (C.c_int, [P, C.POINTER(sp_select_in), C.POINTER(sp_select_out), P]),
         "sp_profile_begin": (C.c_int, [C.c_int]),
         "sp_profile_end": (C.c_int, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]),
@@ -286,9 +288,11 @@ def _select_in(n_vis, n_txt, X, E_text, H, stop_bias, group_size, g, k_max, keep
 
 
 def sp_select(sel: Selector, n_vis, n_txt, *, stop_bias, X=None, E_text=None, H=None, group_size=0, g=1,
-              k_max=192, k_cap=None, traces=True, memory=False, stream=None, ws=None) -> Dict:
+              k_max=192, k_cap=None, traces=True, memory=False, stream=None, ws=None,
+              no_alloc=False) -> Dict:
     """Runs sp_select; returns device tensors idx [B, k_cap], count [B] and, with
-    traces, order / ep_count / margin / gap / rounds / err."""
+    traces, order / ep_count / margin / gap / rounds / err.  no_alloc=True calls
+    sp_select_noalloc instead (no workspace; the library's static scratch)."""
     torch = _torch()
     dev = sel.device
     keep: List = []
@@ -311,6 +315,10 @@ def sp_select(sel: Selector, n_vis, n_txt, *, stop_bias, X=None, E_text=None, H=
     o = sp_select_out(ptr(out["idx"]), int(k_cap), ptr(out["count"]), ptr(out.get("order")),
                       ptr(out.get("ep_count")), ptr(out.get("margin")), ptr(out.get("gap")),
                       ptr(out.get("rounds")), ptr(out.get("memory")), ptr(out["err"]))
+    if no_alloc:
+        _check(lib().sp_select_noalloc(sel.handle, C.byref(inp), C.byref(o), _stream(stream)), "sp_select_noalloc")
+        out["k_cap"] = k_cap
+        return out
     if ws is None:
         ws = workspace(lib().sp_select_workspace(sel.handle, C.byref(inp)), dev)
     _check(lib().sp_select(sel.handle, C.byref(inp), C.byref(o), ptr(ws), ws.numel(), _stream(stream)), "sp_select")

@@ -528,6 +528,27 @@ sp_status sp_select(const sp_selector* s, const sp_select_in* in, const sp_selec
   return select_impl(s, in, out, ws, ws_bytes, (cudaStream_t)stream);
 }
 
+}  // extern "C"
+
+namespace sp {
+sp_status report(sp_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+sp_status select_with_workspace(const sp_selector* s, const sp_select_in* in, const sp_select_out* out, void* ws,
+                                size_t ws_bytes, cudaStream_t st) {
+  return select_impl(s, in, out, ws, ws_bytes, st);
+}
+}  // namespace sp
+
+extern "C" {
+
 // ------------------------------------------------------------------ compaction
 
 static sp_status compact_impl(const sp_compact_in* in, const sp_compact_out* out, cudaStream_t st) {

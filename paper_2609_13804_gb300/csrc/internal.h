@@ -128,6 +128,13 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
 cudaError_t restore_launch(const BatchDesc& bd, const int* order, const int* ep_count, int k_max,
                            int* idx, int k_cap, int* count, int* err, cudaStream_t st);
 
+// ------------------------------------------------------------- entry-point helpers (api.cu)
+// Records a thread-local error message (sp_last_error) and returns `s`.
+sp_status report(sp_status s, const char* fmt, ...);
+// sp_select on an explicit scratch region (used by sp_select_noalloc).
+sp_status select_with_workspace(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
+                                void* ws, size_t ws_bytes, cudaStream_t st);
+
 // ------------------------------------------------------------- compaction
 cudaError_t compact_launch(const BatchDesc& bd, const void* X, int W_vis, const void* text, int W_txt,
                            const int* idx, int k_cap, const int* count, void* packed, int* cu,
