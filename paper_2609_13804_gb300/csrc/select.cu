@@ -6,7 +6,10 @@
 // candidates are split into C contiguous slices; each CTA keeps its slice of
 // the folded pointer keys in shared memory for the whole episode.  A round:
 //   1. attention of the last history position over the history: CTA c takes
-//      positions c, c+C, ... and writes a partial (max, sum, weighted values);
+//      positions c, c+C, ...; each warp loads all rows it needs for the round
+//      at once (query, key and value rows of its positions) so the round pays
+//      one L2 latency, and the warps' partials (max, sum, weighted values) are
+//      folded into the CTA's partial;
 //   2. cluster barrier; every CTA merges the C partials read over DSMEM in rank
 //      order (so all CTAs hold bitwise-identical results), adds the residual and
 //      applies LN2 -> pointer query;
@@ -40,7 +43,7 @@ constexpr int NW = NT / 32;
 constexpr int GMAX = 16;  // largest g; lists hold g + 1 entries
 
 struct SelSmem {
-  size_t kt, part_o, part_ml, top_v, top_i, q, u, xp, lg, taken, hist, sc, misc, total;
+  size_t kt, stopkt, wpart_o, wpart_ml, part_o, part_ml, top_v, top_i, u, xp, lg, taken, hist, misc, total;
 };
 
 __host__ __device__ inline size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
@@ -48,18 +51,20 @@ __host__ __device__ inline size_t al16(size_t x) { return (x + 15) & ~size_t(15)
 __host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C, bool keys_in_smem) {
   SelSmem L;
   size_t o = 0;
+  (void)C;
   L.kt = o;       o += al16(keys_in_smem ? (size_t)n_loc * h * 4 : 0);
+  L.stopkt = o;   o += al16((size_t)h * 4);
+  L.wpart_o = o;  o += al16((size_t)NW * h * 4);
+  L.wpart_ml = o; o += al16((size_t)NW * 2 * 4);
   L.part_o = o;   o += al16((size_t)2 * h * 4);
   L.part_ml = o;  o += al16(2 * 2 * 4);
   L.top_v = o;    o += al16(2 * (GMAX + 1) * 4);
   L.top_i = o;    o += al16(2 * (GMAX + 1) * 4);
-  L.q = o;        o += al16((size_t)h * 4);
   L.u = o;        o += al16((size_t)h * 4);
   L.xp = o;       o += al16((size_t)h * 4);
   L.lg = o;       o += al16((size_t)n_loc * 4);
   L.taken = o;    o += al16((size_t)n_loc);
   L.hist = o;     o += al16((size_t)(k_max + 1) * 4);
-  L.sc = o;       o += al16((size_t)((k_max + 1 + C - 1) / C + 1) * 4);
   L.misc = o;     o += al16(128 * 4);
   L.total = o;
   return L;
@@ -86,8 +91,15 @@ SP_DEVINL float block_sum(float v, float* red) {
   return warp_sum(t);
 }
 
+SP_DEVINL float dot4(const float4& a, const float4& b) { return a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w; }
+
+// HV = h / 128: float4 slices per lane of an h-vector (lane holds elements
+// 4 (lane + 32 k) .. +3, k < HV).  P = history positions a warp loads at once.
+template <int HV>
 __global__ void __launch_bounds__(NT, 1)
 select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in_smem) {
+  constexpr int P = (16 / HV) > 0 ? 16 / HV : 1;
+  constexpr int DPT = (HV * 128) / NT > 0 ? (HV * 128) / NT : 1;  // dims per thread in the merges
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)cluster.num_blocks();
   const int rank = (int)cluster.block_rank();
@@ -114,45 +126,44 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   extern __shared__ __align__(16) uint8_t sm[];
   const SelSmem L = sel_layout(h, n_loc_max, k_max, C, keys_in_smem != 0);
   float* kt_s = reinterpret_cast<float*>(sm + L.kt);
+  float* stopkt = reinterpret_cast<float*>(sm + L.stopkt);
+  float* wpart_o = reinterpret_cast<float*>(sm + L.wpart_o);
+  float* wpart_ml = reinterpret_cast<float*>(sm + L.wpart_ml);
   float* part_o = reinterpret_cast<float*>(sm + L.part_o);
   float* part_ml = reinterpret_cast<float*>(sm + L.part_ml);
   float* top_v = reinterpret_cast<float*>(sm + L.top_v);
   int* top_i = reinterpret_cast<int*>(sm + L.top_i);
-  float* q_s = reinterpret_cast<float*>(sm + L.q);
   float* u_s = reinterpret_cast<float*>(sm + L.u);
   float* xp_s = reinterpret_cast<float*>(sm + L.xp);
   float* lg = reinterpret_cast<float*>(sm + L.lg);
   uint8_t* taken = sm + L.taken;
   int* hist = reinterpret_cast<int*>(sm + L.hist);
-  float* sc = reinterpret_cast<float*>(sm + L.sc);
   float* misc = reinterpret_cast<float*>(sm + L.misc);
   float* red = misc;                                  // [0, 32)
   float* rm = misc + 32;                              // [32, 48)  peer maxima
   float* rl = misc + 48;                              // [48, 64)  peer sums
   float* gtop_v = misc + 64;                          // [64, 81)
   int* gtop_i = reinterpret_cast<int*>(misc + 96);    // [96, 113)
-  float* stop_raw_s = misc + 120;
 
-  // stage this CTA's slice of the folded keys
+  // stage this CTA's slice of the folded keys and the STOP key
   const float* KT = a.KT;
+  const int h4 = h >> 2;
   if (keys_in_smem) {
-    const int h4 = h >> 2;
     for (int i = tid; i < nl * h4; i += NT) {
       const int j = i / h4, c = i % h4;
       reinterpret_cast<float4*>(kt_s)[(size_t)j * h4 + c] =
           __ldg(reinterpret_cast<const float4*>(KT + (size_t)(row0 + j0 + j) * a.ldkt) + c);
     }
   }
+  for (int i = tid; i < h4; i += NT)
+    reinterpret_cast<float4*>(stopkt)[i] = __ldg(reinterpret_cast<const float4*>(KT + (size_t)a.stop_row * a.ldkt) + i);
   for (int j = tid; j < n_loc_max; j += NT) taken[j] = 0;
   if (tid == 0) hist[0] = a.start_row;
   const float bias = __ldg(a.stop_bias + e);
   const size_t trace = (size_t)e * (k_max + 1);
   __syncthreads();
 
-  constexpr int MAXV = 8;  // float4 per lane: h <= 1024
-  const int hv = h >> 7;   // float4 per lane (h multiple of 128)
   int nsel = 0, round = 0;
-
   while (nsel < k_max) {
     const int n_avail = n_e - nsel;
     if (n_avail == 0) {  // only STOP remains: it wins this round
@@ -167,32 +178,90 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     const int t = nsel + 1;
     const int last = hist[t - 1];
 
-    // ---- 1. partial causal self-attention of the last position
-    for (int i = tid; i < h; i += NT) q_s[i] = __ldg(a.QS + (size_t)last * a.ldqs + i);
-    __syncthreads();
-    const int np = (rank < t) ? (t - 1 - rank) / C + 1 : 0;
-    for (int k = warp; k < np; k += NW) {
-      const float* kr = a.KS + (size_t)hist[rank + k * C] * a.ldks;
-      float s = 0.f;
-      for (int i = lane; i < h; i += 32) s += q_s[i] * __ldg(kr + i);
-      s = warp_sum(s);
-      if (lane == 0) sc[k] = s;
+    // ---- 1. partial causal self-attention of the last position.  Every load
+    //      of the round (query, residual, owned history rows) is issued at once.
+    float zr[DPT];
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) zr[d] = (tid + d * NT < h) ? __ldg(a.Z + (size_t)last * a.ldz + tid + d * NT) : 0.f;
+    float4 q[HV];
+    const float4* qrow = reinterpret_cast<const float4*>(a.QS + (size_t)last * a.ldqs);
+#pragma unroll
+    for (int k = 0; k < HV; ++k) q[k] = __ldg(qrow + lane + 32 * k);
+    const int np = (rank < t) ? (t - 1 - rank) / C + 1 : 0;  // positions rank, rank + C, ...
+    float m_w = -INFINITY, l_w = 0.f;
+    float4 o_w[HV];
+#pragma unroll
+    for (int k = 0; k < HV; ++k) o_w[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k0 = warp * P; k0 < np; k0 += NW * P) {
+      float4 kr[P][HV], vr[P][HV];
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        if (k0 + pp < np) {
+          const int row = hist[rank + (k0 + pp) * C];
+          const float4* ks = reinterpret_cast<const float4*>(a.KS + (size_t)row * a.ldks);
+          const float4* vt = reinterpret_cast<const float4*>(a.VT + (size_t)row * a.ldvt);
+#pragma unroll
+          for (int k = 0; k < HV; ++k) {
+            kr[pp][k] = __ldg(ks + lane + 32 * k);
+            vr[pp][k] = __ldg(vt + lane + 32 * k);
+          }
+        }
+      }
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        if (k0 + pp < np) {
+          float s = 0.f;
+#pragma unroll
+          for (int k = 0; k < HV; ++k) s += dot4(q[k], kr[pp][k]);
+          s = warp_sum(s);
+          const float mn = fmaxf(m_w, s);
+          const float cw = (m_w == -INFINITY) ? 0.f : expf(m_w - mn);
+          const float ps = expf(s - mn);
+          l_w = l_w * cw + ps;
+#pragma unroll
+          for (int k = 0; k < HV; ++k) {
+            o_w[k].x = o_w[k].x * cw + ps * vr[pp][k].x;
+            o_w[k].y = o_w[k].y * cw + ps * vr[pp][k].y;
+            o_w[k].z = o_w[k].z * cw + ps * vr[pp][k].z;
+            o_w[k].w = o_w[k].w * cw + ps * vr[pp][k].w;
+          }
+          m_w = mn;
+        }
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < HV; ++k) reinterpret_cast<float4*>(wpart_o + warp * h)[lane + 32 * k] = o_w[k];
+    if (lane == 0) {
+      wpart_ml[warp * 2 + 0] = m_w;
+      wpart_ml[warp * 2 + 1] = l_w;
     }
     __syncthreads();
-    float m_c = -INFINITY;
-    for (int k = 0; k < np; ++k) m_c = fmaxf(m_c, sc[k]);
-    float l_c = 0.f;
-    for (int k = 0; k < np; ++k) l_c += expf(sc[k] - m_c);
-    float* po = part_o + buf * h;
-    for (int i = tid; i < h; i += NT) {
-      float acc = 0.f;
-      for (int k = 0; k < np; ++k)
-        acc += expf(sc[k] - m_c) * __ldg(a.VT + (size_t)hist[rank + k * C] * a.ldvt + i);
-      po[i] = acc;
-    }
-    if (tid == 0) {
-      part_ml[buf * 2 + 0] = m_c;
-      part_ml[buf * 2 + 1] = l_c;
+    {  // this CTA's partial from its warps' partials (warp order)
+      float m_c = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) m_c = fmaxf(m_c, wpart_ml[w * 2]);
+      float cw[NW];
+      float l_c = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float mw = wpart_ml[w * 2];
+        cw[w] = (mw == -INFINITY) ? 0.f : expf(mw - m_c);
+        l_c += cw[w] * wpart_ml[w * 2 + 1];
+      }
+      float* po = part_o + buf * h;
+#pragma unroll
+      for (int d = 0; d < DPT; ++d) {
+        const int i = tid + d * NT;
+        if (i >= h) continue;
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) acc += cw[w] * wpart_o[w * h + i];
+        po[i] = acc;
+      }
+      if (tid == 0) {
+        part_ml[buf * 2 + 0] = m_c;
+        part_ml[buf * 2 + 1] = l_c;
+      }
     }
     cluster.sync();
 
@@ -215,28 +284,34 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     }
     const float inv = 1.f / wsum;
     float s_loc = 0.f;
-    for (int i = tid; i < h; i += NT) {
+    float uv[DPT];
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const int i = tid + d * NT;
+      uv[d] = 0.f;
+      if (i >= h) continue;
+      float ro[16];
+#pragma unroll
+      for (int r = 0; r < 16; ++r) ro[r] = (r < C) ? cluster.map_shared_rank(part_o, r)[buf * h + i] : 0.f;
       float o = 0.f;
 #pragma unroll
-      for (int r = 0; r < 16; ++r) {
-        if (r < C) {
-          const float* ro = cluster.map_shared_rank(part_o, r);
-          o += wr[r] * ro[buf * h + i];
-        }
-      }
-      const float u = __ldg(a.Z + (size_t)last * a.ldz + i) + o * inv;
-      u_s[i] = u;
-      s_loc += u;
+      for (int r = 0; r < 16; ++r) o += wr[r] * ro[r];
+      uv[d] = zr[d] + o * inv;
+      s_loc += uv[d];
     }
     const float mean = block_sum(s_loc, red) / (float)h;
     float v_loc = 0.f;
-    for (int i = tid; i < h; i += NT) {
-      const float c = u_s[i] - mean;
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const float c = (tid + d * NT < h) ? uv[d] - mean : 0.f;
       v_loc += c * c;
     }
     const float rstd = rsqrtf(block_sum(v_loc, red) / (float)h + a.ln_eps);
-    for (int i = tid; i < h; i += NT) {
-      float x = (u_s[i] - mean) * rstd;
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const int i = tid + d * NT;
+      if (i >= h) continue;
+      float x = (uv[d] - mean) * rstd;
       if (a.ln2_g) x *= __ldg(a.ln2_g + i);
       if (a.ln2_b) x += __ldg(a.ln2_b + i);
       xp_s[i] = x;
@@ -244,10 +319,9 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     __syncthreads();
 
     // ---- 3. logits of the available local candidates and the raw STOP logit
-    float4 xr[MAXV];
+    float4 xr[HV];
 #pragma unroll
-    for (int k = 0; k < MAXV; ++k)
-      if (k < hv) xr[k] = reinterpret_cast<const float4*>(xp_s)[lane + 32 * k];
+    for (int k = 0; k < HV; ++k) xr[k] = reinterpret_cast<const float4*>(xp_s)[lane + 32 * k];
     for (int j = warp; j < nl; j += NW) {
       if (taken[j]) {
         if (lane == 0) lg[j] = -INFINITY;
@@ -257,27 +331,16 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
                                       : reinterpret_cast<const float4*>(KT + (size_t)(row0 + j0 + j) * a.ldkt);
       float s = 0.f;
 #pragma unroll
-      for (int k = 0; k < MAXV; ++k) {
-        if (k < hv) {
-          const float4 kv = kr[lane + 32 * k];
-          s += xr[k].x * kv.x + xr[k].y * kv.y + xr[k].z * kv.z + xr[k].w * kv.w;
-        }
-      }
+      for (int k = 0; k < HV; ++k) s += dot4(xr[k], kr[lane + 32 * k]);
       s = warp_sum(s);
       if (lane == 0) lg[j] = s;
     }
-    if (warp == NW - 1) {
-      const float4* kr = reinterpret_cast<const float4*>(KT + (size_t)a.stop_row * a.ldkt);
+    float stop_raw = 0.f;
+    {
       float s = 0.f;
 #pragma unroll
-      for (int k = 0; k < MAXV; ++k) {
-        if (k < hv) {
-          const float4 kv = __ldg(kr + lane + 32 * k);
-          s += xr[k].x * kv.x + xr[k].y * kv.y + xr[k].z * kv.z + xr[k].w * kv.w;
-        }
-      }
-      s = warp_sum(s);
-      if (lane == 0) *stop_raw_s = s;
+      for (int k = 0; k < HV; ++k) s += dot4(xr[k], reinterpret_cast<const float4*>(stopkt)[lane + 32 * k]);
+      stop_raw = warp_sum(s);  // every warp of every CTA computes the same value
     }
     __syncthreads();
 
@@ -291,7 +354,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           const float v = lg[j];
           if (v == -INFINITY) continue;
           bool ex = false;
-          for (int q = 0; q < r; ++q) ex |= (picked[q] == j);
+          for (int q2 = 0; q2 < r; ++q2) ex |= (picked[q2] == j);
           if (!ex && better(v, j, bv, bi)) { bv = v; bi = j; }
         }
         warp_best(bv, bi);
@@ -316,11 +379,11 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
         ev[k] = -INFINITY;
         ei[k] = INT_MAX;
         if (idx < tot) {
-          const int r = idx / per, s = idx % per;
+          const int r = idx / per, s2 = idx % per;
           const float* rv = cluster.map_shared_rank(top_v, r);
           const int* ri = cluster.map_shared_rank(top_i, r);
-          ev[k] = rv[buf * (GMAX + 1) + s];
-          ei[k] = ri[buf * (GMAX + 1) + s];
+          ev[k] = rv[buf * (GMAX + 1) + s2];
+          ei[k] = ri[buf * (GMAX + 1) + s2];
           if (ei[k] == INT_MAX) ev[k] = -INFINITY;
         }
       }
@@ -341,7 +404,6 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
       }
     }
     __syncthreads();
-    const float stop_raw = *stop_raw_s;
     const float stop_logit = stop_raw + bias;
     const float best = gtop_v[0];
     if (rank == 0 && tid == 0) {
@@ -483,11 +545,18 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
   }
   const int n_loc = (n_max + C - 1) / C;
   const SelSmem L = sel_layout(a.h, n_loc, a.k_max, C, keys_in_smem);
-  cudaError_t r = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)L.total);
+  void (*kern)(const BatchDesc, const SelectArgs, int, int) = nullptr;
+  switch (a.h / 128) {
+    case 1: kern = select_kernel<1>; break;
+    case 2: kern = select_kernel<2>; break;
+    case 4: kern = select_kernel<4>; break;
+    case 8: kern = select_kernel<8>; break;
+    default: return cudaErrorInvalidValue;
+  }
+  cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.total);
   if (r != cudaSuccess) return r;
   if (C > 8) {
-    r = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    r = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (r != cudaSuccess) return r;
   }
   cudaLaunchConfig_t cfg = {};
@@ -503,7 +572,7 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   prof_begin_launch(st);
-  r = cudaLaunchKernelEx(&cfg, select_kernel, bd, a, n_loc, keys_in_smem ? 1 : 0);
+  r = cudaLaunchKernelEx(&cfg, kern, bd, a, n_loc, keys_in_smem ? 1 : 0);
   prof_end_launch(st, SP_K_SELECT, 0.0, 0.0);
   return r;
 }
