@@ -28,6 +28,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 from paper_2609_13804_gb300 import synth as S  # noqa: E402
+from paper_2609_13804_gb300.replicas import max_over_ranks  # noqa: E402
 
 METRIC = "pruned-prefill ms/batch"
 UNIT = "ms/batch"
@@ -267,11 +268,7 @@ def run_ours(args):
         ev1.record(st)
         barrier()
     prof = B.sp_profile_end()
-    ms_step = ev0.elapsed_time(ev1) / args.steps
-    if dist:
-        t = torch.tensor([ms_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_step = float(t.item())
+    ms_step = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, dev)
     value = ms_step / world
     launches = sum(v["launches"] for v in prof.values()) // args.steps
     gemm_ms = prof["gemm"]["ms"] / args.steps
@@ -324,6 +321,10 @@ def run_ours(args):
     full_idx = torch.arange(576, dtype=torch.int32, device=dev).repeat(w.B, 1).contiguous()
     full_cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
     full_ms = timed(lambda: prefill_stage(full_idx, full_cnt, 576), reps=3)
+    # compaction at a bandwidth-sized case: every visual token kept (the full prefix)
+    full_compact_ms = timed(lambda: do_compact(full_idx, full_cnt, 576))
+    full_T = sum(w.n_vis) + sum(w.n_txt)
+    full_comp_bytes = 2.0 * (sum(w.n_vis) * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + full_T)
 
     # ---- end to end from host buffers (copies inside the timed region)
     Xh = X.cpu().pin_memory()
@@ -343,11 +344,7 @@ def run_ours(args):
         pipe.host(Xh, Eh, bh, oi, oc, ocu, oh)
     b_.record()
     barrier()
-    e2e_ms = a.elapsed_time(b_) / e2e_steps
-    if dist:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(a.elapsed_time(b_) / e2e_steps, dev)
     h2d = Xh.numel() * 2 + Eh.numel() * 2 + bh.numel() * 4
     d2h = oi.numel() * 4 + oc.numel() * 4 + ocu.numel() * 4 + oh.numel() * 4
 
@@ -377,6 +374,8 @@ def run_ours(args):
             "stages_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()},
             "select_us_per_image": 1e3 * select_ms / w.B,
             "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,
+            "compaction_full_prefix_gbs": full_comp_bytes / (full_compact_ms * 1e-3) / 1e9,
+            "compaction_full_prefix_hbm_frac": full_comp_bytes / (full_compact_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
             "pruned_prefill_ms": pruned_ms,
             "full_prefix_prefill_ms": full_ms,
             "speedup_prefill": full_ms / pruned_ms,

@@ -66,6 +66,7 @@ struct GemmB {
 };
 
 bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg);
+int gemm_pair_policy(int M_cap, int N_acc, int kind);
 
 // C[M, N] = A[M, K] B[N, K]^T with the given epilogue.  A's tensor map has box
 // rows 128.  M_dev (device int, may be NULL) bounds the rows actually computed;
