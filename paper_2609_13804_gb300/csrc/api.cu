@@ -517,7 +517,7 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   a.err = err;
   bool keys_smem = true;
   size_t smem = 0;
-  const int C = select_cluster_size(p.bd, h, &keys_smem, &smem);
+  const int C = select_cluster_size(p.bd, h, in->k_max, &keys_smem, &smem);
   SP_CUDA(select_launch(p.bd, p.E, a, C, keys_smem, smem, st), "selection");
   SP_CUDA(restore_launch(p.bd, a.order, a.ep_count, in->k_max, out->idx, out->k_cap, out->count, err, st), "restore");
   return SP_OK;

@@ -123,7 +123,7 @@ struct SelectArgs {
   int* err;
 };
 
-int select_cluster_size(const BatchDesc& bd, int h, bool* keys_in_smem, size_t* smem_bytes);
+int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes);
 cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs& a,
                           int cluster, bool keys_in_smem, size_t smem_bytes, cudaStream_t st);
 cudaError_t restore_launch(const BatchDesc& bd, const int* order, const int* ep_count, int k_max,

@@ -7,24 +7,27 @@
 // the folded pointer keys in shared memory for the whole episode.  A round:
 //   1. attention of the last history position over the history: CTA c takes
 //      positions c, c+C, ...; each warp loads all rows it needs for the round
-//      at once (query, key and value rows of its positions) so the round pays
-//      one L2 latency, and the warps' partials (max, sum, weighted values) are
-//      folded into the CTA's partial;
-//   2. cluster barrier; every CTA merges the C partials read over DSMEM in rank
-//      order (so all CTAs hold bitwise-identical results), adds the residual and
-//      applies LN2 -> pointer query;
-//   3. every CTA scores its available candidates from shared memory and keeps
-//      its top g+1 (logit desc, index asc); the raw STOP logit is computed by
-//      every CTA identically;
+//      at once (query, key and value rows of its positions), the warps'
+//      partials (max, sum, weighted values) fold into the CTA's partial, which
+//      the CTA pushes into its slot in every CTA's shared memory;
+//   2. cluster barrier; every CTA merges the C partials from its own shared
+//      memory in rank order (so all CTAs hold bitwise-identical results), adds
+//      the residual and applies LN2 -> pointer query;
+//   3. every CTA scores its available candidates from shared memory (four per
+//      warp iteration, shuffle reductions interleaved), each warp keeping a
+//      running top g+1 (logit desc, index asc); warp 0 merges them and pushes
+//      the CTA's list into every CTA; the raw STOP logit is computed by every
+//      CTA identically;
 //   4. cluster barrier; every CTA merges the C lists, takes the same decision
 //      (STOP iff strictly above the best available visual logit, else TopG
 //      truncated to the cap), masks its own slice and extends the history.
+// Exchanges are pushes (remote stores before the barrier, local loads after),
+// double-buffered by round parity, so two cluster barriers per round suffice.
 // The decoder matrices are folded on the host side of the ABI so that no
 // matrix-vector product remains inside the loop:
 //   QS = x Wq_s^T / sqrt(h), KS = x Wk_s^T, VT = x (Wo_s Wv_s)^T   (x = LN1(W_in m))
 //   KT = m (Wq_p^T Wk_p)^T / sqrt(h),  so  l(j) = <LN2(u), KT_j>,
 //   u = Z_last + sum_i softmax_i(<QS_last, KS_i>) VT_i.
-// Double-buffered exchange slots make two cluster barriers per round enough.
 #include <cooperative_groups.h>
 
 #include <climits>
@@ -43,26 +46,31 @@ constexpr int NW = NT / 32;
 constexpr int GMAX = 16;  // largest g; lists hold g + 1 entries
 
 struct SelSmem {
-  size_t kt, stopkt, wpart_o, wpart_ml, part_o, part_ml, top_v, top_i, u, xp, lg, taken, hist, misc, total;
+  size_t kt, lgp, stopkt, wpart_o, wpart_ml, all_o, all_ml, wtop_v, wtop_i, all_tv, all_ti, xp, taken, hist, misc,
+      total;
 };
 
 __host__ __device__ inline size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
 
+// Shared-memory layout.  The all_* slots receive, per round parity, one entry
+// per CTA of the cluster, written remotely by that CTA (push exchange).
 __host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C, bool keys_in_smem) {
   SelSmem L;
   size_t o = 0;
-  (void)C;
-  L.kt = o;       o += al16(keys_in_smem ? (size_t)n_loc * h * 4 : 0);
+  // keys in shared memory: dims-major, (n_loc + 1) columns (the last one is
+  // STOP's key), float4 (d4, j) at d4 * (n_loc + 1) + j
+  L.kt = o;       o += al16(keys_in_smem ? (size_t)(n_loc + 1) * h * 4 : 0);
+  L.lgp = o;      o += al16(keys_in_smem ? (size_t)NW * (n_loc + 1) * 4 : 0);
   L.stopkt = o;   o += al16((size_t)h * 4);
   L.wpart_o = o;  o += al16((size_t)NW * h * 4);
   L.wpart_ml = o; o += al16((size_t)NW * 2 * 4);
-  L.part_o = o;   o += al16((size_t)2 * h * 4);
-  L.part_ml = o;  o += al16(2 * 2 * 4);
-  L.top_v = o;    o += al16(2 * (GMAX + 1) * 4);
-  L.top_i = o;    o += al16(2 * (GMAX + 1) * 4);
-  L.u = o;        o += al16((size_t)h * 4);
+  L.all_o = o;    o += al16((size_t)2 * C * h * 4);
+  L.all_ml = o;   o += al16((size_t)2 * C * 2 * 4);
+  L.wtop_v = o;   o += al16((size_t)NW * (GMAX + 1) * 4);
+  L.wtop_i = o;   o += al16((size_t)NW * (GMAX + 1) * 4);
+  L.all_tv = o;   o += al16((size_t)2 * C * (GMAX + 1) * 4);
+  L.all_ti = o;   o += al16((size_t)2 * C * (GMAX + 1) * 4);
   L.xp = o;       o += al16((size_t)h * 4);
-  L.lg = o;       o += al16((size_t)n_loc * 4);
   L.taken = o;    o += al16((size_t)n_loc);
   L.hist = o;     o += al16((size_t)(k_max + 1) * 4);
   L.misc = o;     o += al16(128 * 4);
@@ -81,31 +89,140 @@ SP_DEVINL void warp_best(float& v, int& i) {
   }
 }
 
-SP_DEVINL float block_sum(float v, float* red) {
-  v = warp_sum(v);
+// Sums of U independent per-lane values across the warp, reductions interleaved.
+template <int U>
+SP_DEVINL void warp_sum_n(float (&v)[U]) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) v[u] += __shfl_xor_sync(0xffffffffu, v[u], o);
+  }
+}
+
+// Block-wide sums of U values per thread (red: NW * U floats); every thread
+// gets the totals, summed in warp order.
+template <int U>
+SP_DEVINL void block_sum_n(float (&v)[U], float* red) {
+  warp_sum_n<U>(v);
   const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) red[w * U + u] = v[u];
+  }
   __syncthreads();
-  if (l == 0) red[w] = v;
-  __syncthreads();
-  float t = (l < NW) ? red[l] : 0.f;
-  return warp_sum(t);
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k < NW; ++k) t += red[k * U + u];
+    v[u] = t;
+  }
 }
 
 SP_DEVINL float dot4(const float4& a, const float4& b) { return a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w; }
 
+// Keeps the best `keep` (value, index) pairs seen so far, best first, in a list
+// of capacity GL.  All lanes of a warp hold the same list.
+template <int GL>
+SP_DEVINL void top_insert(float (&tv)[GL], int (&ti)[GL], float v, int j, int keep) {
+  // the current last kept entry, selected with compile-time indices only so the
+  // list stays in registers
+  float lv = tv[0];
+  int li = ti[0];
+#pragma unroll
+  for (int k = 1; k < GL; ++k) {
+    if (k == keep - 1) {
+      lv = tv[k];
+      li = ti[k];
+    }
+  }
+  if (!better(v, j, lv, li)) return;
+#pragma unroll
+  for (int k = GL - 1; k > 0; --k) {
+    if (k < keep) {
+      if (better(v, j, tv[k - 1], ti[k - 1])) {
+        tv[k] = tv[k - 1];
+        ti[k] = ti[k - 1];
+      } else if (better(v, j, tv[k], ti[k])) {
+        tv[k] = v;
+        ti[k] = j;
+      }
+    }
+  }
+  if (better(v, j, tv[0], ti[0])) {
+    tv[0] = v;
+    ti[0] = j;
+  }
+}
+
+// Order-preserving 32-bit key of a float (larger float -> larger key; -0 is
+// taken as +0); 0 is reserved for "no entry".
+SP_DEVINL uint32_t fkey(float v) {
+  const uint32_t u = __float_as_uint(v + 0.0f);
+  return (u >> 31) ? ~u : (u | 0x80000000u);
+}
+SP_DEVINL float fkey_inv(uint32_t k) {
+  if (k == 0u) return -INFINITY;
+  return __uint_as_float((k >> 31) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// Warp-wide selection of the best `per` of `tot` contiguous (value, index)
+// entries (value desc, index asc), E entries per lane at most; every lane gets
+// the result, best first.  Each pick is two redux.sync reductions: the largest
+// key, then the smallest index holding it.
+template <int GL, int E>
+SP_DEVINL void warp_merge_lists(const float* vin, const int* iin, int tot, int per, float (&out_v)[GL],
+                                int (&out_i)[GL]) {
+  const int lane = threadIdx.x & 31;
+  uint32_t key[E];
+  int ei[E];
+#pragma unroll
+  for (int k = 0; k < E; ++k) {
+    const int idx = lane + 32 * k;
+    key[k] = 0u;
+    ei[k] = INT_MAX;
+    if (idx < tot) {
+      ei[k] = iin[idx];
+      if (ei[k] != INT_MAX) key[k] = fkey(vin[idx]);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < GL; ++r) {
+    out_v[r] = -INFINITY;
+    out_i[r] = INT_MAX;
+    if (r < per) {
+      uint32_t bk = key[0];
+      int bi = ei[0];
+#pragma unroll
+      for (int k = 1; k < E; ++k)
+        if (key[k] > bk || (key[k] == bk && ei[k] < bi)) { bk = key[k]; bi = ei[k]; }
+      const uint32_t mk = __reduce_max_sync(0xffffffffu, bk);
+      const int mi = (int)__reduce_min_sync(0xffffffffu, bk == mk ? (uint32_t)bi : 0x7fffffffu);
+      out_v[r] = fkey_inv(mk);
+      out_i[r] = mk ? mi : INT_MAX;
+#pragma unroll
+      for (int k = 0; k < E; ++k)
+        if (ei[k] == mi) { key[k] = 0u; ei[k] = INT_MAX; }
+    }
+  }
+}
+
 // HV = h / 128: float4 slices per lane of an h-vector (lane holds elements
-// 4 (lane + 32 k) .. +3, k < HV).  P = history positions a warp loads at once.
-template <int HV>
+// 4 (lane + 32 k) .. +3, k < HV).  GL = capacity of the per-round top lists
+// (g + 1 <= GL).  P = history positions a warp loads at once.
+template <int HV, int GL>
 __global__ void __launch_bounds__(NT, 1)
 select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in_smem) {
   constexpr int P = (16 / HV) > 0 ? 16 / HV : 1;
   constexpr int DPT = (HV * 128) / NT > 0 ? (HV * 128) / NT : 1;  // dims per thread in the merges
+  constexpr int U = 4;                                          // candidates per warp iteration
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)cluster.num_blocks();
   const int rank = (int)cluster.block_rank();
   const int e = blockIdx.x / C;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int h = a.h, k_max = a.k_max, g = a.g;
+  const int per = g + 1;
 
   // episode geometry
   int lo = 0, hi = bd.B - 1;
@@ -126,33 +243,34 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   extern __shared__ __align__(16) uint8_t sm[];
   const SelSmem L = sel_layout(h, n_loc_max, k_max, C, keys_in_smem != 0);
   float* kt_s = reinterpret_cast<float*>(sm + L.kt);
+  float* lgp = reinterpret_cast<float*>(sm + L.lgp);
   float* stopkt = reinterpret_cast<float*>(sm + L.stopkt);
   float* wpart_o = reinterpret_cast<float*>(sm + L.wpart_o);
   float* wpart_ml = reinterpret_cast<float*>(sm + L.wpart_ml);
-  float* part_o = reinterpret_cast<float*>(sm + L.part_o);
-  float* part_ml = reinterpret_cast<float*>(sm + L.part_ml);
-  float* top_v = reinterpret_cast<float*>(sm + L.top_v);
-  int* top_i = reinterpret_cast<int*>(sm + L.top_i);
-  float* u_s = reinterpret_cast<float*>(sm + L.u);
+  float* all_o = reinterpret_cast<float*>(sm + L.all_o);
+  float* all_ml = reinterpret_cast<float*>(sm + L.all_ml);
+  float* wtop_v = reinterpret_cast<float*>(sm + L.wtop_v);
+  int* wtop_i = reinterpret_cast<int*>(sm + L.wtop_i);
+  float* all_tv = reinterpret_cast<float*>(sm + L.all_tv);
+  int* all_ti = reinterpret_cast<int*>(sm + L.all_ti);
   float* xp_s = reinterpret_cast<float*>(sm + L.xp);
-  float* lg = reinterpret_cast<float*>(sm + L.lg);
   uint8_t* taken = sm + L.taken;
   int* hist = reinterpret_cast<int*>(sm + L.hist);
   float* misc = reinterpret_cast<float*>(sm + L.misc);
-  float* red = misc;                                  // [0, 32)
-  float* rm = misc + 32;                              // [32, 48)  peer maxima
-  float* rl = misc + 48;                              // [48, 64)  peer sums
+  float* red = misc;                                  // [0, 16)  NW x 2
   float* gtop_v = misc + 64;                          // [64, 81)
   int* gtop_i = reinterpret_cast<int*>(misc + 96);    // [96, 113)
 
   // stage this CTA's slice of the folded keys and the STOP key
   const float* KT = a.KT;
   const int h4 = h >> 2;
+  const int LD = n_loc_max + 1;  // columns of the dims-major key block
   if (keys_in_smem) {
-    for (int i = tid; i < nl * h4; i += NT) {
+    for (int i = tid; i < (nl + 1) * h4; i += NT) {
       const int j = i / h4, c = i % h4;
-      reinterpret_cast<float4*>(kt_s)[(size_t)j * h4 + c] =
-          __ldg(reinterpret_cast<const float4*>(KT + (size_t)(row0 + j0 + j) * a.ldkt) + c);
+      const int row = (j < nl) ? row0 + j0 + j : a.stop_row;  // column nl: STOP
+      reinterpret_cast<float4*>(kt_s)[(size_t)c * LD + j] =
+          __ldg(reinterpret_cast<const float4*>(KT + (size_t)row * a.ldkt) + c);
     }
   }
   for (int i = tid; i < h4; i += NT)
@@ -162,6 +280,21 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   const float bias = __ldg(a.stop_bias + e);
   const size_t trace = (size_t)e * (k_max + 1);
   __syncthreads();
+
+  // query / residual rows of the last history position, loaded one round ahead
+  float zr[DPT];
+  float4 q[HV];
+  float shift;
+  auto load_last = [&](int row) {
+    const float* zrow = a.Z + (size_t)row * a.ldz;
+    shift = __ldg(zrow);  // common shift of the LN moments (any value near the data)
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) zr[d] = (tid + d * NT < h) ? __ldg(zrow + tid + d * NT) : 0.f;
+    const float4* qrow = reinterpret_cast<const float4*>(a.QS + (size_t)row * a.ldqs);
+#pragma unroll
+    for (int k = 0; k < HV; ++k) q[k] = __ldg(qrow + lane + 32 * k);
+  };
+  load_last(a.start_row);
 
   int nsel = 0, round = 0;
   while (nsel < k_max) {
@@ -176,17 +309,10 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     }
     const int buf = round & 1;
     const int t = nsel + 1;
-    const int last = hist[t - 1];
 
-    // ---- 1. partial causal self-attention of the last position.  Every load
-    //      of the round (query, residual, owned history rows) is issued at once.
-    float zr[DPT];
-#pragma unroll
-    for (int d = 0; d < DPT; ++d) zr[d] = (tid + d * NT < h) ? __ldg(a.Z + (size_t)last * a.ldz + tid + d * NT) : 0.f;
-    float4 q[HV];
-    const float4* qrow = reinterpret_cast<const float4*>(a.QS + (size_t)last * a.ldqs);
-#pragma unroll
-    for (int k = 0; k < HV; ++k) q[k] = __ldg(qrow + lane + 32 * k);
+    // ---- 1. partial causal self-attention of the last position (its query and
+    //      residual rows were loaded at the end of the previous round); every
+    //      history row of the round is loaded at once.
     const int np = (rank < t) ? (t - 1 - rank) / C + 1 : 0;  // positions rank, rank + C, ...
     float m_w = -INFINITY, l_w = 0.f;
     float4 o_w[HV];
@@ -207,16 +333,23 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           }
         }
       }
+      float sc[P];
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        sc[pp] = 0.f;
+        if (k0 + pp < np) {
+#pragma unroll
+          for (int k = 0; k < HV; ++k) sc[pp] += dot4(q[k], kr[pp][k]);
+        }
+      }
+      warp_sum_n<P>(sc);
 #pragma unroll
       for (int pp = 0; pp < P; ++pp) {
         if (k0 + pp < np) {
-          float s = 0.f;
-#pragma unroll
-          for (int k = 0; k < HV; ++k) s += dot4(q[k], kr[pp][k]);
-          s = warp_sum(s);
+          const float s = sc[pp];
           const float mn = fmaxf(m_w, s);
-          const float cw = (m_w == -INFINITY) ? 0.f : expf(m_w - mn);
-          const float ps = expf(s - mn);
+          const float cw = (m_w == -INFINITY) ? 0.f : __expf(m_w - mn);
+          const float ps = __expf(s - mn);
           l_w = l_w * cw + ps;
 #pragma unroll
           for (int k = 0; k < HV; ++k) {
@@ -236,19 +369,18 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
       wpart_ml[warp * 2 + 1] = l_w;
     }
     __syncthreads();
-    {  // this CTA's partial from its warps' partials (warp order)
-      float m_c = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) m_c = fmaxf(m_c, wpart_ml[w * 2]);
+    {  // this CTA's partial from its warps' partials (warp order), pushed into
+       // slot [buf][rank] of every CTA of the cluster
+      // lane w holds warp w's (max, sum); one redux for the max, one warp sum
+      const float mwl = lane < NW ? wpart_ml[lane * 2] : -INFINITY;
+      const float lwl = lane < NW ? wpart_ml[lane * 2 + 1] : 0.f;
+      const float m_c = fkey_inv(__reduce_max_sync(0xffffffffu, fkey(mwl)));
+      const float cwl = (mwl == -INFINITY) ? 0.f : __expf(mwl - m_c);
+      const float l_c = warp_sum(cwl * lwl);
       float cw[NW];
-      float l_c = 0.f;
 #pragma unroll
-      for (int w = 0; w < NW; ++w) {
-        const float mw = wpart_ml[w * 2];
-        cw[w] = (mw == -INFINITY) ? 0.f : expf(mw - m_c);
-        l_c += cw[w] * wpart_ml[w * 2 + 1];
-      }
-      float* po = part_o + buf * h;
+      for (int w = 0; w < NW; ++w) cw[w] = __shfl_sync(0xffffffffu, cwl, w);
+      float* slot = all_o + ((size_t)buf * C + rank) * h;
 #pragma unroll
       for (int d = 0; d < DPT; ++d) {
         const int i = tid + d * NT;
@@ -256,57 +388,48 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
         float acc = 0.f;
 #pragma unroll
         for (int w = 0; w < NW; ++w) acc += cw[w] * wpart_o[w * h + i];
-        po[i] = acc;
+        for (int r = 0; r < C; ++r) cluster.map_shared_rank(slot, r)[i] = acc;
       }
-      if (tid == 0) {
-        part_ml[buf * 2 + 0] = m_c;
-        part_ml[buf * 2 + 1] = l_c;
+      if (tid < C) {
+        float* ml = cluster.map_shared_rank(all_ml + ((size_t)buf * C + rank) * 2, tid);
+        ml[0] = m_c;
+        ml[1] = l_c;
       }
     }
     cluster.sync();
 
-    // ---- 2. merge partials (rank order), residual, LN2
-    if (tid < C) {
-      const float* pm = cluster.map_shared_rank(part_ml, tid);
-      rm[tid] = pm[buf * 2 + 0];
-      rl[tid] = pm[buf * 2 + 1];
-    }
-    __syncthreads();
-    float m = -INFINITY;
-    for (int r = 0; r < C; ++r) m = fmaxf(m, rm[r]);
-    float wsum = 0.f;
+    // ---- 2. merge the C partials (rank order, local reads), residual, LN2
+    //      (one reduction of the moments shifted by z_last[0])
+    // lane r holds CTA r's (max, sum); one redux for the max, one warp sum
+    const float mrl = lane < C ? all_ml[(buf * C + lane) * 2] : -INFINITY;
+    const float lrl = lane < C ? all_ml[(buf * C + lane) * 2 + 1] : 0.f;
+    const float m = fkey_inv(__reduce_max_sync(0xffffffffu, fkey(mrl)));
+    const float wrl = (mrl == -INFINITY) ? 0.f : __expf(mrl - m);
+    const float wsum = warp_sum(wrl * lrl);
     float wr[16];
 #pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      wr[r] = 0.f;
-      if (r < C && rm[r] != -INFINITY) wr[r] = expf(rm[r] - m);
-      if (r < C) wsum += wr[r] * rl[r];
-    }
+    for (int r = 0; r < 16; ++r) wr[r] = __shfl_sync(0xffffffffu, wrl, r);
     const float inv = 1.f / wsum;
-    float s_loc = 0.f;
     float uv[DPT];
+    float mom[2] = {0.f, 0.f};
 #pragma unroll
     for (int d = 0; d < DPT; ++d) {
       const int i = tid + d * NT;
       uv[d] = 0.f;
       if (i >= h) continue;
-      float ro[16];
-#pragma unroll
-      for (int r = 0; r < 16; ++r) ro[r] = (r < C) ? cluster.map_shared_rank(part_o, r)[buf * h + i] : 0.f;
       float o = 0.f;
 #pragma unroll
-      for (int r = 0; r < 16; ++r) o += wr[r] * ro[r];
+      for (int r = 0; r < 16; ++r)
+        if (r < C) o += wr[r] * all_o[((size_t)buf * C + r) * h + i];
       uv[d] = zr[d] + o * inv;
-      s_loc += uv[d];
+      const float c = uv[d] - shift;
+      mom[0] += c;
+      mom[1] += c * c;
     }
-    const float mean = block_sum(s_loc, red) / (float)h;
-    float v_loc = 0.f;
-#pragma unroll
-    for (int d = 0; d < DPT; ++d) {
-      const float c = (tid + d * NT < h) ? uv[d] - mean : 0.f;
-      v_loc += c * c;
-    }
-    const float rstd = rsqrtf(block_sum(v_loc, red) / (float)h + a.ln_eps);
+    block_sum_n<2>(mom, red);
+    const float m1 = mom[0] / (float)h;
+    const float mean = shift + m1;
+    const float rstd = rsqrtf(fmaxf(mom[1] / (float)h - m1 * m1, 0.f) + a.ln_eps);
 #pragma unroll
     for (int d = 0; d < DPT; ++d) {
       const int i = tid + d * NT;
@@ -318,88 +441,143 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     }
     __syncthreads();
 
-    // ---- 3. logits of the available local candidates and the raw STOP logit
+    // ---- 3. logits of the available local candidates (U per warp iteration,
+    //      reductions interleaved), per-warp top g+1, and the raw STOP logit
     float4 xr[HV];
 #pragma unroll
     for (int k = 0; k < HV; ++k) xr[k] = reinterpret_cast<const float4*>(xp_s)[lane + 32 * k];
-    for (int j = warp; j < nl; j += NW) {
-      if (taken[j]) {
-        if (lane == 0) lg[j] = -INFINITY;
-        continue;
+    float tv[GL];
+    int ti[GL];
+#pragma unroll
+    for (int k = 0; k < GL; ++k) { tv[k] = -INFINITY; ti[k] = INT_MAX; }
+    float stop_raw;
+    if (keys_in_smem) {
+      // dims-major keys: warp w takes a slice of the dims, lane = column
+      // (candidates and, at column nl, STOP); per-warp partials are summed per
+      // column in warp order, so every CTA computes STOP identically
+      constexpr int JL = 4;  // columns per lane (nl + 1 <= 128)
+      const float4* kt4 = reinterpret_cast<const float4*>(kt_s);
+      const float4* xp4 = reinterpret_cast<const float4*>(xp_s);
+      const int ncol = nl + 1;
+      const int dper = h4 / NW;
+      const int d0 = warp * dper;
+      float acc[JL];
+#pragma unroll
+      for (int c = 0; c < JL; ++c) acc[c] = 0.f;
+      for (int dd = 0; dd < dper; ++dd) {
+        const float4 xv = xp4[d0 + dd];
+        const float4* col = kt4 + (size_t)(d0 + dd) * LD;
+#pragma unroll
+        for (int c = 0; c < JL; ++c) {
+          const int j = lane + 32 * c;
+          if (j < ncol) acc[c] += dot4(xv, col[j]);
+        }
       }
-      const float4* kr = keys_in_smem ? reinterpret_cast<const float4*>(kt_s + (size_t)j * h)
-                                      : reinterpret_cast<const float4*>(KT + (size_t)(row0 + j0 + j) * a.ldkt);
-      float s = 0.f;
 #pragma unroll
-      for (int k = 0; k < HV; ++k) s += dot4(xr[k], kr[lane + 32 * k]);
-      s = warp_sum(s);
-      if (lane == 0) lg[j] = s;
+      for (int c = 0; c < JL; ++c) {
+        const int j = lane + 32 * c;
+        if (j < ncol) lgp[warp * LD + j] = acc[c];
+      }
+      __syncthreads();
+      float sr = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) sr += lgp[w * LD + nl];
+      stop_raw = sr;
+      float v = -INFINITY;
+      int id = INT_MAX;
+      if (tid < nl && !taken[tid]) {
+        float sj = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) sj += lgp[w * LD + tid];
+        v = sj;
+        id = j0 + tid;
+      }
+      // this warp's top g+1 (one candidate per lane)
+      uint32_t key = (id == INT_MAX) ? 0u : fkey(v);
+#pragma unroll
+      for (int r = 0; r < GL; ++r) {
+        tv[r] = -INFINITY;
+        ti[r] = INT_MAX;
+        if (r < per) {
+          const uint32_t mk = __reduce_max_sync(0xffffffffu, key);
+          const int mi = (int)__reduce_min_sync(0xffffffffu, key == mk ? (uint32_t)id : 0x7fffffffu);
+          tv[r] = fkey_inv(mk);
+          ti[r] = mk ? mi : INT_MAX;
+          if (id == mi) { key = 0u; id = INT_MAX; }
+        }
+      }
+    } else {
+      for (int jb = warp * U; jb < nl; jb += NW * U) {
+        float sv[U];
+        bool ok[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int j = jb + u;
+          ok[u] = j < nl && !taken[j];
+          sv[u] = 0.f;
+          const float4* kr = reinterpret_cast<const float4*>(KT + (size_t)(row0 + j0 + min(j, nl - 1)) * a.ldkt);
+#pragma unroll
+          for (int k = 0; k < HV; ++k) sv[u] += dot4(xr[k], __ldg(kr + lane + 32 * k));
+        }
+        warp_sum_n<U>(sv);
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+          if (ok[u]) top_insert<GL>(tv, ti, sv[u], j0 + jb + u, per);
+      }
+      float s1[1] = {0.f};
+#pragma unroll
+      for (int k = 0; k < HV; ++k) s1[0] += dot4(xr[k], reinterpret_cast<const float4*>(stopkt)[lane + 32 * k]);
+      warp_sum_n<1>(s1);
+      stop_raw = s1[0];  // every warp of every CTA computes the same value
     }
-    float stop_raw = 0.f;
-    {
-      float s = 0.f;
+    if (lane == 0) {
 #pragma unroll
-      for (int k = 0; k < HV; ++k) s += dot4(xr[k], reinterpret_cast<const float4*>(stopkt)[lane + 32 * k]);
-      stop_raw = warp_sum(s);  // every warp of every CTA computes the same value
+      for (int k = 0; k < GL; ++k) {
+        if (k < per) {
+          wtop_v[warp * per + k] = tv[k];
+          wtop_i[warp * per + k] = ti[k];
+        }
+      }
     }
     __syncthreads();
-
-    // local top g+1 by (logit desc, index asc)
-    if (warp == 0) {
-      int picked[GMAX + 1];
-      for (int r = 0; r <= g; ++r) {
-        float bv = -INFINITY;
-        int bi = INT_MAX;
-        for (int j = lane; j < nl; j += 32) {
-          const float v = lg[j];
-          if (v == -INFINITY) continue;
-          bool ex = false;
-          for (int q2 = 0; q2 < r; ++q2) ex |= (picked[q2] == j);
-          if (!ex && better(v, j, bv, bi)) { bv = v; bi = j; }
-        }
-        warp_best(bv, bi);
-        picked[r] = bi;
-        if (lane == 0) {
-          top_v[buf * (GMAX + 1) + r] = bv;
-          top_i[buf * (GMAX + 1) + r] = (bi == INT_MAX) ? INT_MAX : j0 + bi;
+    if (warp == 0) {  // CTA list from the warp lists, pushed into slot [buf][rank] of every CTA
+      float cv[GL];
+      int ci[GL];
+      if (NW * per <= 32)
+        warp_merge_lists<GL, 1>(wtop_v, wtop_i, NW * per, per, cv, ci);
+      else
+        warp_merge_lists<GL, 9>(wtop_v, wtop_i, NW * per, per, cv, ci);
+      if (lane < C) {
+        float* dv = cluster.map_shared_rank(all_tv + (size_t)buf * C * (GMAX + 1) + rank * per, lane);
+        int* di = cluster.map_shared_rank(all_ti + (size_t)buf * C * (GMAX + 1) + rank * per, lane);
+#pragma unroll
+        for (int k = 0; k < GL; ++k) {
+          if (k < per) {
+            dv[k] = cv[k];
+            di[k] = ci[k];
+          }
         }
       }
     }
     cluster.sync();
 
-    // ---- 4. merge the C lists (identically in every CTA) and decide
+    // ---- 4. merge the C lists (local reads, identically in every CTA) and decide
     if (warp == 0) {
-      const int per = g + 1;
-      const int tot = C * per;
-      float ev[9];
-      int ei[9];
+      float gv[GL];
+      int gi[GL];
+      const float* lv = all_tv + (size_t)buf * C * (GMAX + 1);
+      const int* li = all_ti + (size_t)buf * C * (GMAX + 1);
+      if (C * per <= 32)
+        warp_merge_lists<GL, 1>(lv, li, C * per, per, gv, gi);
+      else
+        warp_merge_lists<GL, 9>(lv, li, C * per, per, gv, gi);
+      if (lane == 0) {
 #pragma unroll
-      for (int k = 0; k < 9; ++k) {
-        const int idx = lane + 32 * k;
-        ev[k] = -INFINITY;
-        ei[k] = INT_MAX;
-        if (idx < tot) {
-          const int r = idx / per, s2 = idx % per;
-          const float* rv = cluster.map_shared_rank(top_v, r);
-          const int* ri = cluster.map_shared_rank(top_i, r);
-          ev[k] = rv[buf * (GMAX + 1) + s2];
-          ei[k] = ri[buf * (GMAX + 1) + s2];
-          if (ei[k] == INT_MAX) ev[k] = -INFINITY;
-        }
-      }
-      for (int r = 0; r < per; ++r) {
-        float bv = -INFINITY;
-        int bi = INT_MAX;
-#pragma unroll
-        for (int k = 0; k < 9; ++k)
-          if (better(ev[k], ei[k], bv, bi)) { bv = ev[k]; bi = ei[k]; }
-        warp_best(bv, bi);
-#pragma unroll
-        for (int k = 0; k < 9; ++k)
-          if (ei[k] == bi) { ev[k] = -INFINITY; ei[k] = INT_MAX; }
-        if (lane == 0) {
-          gtop_v[r] = bv;
-          gtop_i[r] = bi;
+        for (int k = 0; k < GL; ++k) {
+          if (k < per) {
+            gtop_v[k] = gv[k];
+            gtop_i[k] = gi[k];
+          }
         }
       }
     }
@@ -413,14 +591,14 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
         // {available visual logits} U {STOP}
         float vals[GMAX + 2];
         int n = 0;
-        const int nv = min(g + 1, n_avail);
+        const int nv = min(per, n_avail);
         for (int k = 0; k < nv; ++k) vals[n++] = gtop_v[k];
         int ins = n;
         while (ins > 0 && vals[ins - 1] < stop_logit) --ins;
         for (int k = n; k > ins; --k) vals[k] = vals[k - 1];
         vals[ins] = stop_logit;
         ++n;
-        const int use = min(n, g + 1);
+        const int use = min(n, per);
         float mg = INFINITY;
         for (int k = 0; k + 1 < use; ++k) mg = fminf(mg, vals[k] - vals[k + 1]);
         a.margin[trace + round] = mg;
@@ -429,18 +607,20 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     ++round;
     if (stop_logit > best) break;  // STOP
     const int take = min(min(g, k_max - nsel), n_avail);
-    if (tid == 0) {
-      for (int k = 0; k < take; ++k) {
-        const int jj = gtop_i[k];
-        if (jj < 0 || jj >= n_e) {
-          set_error(a.err, SP_DEVERR_INDEX);
-          hist[t + k] = a.start_row;
-          continue;
-        }
-        hist[t + k] = row0 + jj;
+    if (tid < take) {
+      const int jj = gtop_i[tid];
+      if (jj < 0 || jj >= n_e) {
+        set_error(a.err, SP_DEVERR_INDEX);
+        hist[t + tid] = a.start_row;
+      } else {
+        hist[t + tid] = row0 + jj;
         if (jj >= j0 && jj < j0 + nl) taken[jj - j0] = 1;
-        if (rank == 0 && a.order) a.order[(size_t)e * k_max + nsel + k] = jj;
+        if (rank == 0 && a.order) a.order[(size_t)e * k_max + nsel + tid] = jj;
       }
+    }
+    {  // rows of the next round's last position
+      const int jl = gtop_i[take - 1];
+      load_last((jl >= 0 && jl < n_e) ? row0 + jl : a.start_row);
     }
     nsel += take;
     __syncthreads();
@@ -449,7 +629,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     if (a.ep_count) a.ep_count[e] = nsel;
     if (a.rounds) a.rounds[e] = round;
   }
-  cluster.sync();  // peers may still read this CTA's slots
+  cluster.sync();  // no CTA leaves while a peer may still write into it
 }
 
 // Algorithm 1 step 4: per image, the union of its episodes' selections in
@@ -516,22 +696,24 @@ restore_kernel(const BatchDesc bd, const int* __restrict__ order, const int* __r
 
 }  // namespace
 
-int select_cluster_size(const BatchDesc& bd, int h, bool* keys_in_smem, size_t* smem_bytes) {
+int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes) {
   int n_max = 0;
   for (int b = 0; b < bd.B; ++b) {
     const int n = bd.vis_off[b + 1] - bd.vis_off[b];
     n_max = std::max(n_max, bd.group_size > 0 ? std::min(bd.group_size, n) : n);
   }
-  (void)smem_bytes;
-  const size_t budget = 200 * 1024;
+  const size_t budget = 225 * 1024;
   for (int C : {8, 16}) {
     const int n_loc = (n_max + C - 1) / C;
-    if ((size_t)n_loc * h * 4 + 16 * 1024 <= budget) {
+    const size_t need = sel_layout(h, n_loc, k_max, C, true).total;
+    if (n_loc + 1 <= 128 && need <= budget) {  // the dims-major logits take <= 128 columns
       *keys_in_smem = true;
+      *smem_bytes = need;
       return C;
     }
   }
   *keys_in_smem = false;
+  *smem_bytes = sel_layout(h, (n_max + 15) / 16, k_max, 16, false).total;
   return 16;
 }
 
@@ -546,13 +728,19 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
   const int n_loc = (n_max + C - 1) / C;
   const SelSmem L = sel_layout(a.h, n_loc, a.k_max, C, keys_in_smem);
   void (*kern)(const BatchDesc, const SelectArgs, int, int) = nullptr;
+  const int gl = a.g + 1 <= 2 ? 2 : (a.g + 1 <= 6 ? 6 : 17);
+#define SP_SEL_CASE(HV_)                                                                                   \
+  case HV_:                                                                                                \
+    kern = gl == 2 ? select_kernel<HV_, 2> : (gl == 6 ? select_kernel<HV_, 6> : select_kernel<HV_, 17>); \
+    break;
   switch (a.h / 128) {
-    case 1: kern = select_kernel<1>; break;
-    case 2: kern = select_kernel<2>; break;
-    case 4: kern = select_kernel<4>; break;
-    case 8: kern = select_kernel<8>; break;
+    SP_SEL_CASE(1)
+    SP_SEL_CASE(2)
+    SP_SEL_CASE(4)
+    SP_SEL_CASE(8)
     default: return cudaErrorInvalidValue;
   }
+#undef SP_SEL_CASE
   cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.total);
   if (r != cudaSuccess) return r;
   if (C > 8) {
