@@ -223,6 +223,19 @@ SP_DEVINL bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Bounded wait with cluster-scope acquire, by the calling thread alone.
+SP_DEVINL bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, int* err) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if ((i & 255u) == 0 && globaltimer_ns() - t0 > kWaitLimitNs) {
+      set_error(err, SP_DEVERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
 // Bounded wait with cluster-scope acquire, warp-uniform (lane 0 polls).
 SP_DEVINL bool mbar_wait_cluster_warp(uint64_t* bar, uint32_t parity, int* err) {
   bool ok = true;

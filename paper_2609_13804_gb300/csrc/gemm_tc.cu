@@ -262,22 +262,22 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t IDESC = umma_idesc_bf16_f32(BM, BN);
-    int s = 0;
-    uint32_t ph = 0;
-    int it = 0;
-    bool ok = true;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
-      const int acc = it & 1;
-      const uint32_t aph = (it >> 1) & 1;
-      if (!mbar_wait_warp(&tempty[acc], aph ^ 1u, err)) { ok = false; break; }
-      tc_fence_after();
-      const uint32_t d_tmem = tmem_base + acc * BN;
-      for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait_warp(&full[s], ph, err)) { ok = false; break; }
+    // ------------------------------------------------------------ MMA issuer (one thread)
+    if (lane == 0) {
+      constexpr uint32_t IDESC = umma_idesc_bf16_f32(BM, BN);
+      int s = 0;
+      uint32_t ph = 0;
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
+        const int acc = it & 1;
+        const uint32_t aph = (it >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], aph ^ 1u, err)) { ok = false; break; }
         tc_fence_after();
-        if (lane == 0) {
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&full[s], ph, err)) { ok = false; break; }
+          tc_fence_after();
           const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
           const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
 #pragma unroll
@@ -286,18 +286,16 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                       (kb | k) != 0 ? 1u : 0u);
           }
           umma_commit(&empty[s]);
+          if (++s == C::STAGES) { s = 0; ph ^= 1u; }
         }
-        __syncwarp();
-        if (++s == C::STAGES) { s = 0; ph ^= 1u; }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
       }
-      if (!ok) break;
-      if (lane == 0) umma_commit(&tfull[acc]);
-      __syncwarp();
+      // All MMAs issued by this thread have completed once `done` flips.
+      umma_commit(done);
+      mbar_wait(done, 0, err);
     }
-    // All MMAs issued by this thread have completed once `done` flips.
-    if (lane == 0) umma_commit(done);
     __syncwarp();
-    mbar_wait_warp(done, 0, err);
   } else {
     // ------------------------------------------------------------ epilogue
     const int quad = warp & 3;  // TMEM lane quadrant this warp may access
@@ -424,8 +422,8 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer (even CTA)
-    if (leader) {
+    // ------------------------------------------------------------ MMA issuer (one thread of the even CTA)
+    if (leader && lane == 0) {
       constexpr uint32_t IDESC = umma_idesc_bf16_f32(2 * BM, BN);
       int s = 0;
       uint32_t ph = 0;
@@ -434,33 +432,29 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
       for (int t = pair; t < total && ok; t += npairs, ++it) {
         const int acc = it & 1;
         const uint32_t aph = (it >> 1) & 1;
-        if (!mbar_wait_cluster_warp(&tempty[acc], aph ^ 1u, err)) { ok = false; break; }
+        if (!mbar_wait_cluster(&tempty[acc], aph ^ 1u, err)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait_cluster_warp(&full[s], ph, err)) { ok = false; break; }
+          if (!mbar_wait_cluster(&full[s], ph, err)) { ok = false; break; }
           tc_fence_after();
-          if (lane == 0) {
-            const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
-            const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+          const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
 #pragma unroll
-            for (int k = 0; k < BK / 16; ++k) {
-              umma_bf16_pair(d_tmem, umma_desc_sw128(a0 + k * 32), umma_desc_sw128(b0 + k * 32), IDESC,
-                             (kb | k) != 0 ? 1u : 0u);
-            }
-            umma_commit_pair(&empty[s], (uint16_t)0x3);
+          for (int k = 0; k < BK / 16; ++k) {
+            umma_bf16_pair(d_tmem, umma_desc_sw128(a0 + k * 32), umma_desc_sw128(b0 + k * 32), IDESC,
+                           (kb | k) != 0 ? 1u : 0u);
           }
-          __syncwarp();
+          umma_commit_pair(&empty[s], (uint16_t)0x3);
           if (++s == C::STAGES) { s = 0; ph ^= 1u; }
         }
         if (!ok) break;
-        if (lane == 0) umma_commit_pair(&tfull[acc], (uint16_t)0x3);
-        __syncwarp();
+        umma_commit_pair(&tfull[acc], (uint16_t)0x3);
       }
-      if (lane == 0) umma_commit_pair(done, (uint16_t)0x1);
-      __syncwarp();
-      mbar_wait_warp(done, 0, err);
+      umma_commit_pair(done, (uint16_t)0x1);
+      mbar_wait(done, 0, err);
     }
+    __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue (both CTAs)
     const int quad = warp & 3;
