@@ -34,6 +34,24 @@ METRIC = "pruned-prefill ms/batch"
 UNIT = "ms/batch"
 
 
+# DRAM read + write bytes per prefill GEMM launch (mean over QKV, O, gate/up and
+# down) from the ncu capture summarised in profiles/gemm_tc2_llava15-7b-dims_1layer.md
+# (one 7B-dims layer at T = 1,792 rows, the benchmark's packed length within
+# 0.5%).  The figure belongs to the kernel sources with this digest; once they
+# change it is reported as null until a new capture replaces it.
+GEMM_TRAFFIC = {"bytes_per_launch": 165.6e6, "sources_sha256_16": "f0e7c28b69ab4171"}
+GEMM_SOURCES = ("paper_2609_13804_gb300/csrc/gemm_tc.cu", "paper_2609_13804_gb300/csrc/common.cuh")
+
+
+def gemm_traffic():
+    import hashlib
+    h = hashlib.sha256()
+    for rel in GEMM_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return GEMM_TRAFFIC["bytes_per_launch"] if h.hexdigest()[:16] == GEMM_TRAFFIC["sources_sha256_16"] else None
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -47,22 +65,33 @@ def peaks():
 # ----------------------------------------------------------------------------- clocks
 
 class Clocks:
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+    """nvidia-smi samples every 50 ms; summary() keeps those taken inside the
+    window marked by start() / stop() (the timed region)."""
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
          "clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index):
         self.index = index
         self.proc = None
+        self.t0 = self.t1 = None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
         return self
+
+    def start(self):
+        import datetime
+        self.t0 = datetime.datetime.now()
+
+    def stop(self):
+        import datetime
+        self.t1 = datetime.datetime.now()
 
     def __exit__(self, *a):
         self.lines = []
@@ -76,11 +105,18 @@ class Clocks:
             self.lines = [l for l in out.splitlines() if l.strip()]
 
     def summary(self):
+        import datetime
         sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for l in getattr(self, "lines", []):
             f = [x.strip() for x in l.split(",")]
             if len(f) < 9:
+                continue
+            try:
+                ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f")
+            except ValueError:
+                ts = None  # unknown format: keep the sample
+            if ts and self.t0 and self.t1 and not (self.t0 <= ts <= self.t1):
                 continue
             try:
                 sm.append(float(f[1]))
@@ -260,12 +296,16 @@ def run_ours(args):
     st = torch.cuda.current_stream()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with Clocks(local) as clk:
+        time.sleep(0.3)  # let the sampler start; the warm GPU idles meanwhile
+        pipe(X, E, bias)
         barrier()
+        clk.start()
         ev0.record(st)
         for _ in range(args.steps):
             pipe(X, E, bias)
         ev1.record(st)
         barrier()
+        clk.stop()
     ms_step = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, dev)
     value = ms_step / world
 
@@ -317,7 +357,18 @@ def run_ours(args):
         comp["o"] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
                                  projector_mode=True)
 
-    compact_ms = timed(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap))
+    def kernel_ms(fn, kind, reps=5):
+        # device time of the launches of one kind (events around each launch on
+        # its stream), free of the binding's host overhead between calls
+        fn()
+        torch.cuda.synchronize()
+        B.sp_profile_begin(reps * 16)
+        for _ in range(reps):
+            fn()
+        torch.cuda.synchronize()
+        return B.sp_profile_end()[kind]["ms"] / reps
+
+    compact_ms = kernel_ms(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap), "compact")
     comp_bytes = 2.0 * (K_sum * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
 
     def prefill_stage(idx, count, kc):
@@ -334,7 +385,7 @@ def run_ours(args):
     full_cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
     full_ms = timed(lambda: prefill_stage(full_idx, full_cnt, 576), reps=3)
     # compaction at a bandwidth-sized case: every visual token kept (the full prefix)
-    full_compact_ms = timed(lambda: do_compact(full_idx, full_cnt, 576))
+    full_compact_ms = kernel_ms(lambda: do_compact(full_idx, full_cnt, 576), "compact")
     full_T = sum(w.n_vis) + sum(w.n_txt)
     full_comp_bytes = 2.0 * (sum(w.n_vis) * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + full_T)
 
@@ -377,7 +428,8 @@ def run_ours(args):
                        "l2": "inputs larger than L2: 13.5 GB of weights streamed every step"},
             "roofline": {"kernel": "gemm_tc (tcgen05)", "bound": "tensor", "achieved": achieved,
                          "peak": pk["bf16_sus"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sus"],
-                         "peak_source": pk["source"] + " bf16 sustained", "traffic": None,
+                         "peak_source": pk["source"] + " bf16 sustained", "traffic": gemm_traffic(),
+                         "traffic_unit": "DRAM bytes per launch",
                          "gemm_ms_per_step": gemm_ms, "gemm_flops_per_step": flops},
             "cpu_baseline": cpu_line,
             "e2e": {"value": e2e_ms / world, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
@@ -404,7 +456,7 @@ def run_ours(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
