@@ -114,6 +114,31 @@ bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t
   return true;
 }
 
+bool encode_tmap_2d(CUtensorMap* map, const void* ptr, bool f32, uint64_t rows, uint64_t cols,
+                    uint32_t box_cols, uint32_t box_rows, std::string* msg) {
+  EncodeTiledFn fn = encode_fn(msg);
+  if (!fn) return false;
+  if (rows == 0) rows = 1;
+  const uint64_t es = f32 ? 4 : 2;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * es};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                  const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (msg) {
+      char b[160];
+      snprintf(b, sizeof(b), "cuTensorMapEncodeTiled failed (%d) for %llux%llu box %ux%u", (int)r,
+               (unsigned long long)rows, (unsigned long long)cols, box_cols, box_rows);
+      *msg = b;
+    }
+    return false;
+  }
+  return true;
+}
+
 // ------------------------------------------------------------------ profiling
 
 namespace {
@@ -358,7 +383,9 @@ size_t select_ws(const sp_selector* s, const SelPlan& p, const sp_select_out* ou
   float *P = nullptr, *R = nullptr, *Mall, *ZK, *XL, *QKVs;
   void *Abf = nullptr, *QKV = nullptr, *O = nullptr, *F1 = nullptr;
   int* enc_cu = nullptr;
+  void* gsk = nullptr;
   if (p.encoder && s->cfg.n_enc_layers > 0) {
+    gsk = cv.take<char>(gemm_scratch_bytes());
     P = cv.take<float>((size_t)std::max(p.ntxt, 1) * D);
     R = cv.take<float>((size_t)p.T_enc * D);
     Abf = cv.take<uint16_t>((size_t)p.T_enc * D);
@@ -378,7 +405,7 @@ size_t select_ws(const sp_selector* s, const SelPlan& p, const sp_select_out* ou
   if (parts) {
     parts[0] = P; parts[1] = R; parts[2] = Abf; parts[3] = QKV; parts[4] = O; parts[5] = F1;
     parts[6] = enc_cu; parts[7] = Mall; parts[8] = ZK; parts[9] = XL; parts[10] = QKVs;
-    parts[11] = order; parts[12] = epc;
+    parts[11] = order; parts[12] = epc; parts[13] = gsk;
   }
   return cv.off;
 }
@@ -395,6 +422,8 @@ sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPla
   void* O = parts[4];
   void* F1 = parts[5];
   int* enc_cu = (int*)parts[6];
+  const GemmScratch gs = gemm_scratch_at(parts[13]);
+  SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   std::string msg;
   if (p.ntxt > 0) {
     CUtensorMap tE;
@@ -403,7 +432,7 @@ sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPla
     ep.kind = EPI_F32;
     ep.out = P;
     ep.ldo = D;
-    SP_CUDA(gemm_bf16(tE, p.ntxt, nullptr, s->Wp, D, ep, err, st), "text projection");
+    SP_CUDA(gemm_bf16(tE, p.ntxt, nullptr, s->Wp, D, ep, err, st, &gs), "text projection");
   }
   SP_CUDA(assemble_encoder_input(p.bd, in->X, P, D, s->w.ln_text_g, s->w.ln_text_b, c.ln_eps, c.g_text, R,
                                  p.T_enc, st), "encoder input");
@@ -419,20 +448,20 @@ sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPla
     e1.kind = EPI_BF16;
     e1.out = QKV;
     e1.ldo = 3 * D;
-    SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_qkv[l], 3 * D, e1, err, st), "enc qkv");
+    SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_qkv[l], 3 * D, e1, err, st, &gs), "enc qkv");
     SP_CUDA(attention_varlen(QKV, O, enc_cu, in->B, p.max_enc, nh, nh, c.enc_head_dim, false, st), "enc attention");
     GemmEpi e2;
     e2.kind = EPI_F32_ACC;
     e2.out = R;
     e2.ldo = D;
-    SP_CUDA(gemm_bf16(tO, p.T_enc, nullptr, s->enc_o[l], D, e2, err, st), "enc o");
+    SP_CUDA(gemm_bf16(tO, p.T_enc, nullptr, s->enc_o[l], D, e2, err, st, &gs), "enc o");
     SP_CUDA(layernorm_f32(R, D, s->w.enc_ln2_g[l], s->w.enc_ln2_b[l], nullptr, Abf, D, p.T_enc, D, c.ln_eps, 1.f, st), "enc ln2");
     GemmEpi e3;
     e3.kind = EPI_GELU_BF16;
     e3.out = F1;
     e3.ldo = c.enc_ffn;
-    SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_1[l], c.enc_ffn, e3, err, st), "enc fc1");
-    SP_CUDA(gemm_bf16(tF, p.T_enc, nullptr, s->enc_2[l], D, e2, err, st), "enc fc2");
+    SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_1[l], c.enc_ffn, e3, err, st, &gs), "enc fc1");
+    SP_CUDA(gemm_bf16(tF, p.T_enc, nullptr, s->enc_2[l], D, e2, err, st, &gs), "enc fc2");
   }
   return SP_OK;
 }
@@ -466,7 +495,7 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   }
   if (out->k_cap < need_cap) return fail(SP_ERR_SHAPE, "sp_select: k_cap %d < largest possible count %d", out->k_cap, need_cap);
   Carve cv(ws);
-  void* parts[13];
+  void* parts[14];
   const size_t need = select_ws(s, p, out, cv, parts) + 256;
   if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_select: workspace %zu < %zu bytes", ws_bytes, need);
   if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_select: workspace must be 16-byte aligned");
@@ -659,10 +688,12 @@ void sp_model_destroy(sp_model* m) {
 
 // ------------------------------------------------------------------ projector
 
-static size_t project_ws(const sp_model* m, int rows_cap, Carve& cv, void** tmp) {
+static size_t project_ws(const sp_model* m, int rows_cap, Carve& cv, void** tmp, void** gsk = nullptr) {
   void* t = nullptr;
   if (m->cfg.proj_kind == SP_PROJ_MLP2_GELU) t = cv.take<uint16_t>((size_t)std::max(rows_cap, 1) * m->cfg.proj_hidden);
+  void* g = m->cfg.proj_kind != SP_PROJ_NONE ? cv.take<char>(gemm_scratch_bytes()) : nullptr;
   if (tmp) *tmp = t;
+  if (gsk) *gsk = g;
   return cv.off;
 }
 
@@ -683,9 +714,14 @@ static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* 
   if (io->rows_cap == 0) return SP_OK;
   Carve cv(ws);
   void* tmp = nullptr;
-  const size_t need = project_ws(m, io->rows_cap, cv, &tmp) + 256;
-  if (c.proj_kind == SP_PROJ_MLP2_GELU && (!ws || ws_bytes < need))
+  void* gsk = nullptr;
+  const size_t need = project_ws(m, io->rows_cap, cv, &tmp, &gsk) + 256;
+  const bool have_ws = ws && ws_bytes >= need;
+  if (c.proj_kind == SP_PROJ_MLP2_GELU && !have_ws)
     return fail(SP_ERR_WORKSPACE, "sp_project: workspace %zu < %zu bytes", ws_bytes, need);
+  // a linear projector runs without a workspace too (whole GEMM tiles only)
+  const GemmScratch gs = gemm_scratch_at(have_ws ? gsk : nullptr);
+  SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   std::string msg;
   CUtensorMap tV;
   if (!encode_tmap_bf16(&tV, io->vis_packed, io->rows_cap, c.proj_in, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
@@ -696,17 +732,17 @@ static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* 
   sc.ldo = c.d;
   sc.row_map = io->vis_row_map;
   if (c.proj_kind == SP_PROJ_LINEAR) {
-    SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.d, sc, io->err, st), "projector");
+    SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.d, sc, io->err, st, &gs), "projector");
     return SP_OK;
   }
   GemmEpi g1;
   g1.kind = EPI_GELU_BF16;
   g1.out = tmp;
   g1.ldo = c.proj_hidden;
-  SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.proj_hidden, g1, io->err, st), "projector fc1");
+  SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.proj_hidden, g1, io->err, st, &gs), "projector fc1");
   CUtensorMap tT;
   if (!encode_tmap_bf16(&tT, tmp, io->rows_cap, c.proj_hidden, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
-  SP_CUDA(gemm_bf16(tT, io->rows_cap, M_dev, m->p2, c.d, sc, io->err, st), "projector fc2");
+  SP_CUDA(gemm_bf16(tT, io->rows_cap, M_dev, m->p2, c.d, sc, io->err, st, &gs), "projector fc2");
   return SP_OK;
 }
 
@@ -718,7 +754,7 @@ sp_status sp_project(const sp_model* m, const sp_project_io* io, void* ws, size_
 
 struct PrefillParts {
   float* h32;
-  void *xb, *qkv, *ob, *act;
+  void *xb, *qkv, *ob, *act, *gsk;
 };
 
 static size_t prefill_ws(const sp_model* m, int T_cap, bool own_residual, Carve& cv, PrefillParts* p) {
@@ -730,6 +766,7 @@ static size_t prefill_ws(const sp_model* m, int T_cap, bool own_residual, Carve&
   q.qkv = cv.take<uint16_t>(T * (c.n_heads + 2 * c.n_kv_heads) * c.head_dim);
   q.ob = cv.take<uint16_t>(T * c.n_heads * c.head_dim);
   q.act = cv.take<uint16_t>(T * c.ffn);
+  q.gsk = cv.take<char>(gemm_scratch_bytes());
   if (p) *p = q;
   return cv.off;
 }
@@ -764,6 +801,8 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
   if (!encode_tmap_bf16(&tX, p.xb, T_cap, c.d, 128, &msg) || !encode_tmap_bf16(&tO, p.ob, T_cap, dq, 128, &msg) ||
       !encode_tmap_bf16(&tA, p.act, T_cap, c.ffn, 128, &msg))
     return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  const GemmScratch gs = gemm_scratch_at(p.gsk);
+  SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   SP_CUDA(bf16_to_f32(io->x, h32, T_cap, T_dev, c.d, st), "embed");
   for (int l = 0; l < c.n_layers; ++l) {
     SP_CUDA(rmsnorm_f32_to_bf16(h32, m->w.attn_norm[l], p.xb, T_cap, T_dev, c.d, c.rms_eps, st), "attn norm");
@@ -776,22 +815,22 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
     eq.max_pos = c.max_pos;
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
-    SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->qkv[l], qkvw, eq, io->err, st), "qkv");
+    SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->qkv[l], qkvw, eq, io->err, st, &gs), "qkv");
     SP_CUDA(attention_varlen(p.qkv, p.ob, io->cu_seqlens, io->B, io->max_seqlen_cap, c.n_heads, c.n_kv_heads,
                              c.head_dim, true, st), "attention");
     GemmEpi er;
     er.kind = EPI_F32_ACC;
     er.out = h32;
     er.ldo = c.d;
-    SP_CUDA(gemm_bf16(tO, T_cap, T_dev, m->o[l], c.d, er, io->err, st), "o");
+    SP_CUDA(gemm_bf16(tO, T_cap, T_dev, m->o[l], c.d, er, io->err, st, &gs), "o");
     SP_CUDA(rmsnorm_f32_to_bf16(h32, m->w.mlp_norm[l], p.xb, T_cap, T_dev, c.d, c.rms_eps, st), "mlp norm");
     GemmEpi eg;
     eg.kind = EPI_SWIGLU_BF16;
     eg.out = p.act;
     eg.ldo = c.ffn;
     eg.up_off = c.ffn;
-    SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->gu[l], 2 * c.ffn, eg, io->err, st), "gate/up");
-    SP_CUDA(gemm_bf16(tA, T_cap, T_dev, m->down[l], c.d, er, io->err, st), "down");
+    SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->gu[l], 2 * c.ffn, eg, io->err, st, &gs), "gate/up");
+    SP_CUDA(gemm_bf16(tA, T_cap, T_dev, m->down[l], c.d, er, io->err, st, &gs), "down");
   }
   SP_CUDA(rmsnorm_f32_to_f32(h32, m->w.final_norm, io->hidden, T_cap, T_dev, c.d, c.rms_eps, st), "final norm");
   return SP_OK;

@@ -33,13 +33,19 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;
 
+// Epilogue staging: per epilogue warp two boxes of 32 rows x 128 bytes
+// (128-byte swizzle) that TMA stores (or reduce-adds) to global memory while
+// the warp fills the other one.
+constexpr uint32_t BOX_BYTES = 32 * 128;
+constexpr uint32_t EPI_STAGE_BYTES = 4 * 2 * BOX_BYTES;
+
 template <int BN>
 struct Cfg {
   static constexpr int STAGES = (BN == 256) ? 4 : 6;
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
-  static constexpr size_t SMEM = 1024 + STAGES * (A_BYTES + B_BYTES) + 256;
+  static constexpr size_t SMEM = 1024 + STAGES * (A_BYTES + B_BYTES) + EPI_STAGE_BYTES + 256;
 };
 
 struct KArgs {
@@ -49,7 +55,63 @@ struct KArgs {
   int K;
   GemmEpi e;
   int* err;
+  float* sk_part;  // pair kernel: stream-K partial tiles [pairs][256][BN] (NULL: whole tiles only)
+  int* sk_flags;   // pair kernel: [pairs][8] ready flags, zero between launches
 };
+
+// Partial sums other pairs computed for this tile (stream-K tail): `n` slots,
+// `stride` floats apart, from the slot of the first.  A slot holds a 256-row
+// tile as float4 [BN/32 column chunks][8][256 rows], so that a warp's 32 rows
+// of one float4 column are 512 contiguous bytes.
+struct Fix {
+  const float* p = nullptr;
+  int n = 0;
+  size_t stride = 0;
+  int rit = 0;  // this lane's row within the 256-row tile
+};
+
+SP_DEVINL void fix_add(const Fix& f, int col, float (&v)[32]) {
+#pragma unroll 1
+  for (int q = 0; q < f.n; ++q) {
+    const float4* s = reinterpret_cast<const float4*>(f.p + q * f.stride) + (size_t)(col >> 5) * 8 * 256 + f.rit;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float4 x = __ldcg(s + j * 256);
+      v[4 * j] += x.x;
+      v[4 * j + 1] += x.y;
+      v[4 * j + 2] += x.z;
+      v[4 * j + 3] += x.w;
+    }
+  }
+}
+
+// Completes a tcgen05.ld of 32 columns into v and adds the partials of those
+// columns; the first partial's loads are issued before the TMEM wait so the
+// two latencies overlap.
+SP_DEVINL void fix_add_waited(const Fix& f, int col, float (&v)[32]) {
+  if (f.n == 0) {
+    tmem_ld_wait();
+    return;
+  }
+  float4 x[8];
+  const float4* s = reinterpret_cast<const float4*>(f.p) + (size_t)(col >> 5) * 8 * 256 + f.rit;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) x[j] = __ldcg(s + j * 256);
+  tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    v[4 * j] += x[j].x;
+    v[4 * j + 1] += x[j].y;
+    v[4 * j + 2] += x[j].z;
+    v[4 * j + 3] += x[j].w;
+  }
+  if (f.n > 1) {
+    Fix rest = f;
+    rest.p = f.p + f.stride;
+    rest.n = f.n - 1;
+    fix_add(rest, col, v);
+  }
+}
 
 SP_DEVINL void store_bf16x32(__nv_bfloat16* dst, const float (&v)[32]) {
   uint4* d = reinterpret_cast<uint4*>(dst);
@@ -67,7 +129,8 @@ SP_DEVINL void store_bf16x32(__nv_bfloat16* dst, const float (&v)[32]) {
 // Drains one 128 x BN accumulator tile from TMEM (this warp: 32 rows, lane =
 // row `row`), applies the epilogue and stores the row if it is live.
 template <int BN, int EPI>
-SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool live, int nb, int* err) {
+SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool live, int nb, int* err,
+                             const Fix& fx) {
   float v[32];
 
   if (EPI == EPI_SWIGLU_BF16) {
@@ -78,6 +141,8 @@ SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool liv
       tmem_ld_32x32b_x32(taddr + BN / 2 + c * 32, u);
       tmem_ld_wait();
       if (live) {
+        fix_add(fx, c * 32, v);
+        fix_add(fx, BN / 2 + c * 32, u);
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = silu(v[i]) * u[i];
         __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(e.out) + (size_t)row * e.ldo +
@@ -102,6 +167,8 @@ SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool liv
           tmem_ld_32x32b_x32(taddr + hb + half + c, u);
           tmem_ld_wait();
           if (live) {
+            fix_add(fx, hb + c, v);
+            fix_add(fx, hb + half + c, u);
             const float2* cs = e.rope + (size_t)(pos_ok ? p : 0) * half + c;
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
@@ -122,6 +189,7 @@ SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool liv
           tmem_ld_32x32b_x32(taddr + hb + c, v);
           tmem_ld_wait();
           if (live) {
+            fix_add(fx, hb + c, v);
             __nv_bfloat16* o =
                 reinterpret_cast<__nv_bfloat16*>(e.out) + (size_t)row * e.ldo + col0 + c;
             store_bf16x32(o, v);
@@ -143,6 +211,7 @@ SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool liv
       tmem_ld_32x32b_x32(taddr + c * 32, v);
       tmem_ld_wait();
       if (!store) continue;
+      fix_add(fx, c * 32, v);
       const int col = nb * BN + c * 32;
       if (EPI == EPI_F32 || EPI == EPI_F32_ACC) {
         float4* o = reinterpret_cast<float4*>(reinterpret_cast<float*>(e.out) +
@@ -169,9 +238,192 @@ SP_DEVINL void epilogue_tile(const GemmEpi& e, uint32_t taddr, int row, bool liv
   }
 }
 
+// One 16-byte chunk of this lane's row of a staging box (128-byte swizzle:
+// chunk q of row r sits at chunk q ^ (r % 8), so the 8 rows a shared-memory
+// wavefront serves hit 8 different bank groups).
+SP_DEVINL void box_put(uint8_t* box, int lane, int q, uint4 w) {
+  *reinterpret_cast<uint4*>(box + lane * 128 + ((q ^ (lane & 7)) << 4)) = w;
+}
+
+// 32 fp32 values as bf16 into half h (64 bytes) of this lane's box row.
+SP_DEVINL void box_put_bf16_half(uint8_t* box, int lane, int h, const float (&v)[32]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint4 u;
+    u.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
+    u.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
+    u.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
+    u.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
+    box_put(box, lane, 4 * h + q, u);
+  }
+}
+
+SP_DEVINL void zero32(float (&v)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = 0.f;
+}
+
+// Hands the filled box(es) of this warp to TMA: every lane's shared-memory
+// writes are made visible to the async proxy, then lane 0 issues the copies
+// as one bulk group.
+SP_DEVINL void box_fence(int lane) {
+  fence_proxy_async_smem();
+  __syncwarp();
+}
+
+// Drains this warp's 32 rows (row0 + lane) of a BN-wide accumulator tile
+// from TMEM, applies the epilogue and writes it with TMA through the staging
+// boxes `boxes` (two per warp; `nbox` counts the boxes issued so far).  Rows
+// past M are written as zeros (EPI_F32_ACC: adds zero); rows past the output
+// map's extent are clipped by TMA.
+template <int BN, int EPI>
+SP_DEVINL void epilogue_tma(const GemmEpi& e, const CUtensorMap* tmO, uint32_t taddr, int row0, int lane,
+                            bool live, int nb, uint8_t* boxes, int& nbox, const Fix& fx, int* err) {
+  float v[32];
+  if (EPI == EPI_F32 || EPI == EPI_F32_ACC) {
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      tmem_ld_32x32b_x32(taddr + c * 32, v);
+      fix_add_waited(fx, c * 32, v);
+      if (!live) zero32(v);
+      if (lane == 0) bulk_wait_read<1>();
+      __syncwarp();
+      uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        box_put(box, lane, q, make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]),
+                                         __float_as_uint(v[4 * q + 2]), __float_as_uint(v[4 * q + 3])));
+      box_fence(lane);
+      if (lane == 0) {
+        if (EPI == EPI_F32_ACC)
+          tma_reduce_add_2d(tmO, box, nb * BN + c * 32, row0);
+        else
+          tma_store_2d(tmO, box, nb * BN + c * 32, row0);
+        bulk_commit();
+      }
+      ++nbox;
+    }
+  } else if (EPI == EPI_BF16 || EPI == EPI_GELU_BF16) {
+#pragma unroll 1
+    for (int c2 = 0; c2 < BN / 64; ++c2) {
+      if (lane == 0) bulk_wait_read<1>();
+      __syncwarp();
+      uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        tmem_ld_32x32b_x32(taddr + c2 * 64 + h * 32, v);
+        fix_add_waited(fx, c2 * 64 + h * 32, v);
+        if (EPI == EPI_GELU_BF16) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
+        }
+        if (!live) zero32(v);
+        box_put_bf16_half(box, lane, h, v);
+      }
+      box_fence(lane);
+      if (lane == 0) {
+        tma_store_2d(tmO, box, nb * BN + c2 * 64, row0);
+        bulk_commit();
+      }
+      ++nbox;
+    }
+  } else if (EPI == EPI_SWIGLU_BF16) {
+    // accumulator columns [0, BN/2) gate, [BN/2, BN) up -> BN/2 output columns
+    float u[32];
+#pragma unroll 1
+    for (int c2 = 0; c2 < BN / 128; ++c2) {
+      if (lane == 0) bulk_wait_read<1>();
+      __syncwarp();
+      uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        const int c = c2 * 64 + h * 32;
+        tmem_ld_32x32b_x32(taddr + c, v);
+        tmem_ld_32x32b_x32(taddr + BN / 2 + c, u);
+        fix_add_waited(fx, c, v);
+        fix_add(fx, BN / 2 + c, u);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = silu(v[i]) * u[i];
+        if (!live) zero32(v);
+        box_put_bf16_half(box, lane, h, v);
+      }
+      box_fence(lane);
+      if (lane == 0) {
+        tma_store_2d(tmO, box, nb * (BN / 2) + c2 * 64, row0);
+        bulk_commit();
+      }
+      ++nbox;
+    }
+  } else if (EPI == EPI_BF16_ROPE) {
+    // per head of dh = 64 or 128 columns: dh / 64 boxes; rotate-half pairs
+    // column c of the first half with column c + dh/2
+    const int dh = e.head_dim;
+    const int half = dh >> 1;
+    const int row = row0 + lane;
+    const int p = live ? __ldg(e.pos + row) : 0;
+    const bool pos_ok = p >= 0 && p < e.max_pos;
+    if (live && !pos_ok) set_error(err, SP_DEVERR_INDEX);
+    const int nbx = dh >> 6;
+    float u[32];
+#pragma unroll 1
+    for (int hb = 0; hb < BN; hb += dh) {
+      const int col0 = nb * BN + hb;
+      if (lane == 0) {
+        if (nbx == 2) bulk_wait_read<0>(); else bulk_wait_read<1>();
+      }
+      __syncwarp();
+      uint8_t* bx0 = boxes + (nbox & 1) * BOX_BYTES;
+      uint8_t* bx1 = boxes + ((nbox + 1) & 1) * BOX_BYTES;
+      if (col0 < e.rope_cols) {
+#pragma unroll 1
+        for (int c = 0; c < half; c += 32) {
+          tmem_ld_32x32b_x32(taddr + hb + c, v);
+          tmem_ld_32x32b_x32(taddr + hb + half + c, u);
+          fix_add_waited(fx, hb + c, v);
+          fix_add(fx, hb + half + c, u);
+          if (live) {
+            const float4* cs = reinterpret_cast<const float4*>(e.rope + (size_t)(pos_ok ? p : 0) * half + c);
+#pragma unroll
+            for (int i2 = 0; i2 < 16; ++i2) {
+              const float4 r = __ldg(cs + i2);
+              const float a0 = v[2 * i2], b0 = u[2 * i2], a1 = v[2 * i2 + 1], b1 = u[2 * i2 + 1];
+              v[2 * i2] = a0 * r.x - b0 * r.y;
+              u[2 * i2] = b0 * r.x + a0 * r.y;
+              v[2 * i2 + 1] = a1 * r.z - b1 * r.w;
+              u[2 * i2 + 1] = b1 * r.z + a1 * r.w;
+            }
+          } else {
+            zero32(v);
+            zero32(u);
+          }
+          const int ov = c, ou = c + half;  // output offsets within the head
+          box_put_bf16_half((ov >> 6) ? bx1 : bx0, lane, (ov >> 5) & 1, v);
+          box_put_bf16_half((ou >> 6) ? bx1 : bx0, lane, (ou >> 5) & 1, u);
+        }
+      } else {
+#pragma unroll 1
+        for (int o = 0; o < dh; o += 32) {
+          tmem_ld_32x32b_x32(taddr + hb + o, v);
+          fix_add_waited(fx, hb + o, v);
+          if (!live) zero32(v);
+          box_put_bf16_half((o >> 6) ? bx1 : bx0, lane, (o >> 5) & 1, v);
+        }
+      }
+      box_fence(lane);
+      if (lane == 0) {
+        tma_store_2d(tmO, bx0, col0, row0);
+        if (nbx == 2) tma_store_2d(tmO, bx1, col0 + 64, row0);
+        bulk_commit();
+      }
+      nbox += nbx;
+    }
+  }
+}
+
 template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmO,
                const KArgs args) {
   using C = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
@@ -179,7 +431,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                                              ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  uint8_t* sE = sB + C::STAGES * C::B_BYTES;  // epilogue staging boxes (1024-byte aligned)
+  uint64_t* full = reinterpret_cast<uint64_t*>(sE + EPI_STAGE_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;
   uint64_t* tempty = tfull + 2;
@@ -299,6 +552,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   } else {
     // ------------------------------------------------------------ epilogue
     const int quad = warp & 3;  // TMEM lane quadrant this warp may access
+    uint8_t* boxes = sE + quad * 2 * BOX_BYTES;
+    int nbox = 0;
     int it = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
       const int acc = it & 1;
@@ -306,13 +561,18 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (!mbar_wait_warp(&tfull[acc], aph, err)) break;
       tc_fence_after();
       const int mb = t % num_m, nb = t / num_m;
-      const int row = mb * BM + quad * 32 + lane;
+      const int row0 = mb * BM + quad * 32;
+      const int row = row0 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + acc * BN;
-      epilogue_tile<BN, EPI>(args.e, taddr, row, row < M, nb, err);
+      if (EPI == EPI_SCATTER_BF16)
+        epilogue_tile<BN, EPI>(args.e, taddr, row, row < M, nb, err, Fix());
+      else
+        epilogue_tma<BN, EPI>(args.e, &tmO, taddr, row0, lane, row < M, nb, boxes, nbox, Fix(), err);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
     }
+    if (lane == 0) bulk_wait<0>();  // the staging boxes stay valid until every copy is done
   }
 
   tc_fence_before();
@@ -320,6 +580,116 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+
+// Work split of the pair kernel over its W pairs.  Whole tiles go round-robin
+// while every pair gets one (data-parallel waves); when the last, partial
+// wave would leave at least half of the pairs idle, its r tiles are instead
+// cut along K into s = min(W / r, kSkMaxSplit) equal ranges spread over r*s
+// pairs (a stream-K tail, after Osama et al., PPoPP 2023).  The pair with a
+// tile's first K range finishes the tile after adding the fp32 partials the
+// other s - 1 pairs wrote to their slots.  The general form below also
+// allows ranges that straddle tiles (at most two fragments per pair: the end
+// of one tile, written as a partial, and the start of the next).
+constexpr int kSkMinIters = 8;   // K blocks per tail range at least (fix-up traffic vs balance)
+constexpr int kSkMaxSplit = 2;   // one partial per tile: the finishing epilogue waits on one pair
+
+struct Sched {
+  int num_m, KB, W, p;
+  int full;        // tiles of the data-parallel waves
+  int Wt;          // pairs sharing the tail (0: no tail)
+  long long I;     // K-block iterations of the tail
+  SP_DEVINL long long bnd(int q) const { return (long long)q * I / Wt; }
+};
+
+struct Frag {
+  int t, k0, k1;
+  int kind;        // 0 whole tile, 1 first K range (finishes the tile), 2 later K range (partial)
+};
+
+SP_DEVINL Sched make_sched(int total, int num_m, int KB, int W, int p, bool stream_k) {
+  Sched s;
+  s.num_m = num_m;
+  s.KB = KB;
+  s.W = W;
+  s.p = p;
+  s.full = total;
+  s.Wt = 0;
+  s.I = 0;
+  const int r = total % W;
+  if (stream_k && r != 0) {
+    const long long I = (long long)r * KB;
+    const int split = min(min(W / r, kSkMaxSplit), KB / kSkMinIters);
+    const int Wt = r * split;
+    if (split > 1) {
+      s.full = total - r;
+      s.Wt = Wt;
+      s.I = I;
+    }
+  }
+  return s;
+}
+
+struct Cursor {
+  int j = 0;
+  long long g = -1;
+};
+
+SP_DEVINL bool sched_next(const Sched& s, Cursor& c, Frag& f) {
+  const int t = s.p + c.j * s.W;
+  if (t < s.full) {
+    f.t = t;
+    f.k0 = 0;
+    f.k1 = s.KB;
+    f.kind = 0;
+    ++c.j;
+    return true;
+  }
+  if (s.p >= s.Wt) return false;
+  if (c.g < 0) c.g = s.bnd(s.p);
+  const long long e = s.bnd(s.p + 1);
+  if (c.g >= e) return false;
+  const int tl = (int)(c.g / s.KB);
+  const int k0 = (int)(c.g - (long long)tl * s.KB);
+  const int k1 = (int)min((long long)s.KB, (long long)k0 + (e - c.g));
+  f.t = s.full + tl;
+  f.k0 = k0;
+  f.k1 = k1;
+  f.kind = k0 > 0 ? 2 : (k1 < s.KB ? 1 : 0);
+  c.g += k1 - k0;
+  return true;
+}
+
+// Pairs after `p` whose first tail fragment belongs to tail tile `t`.
+SP_DEVINL int sched_contributors(const Sched& s, int t) {
+  const long long g1 = (long long)(t - s.full + 1) * s.KB;
+  int n = 0;
+  for (int q = s.p + 1; q < s.Wt && s.bnd(q) < g1; ++q) ++n;
+  return n;
+}
+
+SP_DEVINL int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+SP_DEVINL void st_release_gpu(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// The calling thread waits until *flag == 1 (bounded).
+SP_DEVINL bool wait_flag(const int* flag, int* err) {
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 0;; ++i) {
+    if (ld_acquire_gpu(flag) == 1) return true;
+    if ((i & 63u) == 0 && globaltimer_ns() - t0 > kWaitLimitNs) {
+      set_error(err, SP_DEVERR_TIMEOUT);
+      return false;
+    }
+    __nanosleep(32);
   }
 }
 
@@ -338,12 +708,13 @@ struct Cfg2 {
   static constexpr uint32_t B_BYTES = (BN / 2) * BK * 2;
   static constexpr int STAGES = (BN == 256) ? 6 : 8;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
-  static constexpr size_t SMEM = 1024 + STAGES * (A_BYTES + B_BYTES) + 256;
+  static constexpr size_t SMEM = 1024 + STAGES * (A_BYTES + B_BYTES) + EPI_STAGE_BYTES + 256;
 };
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
 gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmO,
                 const KArgs args) {
   using C = Cfg2<BN>;
   extern __shared__ uint8_t smem_raw[];
@@ -351,7 +722,8 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
                                              ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  uint8_t* sE = sB + C::STAGES * C::B_BYTES;  // epilogue staging boxes (1024-byte aligned)
+  uint64_t* full = reinterpret_cast<uint64_t*>(sE + EPI_STAGE_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;
   uint64_t* tempty = tfull + 2;
@@ -372,6 +744,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   const int total = num_m * num_n;
   const int KB = args.K / BK;
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const Sched sc = make_sched(total, num_m, KB, npairs, pair, args.sk_part != nullptr && args.sk_flags != nullptr);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -401,8 +774,10 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
       tma_prefetch_desc(&tmB);
       int s = 0;
       uint32_t ph = 0;
-      for (int t = pair; t < total; t += npairs) {
-        const int mb = t % num_m, nb = t / num_m;
+      Cursor cur;
+      Frag f;
+      while (sched_next(sc, cur, f)) {
+        const int mb = f.t % num_m, nb = f.t / num_m;
         const int a_row = mb * 2 * BM + (int)rank * BM;
         int b_row;
         if (EPI == EPI_SWIGLU_BF16)
@@ -410,7 +785,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
         else
           b_row = nb * BN + (int)rank * (BN / 2);
         bool ok = true;
-        for (int kb = 0; kb < KB; ++kb) {
+        for (int kb = f.k0; kb < f.k1; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, err)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[s], 2 * (C::A_BYTES + C::B_BYTES));
           const uint32_t bar = mapa_shared(smem_u32(&full[s]), 0);
@@ -429,13 +804,15 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
       uint32_t ph = 0;
       int it = 0;
       bool ok = true;
-      for (int t = pair; t < total && ok; t += npairs, ++it) {
+      Cursor cur;
+      Frag f;
+      for (; ok && sched_next(sc, cur, f); ++it) {
         const int acc = it & 1;
         const uint32_t aph = (it >> 1) & 1;
         if (!mbar_wait_cluster(&tempty[acc], aph ^ 1u, err)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        for (int kb = 0; kb < KB; ++kb) {
+        for (int kb = f.k0; kb < f.k1; ++kb) {
           if (!mbar_wait_cluster(&full[s], ph, err)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
@@ -443,7 +820,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             umma_bf16_pair(d_tmem, umma_desc_sw128(a0 + k * 32), umma_desc_sw128(b0 + k * 32), IDESC,
-                           (kb | k) != 0 ? 1u : 0u);
+                           (kb != f.k0 || k != 0) ? 1u : 0u);
           }
           umma_commit_pair(&empty[s], (uint16_t)0x3);
           if (++s == C::STAGES) { s = 0; ph ^= 1u; }
@@ -458,20 +835,67 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   } else {
     // ------------------------------------------------------------ epilogue (both CTAs)
     const int quad = warp & 3;
+    const int rit = (int)rank * BM + quad * 32 + lane;  // row within the 256-row pair tile
+    const int fslot = (int)rank * 4 + quad;              // this warp's ready flag within a pair's 8
+    const size_t slot_floats = (size_t)2 * BM * BN;
+    uint8_t* boxes = sE + quad * 2 * BOX_BYTES;
+    int nbox = 0;
     int it = 0;
-    for (int t = pair; t < total; t += npairs, ++it) {
+    Cursor cur;
+    Frag f;
+    for (; sched_next(sc, cur, f); ++it) {
       const int acc = it & 1;
       const uint32_t aph = (it >> 1) & 1;
       if (!mbar_wait_cluster_warp(&tfull[acc], aph, err)) break;
       tc_fence_after();
-      const int mb = t % num_m, nb = t / num_m;
-      const int row = mb * 2 * BM + (int)rank * BM + quad * 32 + lane;
+      const int mb = f.t % num_m, nb = f.t / num_m;
+      const int row0 = mb * 2 * BM + (int)rank * BM + quad * 32;
+      const int row = row0 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + acc * BN;
-      epilogue_tile<BN, EPI>(args.e, taddr, row, row < M, nb, err);
+      if (f.kind == 2) {
+        // a later K range: hand the raw fp32 partial to the pair finishing the tile
+        float v[32];
+        float4* dst = reinterpret_cast<float4*>(args.sk_part + pair * slot_floats) + rit;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld_32x32b_x32(taddr + c * 32, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            __stcg(dst + (size_t)(c * 8 + q) * 256, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+        }
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) st_release_gpu(args.sk_flags + pair * 8 + fslot, 1);
+      } else {
+        Fix fx;
+        if (f.kind == 1) {
+          // the first K range: wait for the partials of the pairs that did the rest
+          fx.n = sched_contributors(sc, f.t);
+          fx.p = args.sk_part + (pair + 1) * slot_floats;
+          fx.stride = slot_floats;
+          fx.rit = rit;
+          for (int q = 0; q < fx.n; ++q) {
+            int* flag = args.sk_flags + (pair + 1 + q) * 8 + fslot;
+            int ok = 1;
+            if (lane == 0) ok = wait_flag(flag, err) ? 1 : 0;
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) { fx.n = q; break; }  // warp-uniform
+            (void)ld_acquire_gpu(flag);     // every lane synchronises with the writer's release
+            __syncwarp();
+            if (lane == 0) *flag = 0;       // the only reader: leave the flags zero for the next launch
+          }
+        }
+        if (EPI == EPI_SCATTER_BF16)
+          epilogue_tile<BN, EPI>(args.e, taddr, row, row < M, nb, err, fx);
+        else
+          epilogue_tma<BN, EPI>(args.e, &tmO, taddr, row0, lane, row < M, nb, boxes, nbox, fx, err);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[acc]), 0));
     }
+    if (lane == 0) bulk_wait<0>();  // the staging boxes stay valid until every copy is done
   }
 
   tc_fence_before();
@@ -482,9 +906,43 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   }
 }
 
+constexpr size_t kSlotFloats = (size_t)2 * BM * 256;  // one 256 x 256 fp32 partial tile
+
+// Clusters of the pair kernel that fit on the device at once (0 if unknown).
+// The stream-K tail needs every pair resident: a pair finishing a tile waits
+// for pairs with higher indices.
 template <int BN, int EPI>
-cudaError_t launch_pair(const CUtensorMap& A, const CUtensorMap& B, const KArgs& a, int grid,
-                        cudaStream_t st) {
+int pair_max_clusters() {
+  static int cached_dev = -1, n = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev != cached_dev) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2, 1, 1);
+    cfg.blockDim = dim3(192, 1, 1);
+    cfg.dynamicSmemBytes = Cfg2<BN>::SMEM;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int c = 0;
+    if (cudaOccupancyMaxActiveClusters(&c, gemm_tc2_kernel<BN, EPI>, &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();
+      c = 0;
+    }
+    n = c;
+    cached_dev = dev;
+  }
+  return n;
+}
+
+// tiles: pair tiles for M_cap rows (an upper bound of the device row count).
+template <int BN, int EPI>
+cudaError_t launch_pair(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& O, KArgs a, int tiles,
+                        int slots, cudaStream_t st) {
   using C = Cfg2<BN>;
   static bool attr_done = false;
   if (!attr_done) {
@@ -493,8 +951,14 @@ cudaError_t launch_pair(const CUtensorMap& A, const CUtensorMap& B, const KArgs&
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
+  const int maxc = pair_max_clusters<BN, EPI>();
+  const int pairs = std::max(1, std::min(tiles, maxc > 0 ? maxc : device_sm_count() / 2));
+  if (maxc <= 0 || pairs > slots) {
+    a.sk_part = nullptr;
+    a.sk_flags = nullptr;
+  }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.gridDim = dim3(2 * pairs, 1, 1);
   cfg.blockDim = dim3(192, 1, 1);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
@@ -505,26 +969,26 @@ cudaError_t launch_pair(const CUtensorMap& A, const CUtensorMap& B, const KArgs&
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemm_tc2_kernel<BN, EPI>, A, B, a);
+  return cudaLaunchKernelEx(&cfg, gemm_tc2_kernel<BN, EPI>, A, B, O, a);
 }
 
 template <int BN>
-cudaError_t dispatch_pair(const CUtensorMap& A, const CUtensorMap& B, const KArgs& a, int grid,
-                          cudaStream_t st) {
+cudaError_t dispatch_pair(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& O, const KArgs& a,
+                          int tiles, int slots, cudaStream_t st) {
   switch (a.e.kind) {
-    case EPI_BF16: return launch_pair<BN, EPI_BF16>(A, B, a, grid, st);
-    case EPI_BF16_ROPE: return launch_pair<BN, EPI_BF16_ROPE>(A, B, a, grid, st);
-    case EPI_F32: return launch_pair<BN, EPI_F32>(A, B, a, grid, st);
-    case EPI_F32_ACC: return launch_pair<BN, EPI_F32_ACC>(A, B, a, grid, st);
-    case EPI_GELU_BF16: return launch_pair<BN, EPI_GELU_BF16>(A, B, a, grid, st);
-    case EPI_SWIGLU_BF16: return launch_pair<BN, EPI_SWIGLU_BF16>(A, B, a, grid, st);
-    case EPI_SCATTER_BF16: return launch_pair<BN, EPI_SCATTER_BF16>(A, B, a, grid, st);
+    case EPI_BF16: return launch_pair<BN, EPI_BF16>(A, B, O, a, tiles, slots, st);
+    case EPI_BF16_ROPE: return launch_pair<BN, EPI_BF16_ROPE>(A, B, O, a, tiles, slots, st);
+    case EPI_F32: return launch_pair<BN, EPI_F32>(A, B, O, a, tiles, slots, st);
+    case EPI_F32_ACC: return launch_pair<BN, EPI_F32_ACC>(A, B, O, a, tiles, slots, st);
+    case EPI_GELU_BF16: return launch_pair<BN, EPI_GELU_BF16>(A, B, O, a, tiles, slots, st);
+    case EPI_SWIGLU_BF16: return launch_pair<BN, EPI_SWIGLU_BF16>(A, B, O, a, tiles, slots, st);
+    case EPI_SCATTER_BF16: return launch_pair<BN, EPI_SCATTER_BF16>(A, B, O, a, tiles, slots, st);
     default: return cudaErrorInvalidValue;
   }
 }
 
 template <int BN, int EPI>
-cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const KArgs& a, int grid,
+cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& O, const KArgs& a, int grid,
                        cudaStream_t st) {
   using C = Cfg<BN>;
   static bool attr_done = false;  // per (BN, EPI) instantiation
@@ -534,21 +998,21 @@ cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const KArgs& 
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  gemm_tc_kernel<BN, EPI><<<grid, 192, C::SMEM, st>>>(A, B, a);
+  gemm_tc_kernel<BN, EPI><<<grid, 192, C::SMEM, st>>>(A, B, O, a);
   return cudaGetLastError();
 }
 
 template <int BN>
-cudaError_t dispatch(const CUtensorMap& A, const CUtensorMap& B, const KArgs& a, int grid,
+cudaError_t dispatch(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& O, const KArgs& a, int grid,
                      cudaStream_t st) {
   switch (a.e.kind) {
-    case EPI_BF16: return launch_one<BN, EPI_BF16>(A, B, a, grid, st);
-    case EPI_BF16_ROPE: return launch_one<BN, EPI_BF16_ROPE>(A, B, a, grid, st);
-    case EPI_F32: return launch_one<BN, EPI_F32>(A, B, a, grid, st);
-    case EPI_F32_ACC: return launch_one<BN, EPI_F32_ACC>(A, B, a, grid, st);
-    case EPI_GELU_BF16: return launch_one<BN, EPI_GELU_BF16>(A, B, a, grid, st);
-    case EPI_SWIGLU_BF16: return launch_one<BN, EPI_SWIGLU_BF16>(A, B, a, grid, st);
-    case EPI_SCATTER_BF16: return launch_one<BN, EPI_SCATTER_BF16>(A, B, a, grid, st);
+    case EPI_BF16: return launch_one<BN, EPI_BF16>(A, B, O, a, grid, st);
+    case EPI_BF16_ROPE: return launch_one<BN, EPI_BF16_ROPE>(A, B, O, a, grid, st);
+    case EPI_F32: return launch_one<BN, EPI_F32>(A, B, O, a, grid, st);
+    case EPI_F32_ACC: return launch_one<BN, EPI_F32_ACC>(A, B, O, a, grid, st);
+    case EPI_GELU_BF16: return launch_one<BN, EPI_GELU_BF16>(A, B, O, a, grid, st);
+    case EPI_SWIGLU_BF16: return launch_one<BN, EPI_SWIGLU_BF16>(A, B, O, a, grid, st);
+    case EPI_SCATTER_BF16: return launch_one<BN, EPI_SCATTER_BF16>(A, B, O, a, grid, st);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -561,6 +1025,16 @@ cudaError_t dispatch(const CUtensorMap& A, const CUtensorMap& B, const KArgs& a,
 // pair tiles lose (the MMA issue per stage no longer hides behind the MMA).
 // SP_GEMM_PAIRS=0 in the environment selects the single-CTA kernel (A/B runs);
 // SP_GEMM_PAIRS=1 allows 128-wide pair tiles where the column-tile count is small.
+// SP_GEMM_STREAMK=0 in the environment turns the stream-K tail off (A/B runs).
+static bool gemm_stream_k_enabled() {
+  static int mode = -1;
+  if (mode < 0) {
+    const char* s = getenv("SP_GEMM_STREAMK");
+    mode = s ? atoi(s) : 1;
+  }
+  return mode != 0;
+}
+
 int gemm_pair_policy(int M_cap, int N_acc, int kind) {
   static int mode = -1;
   if (mode < 0) {
@@ -572,6 +1046,25 @@ int gemm_pair_policy(int M_cap, int N_acc, int kind) {
   return (N_acc % 128 == 0 && mode == 1) ? 128 : 0;
 }
 
+size_t gemm_scratch_bytes() {
+  const size_t slots = (size_t)(device_sm_count() / 2);
+  return slots * kSlotFloats * sizeof(float) + slots * 8 * sizeof(int);
+}
+
+GemmScratch gemm_scratch_at(void* p) {
+  GemmScratch g;
+  if (!p) return g;
+  g.slots = device_sm_count() / 2;
+  g.part = static_cast<float*>(p);
+  g.flags = reinterpret_cast<int*>(g.part + (size_t)g.slots * kSlotFloats);
+  return g;
+}
+
+cudaError_t gemm_scratch_clear(const GemmScratch& g, cudaStream_t st) {
+  if (!g.flags) return cudaSuccess;
+  return cudaMemsetAsync(g.flags, 0, (size_t)g.slots * 8 * sizeof(int), st);
+}
+
 bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {
   b->N = N;
   b->K = K;
@@ -580,7 +1073,7 @@ bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {
 }
 
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B, int N_acc,
-                      const GemmEpi& e, int* err, cudaStream_t st) {
+                      const GemmEpi& e, int* err, cudaStream_t st, const GemmScratch* sk) {
   if (M_cap <= 0) return cudaSuccess;
   const int sms = device_sm_count();
   const int mt = (M_cap + BM - 1) / BM;
@@ -601,22 +1094,39 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
   a.K = B.K;
   a.e = e;
   a.err = err;
+  a.sk_part = nullptr;
+  a.sk_flags = nullptr;
+  // output map for the TMA epilogue (box 32 rows x 128 bytes); the row-scatter
+  // epilogue stores directly and needs none
+  CUtensorMap tmO;
+  std::memset(&tmO, 0, sizeof(tmO));
+  if (e.kind != EPI_SCATTER_BF16) {
+    const bool f32 = e.kind == EPI_F32 || e.kind == EPI_F32_ACC;
+    if (!encode_tmap_2d(&tmO, e.out, f32, (uint64_t)M_cap, (uint64_t)e.ldo, f32 ? 32 : 64, 32, nullptr))
+      return cudaErrorInvalidValue;
+  }
   cudaError_t r;
   const int pair_bn = gemm_pair_policy(M_cap, N_acc, e.kind);
   if (pair_bn) {
     const int mp = (M_cap + 2 * BM - 1) / (2 * BM);
     const int tiles = mp * (N_acc / pair_bn);
-    const int grid = 2 * std::max(1, std::min(tiles, sms / 2));
+    int slots = 0;
+    if (sk && sk->part && sk->flags && gemm_stream_k_enabled()) {
+      a.sk_part = sk->part;
+      a.sk_flags = sk->flags;
+      slots = sk->slots;
+    }
     prof_begin_launch(st);
-    r = pair_bn == 256 ? dispatch_pair<256>(A, B.map256, a, grid, st) : dispatch_pair<128>(A, B.map128, a, grid, st);
+    r = pair_bn == 256 ? dispatch_pair<256>(A, B.map256, tmO, a, tiles, slots, st)
+                       : dispatch_pair<128>(A, B.map128, tmO, a, tiles, slots, st);
     prof_end_launch(st, SP_K_GEMM, 2.0 * (double)M_cap * (double)N_acc * (double)B.K, 0.0);
     return r;
   }
   const int tiles = mt * (N_acc / (use256 ? 256 : 128));
   const int grid = std::max(1, std::min(tiles, sms));
   prof_begin_launch(st);
-  r = use256 ? dispatch<256>(A, B.map256, a, grid, st)
-             : dispatch<128>(A, B.map128, a, grid, st);
+  r = use256 ? dispatch<256>(A, B.map256, tmO, a, grid, st)
+             : dispatch<128>(A, B.map128, tmO, a, grid, st);
   double flops = 2.0 * (double)M_cap * (double)N_acc * (double)B.K;
   prof_end_launch(st, SP_K_GEMM, flops, 0.0);
   return r;

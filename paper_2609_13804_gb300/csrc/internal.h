@@ -32,6 +32,10 @@ bool prof_enabled();
 // ------------------------------------------------------------- tensor maps
 bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
                       uint32_t box_rows, std::string* msg);
+// 2-D map over a row-major [rows, cols] matrix of 2- or 4-byte elements with a
+// box of box_cols x box_rows and 128-byte swizzle (box_cols * esize <= 128).
+bool encode_tmap_2d(CUtensorMap* map, const void* ptr, bool f32, uint64_t rows, uint64_t cols,
+                    uint32_t box_cols, uint32_t box_rows, std::string* msg);
 
 // ------------------------------------------------------------- tcgen05 GEMM
 enum EpiKind {
@@ -72,8 +76,22 @@ int gemm_pair_policy(int M_cap, int N_acc, int kind);
 // rows 128.  M_dev (device int, may be NULL) bounds the rows actually computed;
 // M_cap bounds it on the host.  N_out is the accumulator width (N of B, or the
 // tile columns for SWIGLU: 2 F).
+// Scratch of the CTA-pair GEMM's stream-K tail: per SM pair one fp32 256 x 256
+// partial tile and 8 ready flags.  The flags must be zero when a GEMM starts;
+// every launch leaves them zero, so one gemm_scratch_clear per API call does.
+// Without scratch (NULL) the GEMM runs whole tiles only.
+struct GemmScratch {
+  float* part = nullptr;
+  int* flags = nullptr;
+  int slots = 0;
+};
+size_t gemm_scratch_bytes();
+GemmScratch gemm_scratch_at(void* p);  // p: gemm_scratch_bytes() bytes, 256-byte aligned (or NULL)
+cudaError_t gemm_scratch_clear(const GemmScratch& g, cudaStream_t st);
+
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B,
-                      int N_acc, const GemmEpi& e, int* err, cudaStream_t st);
+                      int N_acc, const GemmEpi& e, int* err, cudaStream_t st,
+                      const GemmScratch* sk = nullptr);
 
 // ------------------------------------------------------------- fp32 SIMT GEMM
 // C[M, N] = A[M, K] B[N, K]^T, fp32, row-major with leading dims.
