@@ -223,8 +223,12 @@ using namespace sp;
 struct sp_selector_s {
   sp_selector_cfg cfg;
   sp_selector_weights w;
-  float* Wcat1 = nullptr;  // [2h, D]  rows: W_in | Wq_p^T Wk_p / sqrt(h)
-  float* Wcat2 = nullptr;  // [3h, h]  rows: Wq_s / sqrt(h) | Wk_s | Wo_s Wv_s
+  // candidate precompute weights as six bf16 segments b0 b1 b0 b2 b1 b0 of
+  //   Wcat1 [2h, D]: rows W_in | Wq_p^T Wk_p / sqrt(h)
+  //   Wcat2 [3h, h]: rows Wq_s / sqrt(h) | Wk_s | Wo_s Wv_s
+  void* P1s = nullptr;  // [2h, 6D]
+  void* P2s = nullptr;  // [3h, 6h]
+  GemmB P1, P2;
   GemmB Wp;
   GemmB enc_qkv[SP_MAX_ENC_LAYERS], enc_o[SP_MAX_ENC_LAYERS], enc_1[SP_MAX_ENC_LAYERS],
       enc_2[SP_MAX_ENC_LAYERS];
@@ -300,12 +304,15 @@ sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weigh
   s->cfg = c;
   s->w = *w;
   const int h = c.h, D = c.D;
-  cudaError_t e = cudaMalloc(&s->Wcat1, (size_t)2 * h * D * sizeof(float));
-  if (e == cudaSuccess) e = cudaMalloc(&s->Wcat2, (size_t)3 * h * h * sizeof(float));
+  float *Wcat1 = nullptr, *Wcat2 = nullptr;
+  cudaError_t e = cudaMalloc(&Wcat1, (size_t)2 * h * D * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&Wcat2, (size_t)3 * h * h * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&s->P1s, (size_t)2 * h * 6 * D * sizeof(uint16_t));
+  if (e == cudaSuccess) e = cudaMalloc(&s->P2s, (size_t)3 * h * 6 * h * sizeof(uint16_t));
   const float rs = 1.0f / std::sqrt((float)h);
-  if (e == cudaSuccess) e = cudaMemcpy2D(s->Wcat1, D * sizeof(float), w->W_in, D * sizeof(float), D * sizeof(float), h, cudaMemcpyDeviceToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy2D(Wcat1, D * sizeof(float), w->W_in, D * sizeof(float), D * sizeof(float), h, cudaMemcpyDeviceToDevice);
   // Wq_p^T Wk_p / sqrt(h): (i, j) = sum_k Wq_p[k, i] Wk_p[k, j]
-  if (e == cudaSuccess) e = fold_matmul(w->Wq_p, 1, h, w->Wk_p, D, 1, s->Wcat1 + (size_t)h * D, D, h, D, h, rs, 0);
+  if (e == cudaSuccess) e = fold_matmul(w->Wq_p, 1, h, w->Wk_p, D, 1, Wcat1 + (size_t)h * D, D, h, D, h, rs, 0);
   // Wq_s / sqrt(h), as Wq_s times the identity through the same fold kernel
   std::vector<float> eye;
   float* dI = nullptr;
@@ -315,19 +322,23 @@ sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weigh
     e = cudaMalloc(&dI, (size_t)h * h * sizeof(float));
     if (e == cudaSuccess) e = cudaMemcpy(dI, eye.data(), eye.size() * sizeof(float), cudaMemcpyHostToDevice);
   }
-  if (e == cudaSuccess) e = fold_matmul(w->Wq_s, h, 1, dI, h, 1, s->Wcat2, h, h, h, h, rs, 0);
-  if (e == cudaSuccess) e = cudaMemcpy(s->Wcat2 + (size_t)h * h, w->Wk_s, (size_t)h * h * sizeof(float), cudaMemcpyDeviceToDevice);
+  if (e == cudaSuccess) e = fold_matmul(w->Wq_s, h, 1, dI, h, 1, Wcat2, h, h, h, h, rs, 0);
+  if (e == cudaSuccess) e = cudaMemcpy(Wcat2 + (size_t)h * h, w->Wk_s, (size_t)h * h * sizeof(float), cudaMemcpyDeviceToDevice);
   // Wo_s Wv_s: (i, j) = sum_k Wo_s[i, k] Wv_s[k, j]
-  if (e == cudaSuccess) e = fold_matmul(w->Wo_s, h, 1, w->Wv_s, h, 1, s->Wcat2 + (size_t)2 * h * h, h, h, h, h, 1.f, 0);
+  if (e == cudaSuccess) e = fold_matmul(w->Wo_s, h, 1, w->Wv_s, h, 1, Wcat2 + (size_t)2 * h * h, h, h, h, h, 1.f, 0);
+  if (e == cudaSuccess) e = split6_weights(Wcat1, 2 * h, D, s->P1s, 0);
+  if (e == cudaSuccess) e = split6_weights(Wcat2, 3 * h, h, s->P2s, 0);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (dI) cudaFree(dI);
+  if (Wcat1) cudaFree(Wcat1);
+  if (Wcat2) cudaFree(Wcat2);
   if (e != cudaSuccess) {
     sp_selector_destroy(s);
     return cuda_fail(e, "sp_selector_create (fold)");
   }
   std::string msg;
-  bool ok = true;
-  if (c.n_enc_layers > 0) {
+  bool ok = make_gemm_b(&s->P1, s->P1s, 2 * h, 6 * D, &msg) && make_gemm_b(&s->P2, s->P2s, 3 * h, 6 * h, &msg);
+  if (ok && c.n_enc_layers > 0) {
     ok = make_gemm_b(&s->Wp, w->W_p, D, c.D_text, &msg);
     for (int i = 0; ok && i < c.n_enc_layers; ++i) {
       ok = make_gemm_b(&s->enc_qkv[i], w->enc_wqkv[i], 3 * D, D, &msg) &&
@@ -346,8 +357,8 @@ sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weigh
 
 void sp_selector_destroy(sp_selector* s) {
   if (!s) return;
-  if (s->Wcat1) cudaFree(s->Wcat1);
-  if (s->Wcat2) cudaFree(s->Wcat2);
+  if (s->P1s) cudaFree(s->P1s);
+  if (s->P2s) cudaFree(s->P2s);
   delete s;
 }
 
@@ -383,7 +394,7 @@ size_t select_ws(const sp_selector* s, const SelPlan& p, const sp_select_out* ou
   float *P = nullptr, *R = nullptr, *Mall, *ZK, *XL, *QKVs;
   void *Abf = nullptr, *QKV = nullptr, *O = nullptr, *F1 = nullptr;
   int* enc_cu = nullptr;
-  void* gsk = nullptr;
+  void* gsk = nullptr;  // stream-K scratch of the encoder GEMMs (the precompute GEMMs run whole tiles)
   if (p.encoder && s->cfg.n_enc_layers > 0) {
     gsk = cv.take<char>(gemm_scratch_bytes());
     P = cv.take<float>((size_t)std::max(p.ntxt, 1) * D);
@@ -400,12 +411,13 @@ size_t select_ws(const sp_selector* s, const SelPlan& p, const sp_select_out* ou
   ZK = cv.take<float>((size_t)p.rows * 2 * h);
   XL = cv.take<float>((size_t)p.rows * h);
   QKVs = cv.take<float>((size_t)p.rows * 3 * h);
+  void* Asp = cv.take<uint16_t>((size_t)p.rows * 3 * std::max(D, h));  // split operand of the precompute GEMMs
   int* order = (out && out->order) ? nullptr : cv.take<int>((size_t)p.E * SP_MAX_KMAX);
   int* epc = (out && out->ep_count) ? nullptr : cv.take<int>((size_t)p.E);
   if (parts) {
     parts[0] = P; parts[1] = R; parts[2] = Abf; parts[3] = QKV; parts[4] = O; parts[5] = F1;
     parts[6] = enc_cu; parts[7] = Mall; parts[8] = ZK; parts[9] = XL; parts[10] = QKVs;
-    parts[11] = order; parts[12] = epc; parts[13] = gsk;
+    parts[11] = order; parts[12] = epc; parts[13] = gsk; parts[14] = Asp;
   }
   return cv.off;
 }
@@ -422,8 +434,7 @@ sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPla
   void* O = parts[4];
   void* F1 = parts[5];
   int* enc_cu = (int*)parts[6];
-  const GemmScratch gs = gemm_scratch_at(parts[13]);
-  SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
+  const GemmScratch gs = gemm_scratch_at(parts[13]);  // cleared by the caller
   std::string msg;
   if (p.ntxt > 0) {
     CUtensorMap tE;
@@ -495,12 +506,14 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   }
   if (out->k_cap < need_cap) return fail(SP_ERR_SHAPE, "sp_select: k_cap %d < largest possible count %d", out->k_cap, need_cap);
   Carve cv(ws);
-  void* parts[14];
+  void* parts[15];
   const size_t need = select_ws(s, p, out, cv, parts) + 256;
   if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_select: workspace %zu < %zu bytes", ws_bytes, need);
   if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_select: workspace must be 16-byte aligned");
   int* err = out->err;
   const int D = s->cfg.D, h = s->cfg.h;
+  const GemmScratch gs = gemm_scratch_at(parts[13]);
+  SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
 
   if (p.encoder && s->cfg.n_enc_layers > 0) {
     rs = run_encoder(s, in, p, parts, err, st);
@@ -524,9 +537,28 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   float* QKVs = (float*)parts[10];
   // candidate precompute (fp32): [z | KT] = M [W_in; Wq_p^T Wk_p / sqrt h]^T, x = LN1(z),
   // [QS | KS | VT] = x [Wq_s / sqrt h; Wk_s; Wo_s Wv_s]^T
-  SP_CUDA(sgemm_f32(Mall, D, s->Wcat1, D, ZK, 2 * h, p.rows, 2 * h, D, st), "precompute 1");
-  SP_CUDA(layernorm_f32(ZK, 2 * h, s->w.ln1_g, s->w.ln1_b, XL, nullptr, h, p.rows, h, s->cfg.ln_eps, 1.f, st), "ln1");
-  SP_CUDA(sgemm_f32(XL, h, s->Wcat2, h, QKVs, 3 * h, p.rows, 3 * h, h, st), "precompute 2");
+  // (fp32-accurate products on the bf16 tensor cores: three-way operand split)
+  {
+    void* Asp = parts[14];
+    std::string msg;
+    CUtensorMap t1, t2;
+    if (!encode_tmap_bf16(&t1, Asp, p.rows, 3 * D, 128, &msg) || !encode_tmap_bf16(&t2, Asp, p.rows, 3 * h, 128, &msg))
+      return fail(SP_ERR_CUDA, "%s", msg.c_str());
+    GemmEpi e1;
+    e1.kind = EPI_F32;
+    e1.out = ZK;
+    e1.ldo = 2 * h;
+    const GemmASplit a1 = split3_a_map(D), a2 = split3_a_map(h);
+    SP_CUDA(split3_bf16(Mall, D, p.rows, D, Asp, st), "precompute split 1");
+    SP_CUDA(gemm_bf16(t1, p.rows, nullptr, s->P1, 2 * h, e1, err, st, nullptr, &a1), "precompute 1");
+    SP_CUDA(layernorm_f32(ZK, 2 * h, s->w.ln1_g, s->w.ln1_b, XL, nullptr, h, p.rows, h, s->cfg.ln_eps, 1.f, st), "ln1");
+    GemmEpi e2;
+    e2.kind = EPI_F32;
+    e2.out = QKVs;
+    e2.ldo = 3 * h;
+    SP_CUDA(split3_bf16(XL, h, p.rows, h, Asp, st), "precompute split 2");
+    SP_CUDA(gemm_bf16(t2, p.rows, nullptr, s->P2, 3 * h, e2, err, st, nullptr, &a2), "precompute 2");
+  }
 
   SelectArgs a;
   a.Z = ZK; a.ldz = 2 * h;

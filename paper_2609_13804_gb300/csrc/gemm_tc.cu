@@ -55,9 +55,18 @@ struct KArgs {
   int K;
   GemmEpi e;
   int* err;
+  int a_seg;       // A k-segment remap (GemmASplit); 0: none
+  uint32_t a_map;
   float* sk_part;  // pair kernel: stream-K partial tiles [pairs][256][BN] (NULL: whole tiles only)
   int* sk_flags;   // pair kernel: [pairs][8] ready flags, zero between launches
 };
+
+// Column of A's tensor map holding the GEMM's k-coordinate k.
+SP_DEVINL int a_col(const KArgs& a, int k) {
+  if (a.a_seg == 0) return k;
+  const int s = k / a.a_seg;
+  return (int)((a.a_map >> (4 * s)) & 15u) * a.a_seg + (k - s * a.a_seg);
+}
 
 // Partial sums other pairs computed for this tile (stream-K tail): `n` slots,
 // `stride` floats apart, from the slot of the first.  A slot holds a 256-row
@@ -495,7 +504,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, err)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[s], C::A_BYTES + C::B_BYTES);
-          tma_load_2d(sA + s * C::A_BYTES, &tmA, &full[s], kb * BK, m0);
+          tma_load_2d(sA + s * C::A_BYTES, &tmA, &full[s], a_col(args, kb * BK), m0);
           tma_load_2d(sB + s * C::B_BYTES, &tmB, &full[s], kb * BK, b0);
           tma_load_2d(sB + s * C::B_BYTES + C::B_BYTES / 2, &tmB, &full[s], kb * BK, b1);
           ++issued;
@@ -789,7 +798,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
           if (!mbar_wait(&empty[s], ph ^ 1u, err)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[s], 2 * (C::A_BYTES + C::B_BYTES));
           const uint32_t bar = mapa_shared(smem_u32(&full[s]), 0);
-          tma_load_2d_pair(sA + s * C::A_BYTES, &tmA, bar, kb * BK, a_row);
+          tma_load_2d_pair(sA + s * C::A_BYTES, &tmA, bar, a_col(args, kb * BK), a_row);
           tma_load_2d_pair(sB + s * C::B_BYTES, &tmB, bar, kb * BK, b_row);
           if (++s == C::STAGES) { s = 0; ph ^= 1u; }
         }
@@ -1073,7 +1082,8 @@ bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {
 }
 
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B, int N_acc,
-                      const GemmEpi& e, int* err, cudaStream_t st, const GemmScratch* sk) {
+                      const GemmEpi& e, int* err, cudaStream_t st, const GemmScratch* sk,
+                      const GemmASplit* as) {
   if (M_cap <= 0) return cudaSuccess;
   const int sms = device_sm_count();
   const int mt = (M_cap + BM - 1) / BM;
@@ -1096,6 +1106,13 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
   a.err = err;
   a.sk_part = nullptr;
   a.sk_flags = nullptr;
+  a.a_seg = 0;
+  a.a_map = 0;
+  if (as && as->seg > 0) {
+    if (as->seg % BK != 0 || B.K > 8 * as->seg) return cudaErrorInvalidValue;
+    a.a_seg = as->seg;
+    a.a_map = as->map;
+  }
   // output map for the TMA epilogue (box 32 rows x 128 bytes); the row-scatter
   // epilogue stores directly and needs none
   CUtensorMap tmO;

@@ -89,15 +89,25 @@ size_t gemm_scratch_bytes();
 GemmScratch gemm_scratch_at(void* p);  // p: gemm_scratch_bytes() bytes, 256-byte aligned (or NULL)
 cudaError_t gemm_scratch_clear(const GemmScratch& g, cudaStream_t st);
 
+// K-segment map of the A operand: A's k-coordinate k (of the GEMM's K = B.K)
+// lies in segment s = k / seg and is read from column ((map >> 4s) & 15) * seg
+// + k % seg of A's tensor map (seg = 0: identity).  Lets one stored copy of a
+// part feed several K segments (the split fp32 product, precompute.cu).
+struct GemmASplit {
+  int seg = 0;
+  uint32_t map = 0;
+};
+
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B,
                       int N_acc, const GemmEpi& e, int* err, cudaStream_t st,
-                      const GemmScratch* sk = nullptr);
+                      const GemmScratch* sk = nullptr, const GemmASplit* as = nullptr);
 
-// ------------------------------------------------------------- fp32 SIMT GEMM
-// C[M, N] = A[M, K] B[N, K]^T, fp32, row-major with leading dims.
-cudaError_t sgemm_f32(const float* A, int lda, const float* B, int ldb, float* C, int ldc, int M,
-                      int N, int K, cudaStream_t st);
-// C[i, j] = scale * sum_k A(i, k) B(k, j), fp64 accumulation, arbitrary strides (set-up only).
+// ------------------------------------------------------------- candidate precompute
+// out [rows, 3K] bf16 = the three bf16 parts of x [rows, K] (fp32, row stride ldx).
+cudaError_t split3_bf16(const float* x, int ldx, int rows, int K, void* out, cudaStream_t st);
+// out [N, 6K] bf16 = the weight segments b0 b1 b0 b2 b1 b0 of w [N, K] (fp32).
+cudaError_t split6_weights(const float* w, int N, int K, void* out, cudaStream_t st);
+GemmASplit split3_a_map(int K);
 cudaError_t fold_matmul(const float* A, long sai, long sak, const float* B, long sbk, long sbj,
                         float* C, int ldc, int I, int J, int K, float scale, cudaStream_t st);
 
