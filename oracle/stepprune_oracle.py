@@ -29,6 +29,8 @@ Parity status of each function:
   rope                                  pinned (rotation closed form, relative-position property)
   round_bf16                            pinned (torch's float32 -> bfloat16 conversion)
   projector, prefill_layer, prefill     pinned through their parts plus special cases
+                                        (acc='fp32' variant: pinned against acc='fp64'
+                                        to fp32 precision)
                                         (zero output weights -> identity; uniform attention);
                                         the composition of a whole random-weight LM is
                                         parity unpinned beyond those checks.
@@ -418,18 +420,31 @@ def rope(x, pos, n_heads: int, head_dim: int, theta: float) -> np.ndarray:
     return np.concatenate([a * c - b * s, b * c + a * s], axis=-1).reshape(x.shape[0], -1)
 
 
-def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = None) -> np.ndarray:
+def _mm(a, b, acc: str) -> np.ndarray:
+    """a @ b with fp64 arithmetic, or (acc='fp32') with fp32 operands and an
+    fp32 result, the precision of a tensor-core product's accumulator."""
+    if acc == "fp64":
+        return a @ b
+    if acc == "fp32":
+        return (np.asarray(a, np.float32) @ np.asarray(b, np.float32)).astype(F64)
+    raise ValueError(acc)
+
+
+def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = None,
+                  acc: str = "fp64") -> np.ndarray:
     """One pre-norm decoder layer of the frozen LM over the packed sequences:
     h += Wo Attn(RoPE(Wq x), RoPE(Wk x), Wv x), x = RMSNorm(h);
     h += Wdown (SiLU(Wg x') * Wu x'), x' = RMSNorm(h).  Attention is causal and
     never crosses a sequence boundary.  The residual stream h stays fp64; with
     store='bf16' the activations a bf16 model keeps between ops (normalised
     inputs, rotated q / k, v, attention output, SwiGLU output) are rounded to
-    bf16 where they are stored."""
+    bf16 where they are stored.  acc='fp32' computes the four projections in
+    fp32 instead of fp64 (used only to size how far two exact bf16 prefills
+    drift apart through rounding decisions alone)."""
     h = _f(h).copy()
     Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
     x = _store(rms_norm(h, m.rms_eps, L.get("attn_norm")), store)
-    qkv = x @ _f(L["Wqkv"]).T
+    qkv = _mm(x, _f(L["Wqkv"]).T, acc)
     q = _store(rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta), store)
     k = _store(rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta), store)
     v = _store(qkv[:, (Hq + Hkv) * dh:], store)
@@ -438,10 +453,10 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
         s, e = int(cu[b]), int(cu[b + 1])
         if e > s:
             o[s:e] = attention(q[s:e], k[s:e], v[s:e], Hq, Hkv, causal=True)
-    h = h + _store(o, store) @ _f(L["Wo"]).T
+    h = h + _mm(_store(o, store), _f(L["Wo"]).T, acc)
     x2 = _store(rms_norm(h, m.rms_eps, L.get("mlp_norm")), store)
-    gu = x2 @ _f(L["Wgu"]).T
-    h = h + _store(silu(gu[:, :F]) * gu[:, F:], store) @ _f(L["Wdown"]).T
+    gu = _mm(x2, _f(L["Wgu"]).T, acc)
+    h = h + _mm(_store(silu(gu[:, :F]) * gu[:, F:], store), _f(L["Wdown"]).T, acc)
     return h
 
 
@@ -451,10 +466,11 @@ def final_norm(h, m, gain=None) -> np.ndarray:
     return rms_norm(h, m.rms_eps, gain)
 
 
-def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None, store: Optional[str] = None) -> np.ndarray:
+def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None, store: Optional[str] = None,
+            acc: str = "fp64") -> np.ndarray:
     h = _f(x)
     for L in layers:
-        h = prefill_layer(h, L, m, cu, pos, store)
+        h = prefill_layer(h, L, m, cu, pos, store, acc)
     return final_norm(h, m, final_gain)
 
 

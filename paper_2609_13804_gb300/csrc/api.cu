@@ -460,7 +460,8 @@ sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPla
     e1.out = QKV;
     e1.ldo = 3 * D;
     SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_qkv[l], 3 * D, e1, err, st, &gs), "enc qkv");
-    SP_CUDA(attention_varlen(QKV, O, enc_cu, in->B, p.max_enc, nh, nh, c.enc_head_dim, false, st), "enc attention");
+    SP_CUDA(attention_varlen(QKV, O, enc_cu, in->B, p.max_enc, p.T_enc, nh, nh, c.enc_head_dim, false, err, st),
+            "enc attention");
     GemmEpi e2;
     e2.kind = EPI_F32_ACC;
     e2.out = R;
@@ -836,6 +837,9 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
   const GemmScratch gs = gemm_scratch_at(p.gsk);
   SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   SP_CUDA(bf16_to_f32(io->x, h32, T_cap, T_dev, c.d, st), "embed");
+  // the attention's last key tile reads up to 63 rows past the packed length
+  // (weighted by zero); keep them finite: the QKV GEMMs leave them untouched
+  SP_CUDA(zero_rows_after(p.qkv, (size_t)qkvw * 2, T_dev, T_cap, 64, st), "qkv tail");
   for (int l = 0; l < c.n_layers; ++l) {
     SP_CUDA(rmsnorm_f32_to_bf16(h32, m->w.attn_norm[l], p.xb, T_cap, T_dev, c.d, c.rms_eps, st), "attn norm");
     GemmEpi eq;
@@ -848,8 +852,8 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
     SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->qkv[l], qkvw, eq, io->err, st, &gs), "qkv");
-    SP_CUDA(attention_varlen(p.qkv, p.ob, io->cu_seqlens, io->B, io->max_seqlen_cap, c.n_heads, c.n_kv_heads,
-                             c.head_dim, true, st), "attention");
+    SP_CUDA(attention_varlen(p.qkv, p.ob, io->cu_seqlens, io->B, io->max_seqlen_cap, T_cap, c.n_heads, c.n_kv_heads,
+                             c.head_dim, true, io->err, st), "attention");
     GemmEpi er;
     er.kind = EPI_F32_ACC;
     er.out = h32;

@@ -120,6 +120,9 @@ cudaError_t rmsnorm_f32_to_f32(const float* x, const float* gain, float* out, in
 cudaError_t layernorm_f32(const float* x, int ldx, const float* gain, const float* bias, float* out_f32,
                           void* out_bf16, int ldo, int rows, int d, float eps, float scale,
                           cudaStream_t st);
+// Zeroes rows [T, T + nrows) (below rows_cap) of a row-major buffer, T = *row_count.
+cudaError_t zero_rows_after(void* buf, size_t row_bytes, const int* row_count, int rows_cap, int nrows,
+                            cudaStream_t st);
 cudaError_t bf16_to_f32(const void* x, float* out, int rows_cap, const int* row_count, int d,
                         cudaStream_t st);
 cudaError_t assemble_encoder_input(const BatchDesc& bd, const void* X, const float* P, int D,
@@ -130,10 +133,11 @@ cudaError_t gather_memory(const BatchDesc& bd, const float* R, const float* H, c
 cudaError_t write_enc_cu(const BatchDesc& bd, int* cu, cudaStream_t st);
 
 // ------------------------------------------------------------- attention
-// Varlen attention over packed qkv [T, (Hq + 2 Hkv) dh] bf16 -> out [T, Hq dh] bf16.
+// Varlen attention over packed qkv [rows_cap, (Hq + 2 Hkv) dh] bf16 -> out [T, Hq dh] bf16
+// (rows of sequence b from cu_seqlens[b]; rows_cap bounds the buffer for TMA).
 cudaError_t attention_varlen(const void* qkv, void* out, const int* cu_seqlens, int B,
-                             int max_seqlen_cap, int Hq, int Hkv, int dh, bool causal,
-                             cudaStream_t st);
+                             int max_seqlen_cap, int rows_cap, int Hq, int Hkv, int dh, bool causal,
+                             int* err, cudaStream_t st);
 
 // ------------------------------------------------------------- selection
 struct SelectArgs {

@@ -105,6 +105,14 @@ __global__ void bf16_to_f32_kernel(const uint2* __restrict__ x, float4* __restri
   }
 }
 
+// Rows [T, T + gridDim.x) of a row-major buffer, T = *row_count, below rows_cap, set to zero.
+__global__ void zero_rows_after_kernel(uint4* __restrict__ buf, int row_u4, const int* __restrict__ row_count,
+                                       int rows_cap) {
+  const int row = __ldg(row_count) + blockIdx.x;
+  if (row < 0 || row >= rows_cap) return;
+  for (int i = threadIdx.x; i < row_u4; i += blockDim.x) buf[(size_t)row * row_u4 + i] = make_uint4(0, 0, 0, 0);
+}
+
 SP_DEVINL int find_image(const int* off, int B, int r) {
   // largest b with off[b] <= r
   int lo = 0, hi = B - 1;
@@ -216,6 +224,17 @@ cudaError_t layernorm_f32(const float* x, int ldx, const float* gain, const floa
   layernorm_kernel<<<rows, NT, d * sizeof(float), st>>>(x, ldx, gain, bias, out_f32, out_bf16, ldo, rows,
                                                         d, eps, scale);
   prof_end_launch(st, SP_K_NORM, 0.0, 6.0 * rows * (double)d);
+  return cudaGetLastError();
+}
+
+cudaError_t zero_rows_after(void* buf, size_t row_bytes, const int* row_count, int rows_cap, int nrows,
+                            cudaStream_t st) {
+  if (rows_cap <= 0 || nrows <= 0) return cudaSuccess;
+  if (row_bytes % 16 != 0) return cudaErrorInvalidValue;
+  prof_begin_launch(st);
+  zero_rows_after_kernel<<<nrows, 256, 0, st>>>(reinterpret_cast<uint4*>(buf), (int)(row_bytes / 16), row_count,
+                                                 rows_cap);
+  prof_end_launch(st, SP_K_MISC, 0.0, (double)nrows * row_bytes);
   return cudaGetLastError();
 }
 

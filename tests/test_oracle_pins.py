@@ -366,6 +366,20 @@ def test_prefill_varlen_isolation_and_causality():
     np.testing.assert_allclose(pert[6:], both[6:], atol=1e-12)
 
 
+def test_prefill_fp32_accumulation_variant_is_fp32_close():
+    """acc='fp32' only lowers the projections' precision: without storage
+    rounding it matches the fp64 layer to fp32 round-off, and it is not the
+    fp64 layer bit for bit (the option reaches the matmuls)."""
+    w, L = _tiny_lm(16)
+    m = w.model
+    x = S.normal(16, "x", (10, m.d)).astype(np.float64)
+    cu, pos = [0, 10], np.arange(10)
+    a = O.prefill(x, [L, L], m, cu, pos)
+    b = O.prefill(x, [L, L], m, cu, pos, acc="fp32")
+    np.testing.assert_allclose(b, a, rtol=1e-4, atol=1e-5)
+    assert np.abs(b - a).max() > 0.0
+
+
 def test_projector_forms():
     w = S.tiny_workload(15, [4], [2], D=12, d=20)
     head = S.make_model_head(w)
