@@ -79,7 +79,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   const int b = blockIdx.z, h = blockIdx.y;
   const int s0 = __ldg(cu + b);
   const int len = __ldg(cu + b + 1) - s0;
-  const int q0 = blockIdx.x * BQ;
+  // causal: the last query tiles see the most keys; launch them first
+  const int q0 = (gridDim.x - 1 - blockIdx.x) * BQ;
   if (q0 >= len) return;
   const int kvh = h / (Hq / Hkv);
   const int qcol = h * DH, kcol = (Hq + kvh) * DH, vcol = (Hq + Hkv + kvh) * DH;
