@@ -196,6 +196,44 @@ def cpu_oracle_sample(w, n_images=1, n_layers=1):
     return per_image_ms * w.B, t_sel + t_proj + t_lm
 
 
+def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
+    """The selection kernel against its on-chip roofline: algorithmic bytes per
+    round per episode are the folded pointer keys of its candidates, (N_e + 1) h
+    fp32 from shared memory, plus the history rows the round's attention reads,
+    2 t h fp32 from L2 (t = history length); the kernel's time is the longest
+    episode's rounds.  Peaks and the synchronisation floor come from the
+    library's probes."""
+    r = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bias, group_size=w.group_size, g=w.g,
+                    k_max=w.k_max)
+    import torch
+    torch.cuda.synchronize()
+    rounds = r["rounds"].cpu().numpy().astype(int)
+    h = w.selector.h
+    eps = w.episodes()
+    smem_b = l2_b = 0.0
+    for (_, _, n_e), R in zip(eps, rounds):
+        for t_round in range(int(R)):
+            t = min(1 + w.g * t_round, w.k_max)
+            smem_b += (n_e + 1) * h * 4.0
+            l2_b += 2.0 * t * h * 4.0
+    n_max = max(n for (_, _, n) in eps)
+    C = 8 if (n_max + 7) // 8 + 1 <= 128 else 16
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    smem_peak = B.probe_smem_gbs()
+    l2_peak = B.probe_l2_gbs()
+    r_max = int(rounds.max())
+    floor_us = B.probe_select_floor(C, h, max(r_max, 1), len(eps))
+    ks = kernel_ms * 1e-3
+    used = min(len(eps) * C, sms) / sms
+    return {"kernel_ms": kernel_ms, "episodes": len(eps), "cluster_size": C, "max_rounds": r_max,
+            "us_per_round": kernel_ms * 1e3 / max(r_max, 1), "floor_us_per_round": floor_us,
+            "smem_bytes": smem_b, "l2_bytes": l2_b,
+            "smem_gbs": smem_b / ks / 1e9, "l2_gbs": l2_b / ks / 1e9,
+            "smem_peak_gbs": smem_peak, "smem_peak_used_sms_gbs": smem_peak * used, "l2_peak_gbs": l2_peak,
+            "smem_frac_of_used_sms": smem_b / ks / 1e9 / (smem_peak * used), "l2_frac": l2_b / ks / 1e9 / l2_peak,
+            "note": "latency-bound dependent chain: compare us_per_round with floor_us_per_round"}
+
+
 def cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -351,6 +389,7 @@ def run_ours(args):
     sel_out = do_select()
     select_ms = timed(do_select)
     k_cap = pipe.k_cap
+    sel_report = selection_report(B, w, selector, X, E, bias, prof["select"]["ms"] / args.steps, dev)
     comp = {}
 
     def do_compact(idx, count, kc):
@@ -359,9 +398,12 @@ def run_ours(args):
 
     def kernel_ms(fn, kind, reps=5):
         # device time of the launches of one kind (events around each launch on
-        # its stream), free of the binding's host overhead between calls
+        # its stream): a spin kernel ahead of them keeps the GPU busy while the
+        # host enqueues the calls, so no launch waits on the host inside a pair
+        # of events
         fn()
         torch.cuda.synchronize()
+        torch.cuda._sleep(4_000_000)
         B.sp_profile_begin(reps * 16)
         for _ in range(reps):
             fn()
@@ -438,6 +480,7 @@ def run_ours(args):
             "stages_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()},
             "ms_per_step_with_launch_events": ms_step_profiled,
             "select_us_per_image": 1e3 * select_ms / w.B,
+            "selection": sel_report,
             "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,
             "compaction_full_prefix_gbs": full_comp_bytes / (full_compact_ms * 1e-3) / 1e9,
             "compaction_full_prefix_hbm_frac": full_comp_bytes / (full_compact_ms * 1e-3) / 1e9 / pk["hbm_gbs"],

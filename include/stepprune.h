@@ -416,6 +416,29 @@ SP_API sp_status sp_profile_begin(int capacity);
  * summed milliseconds, launch counts and algorithmic flops / bytes. */
 SP_API sp_status sp_profile_end(double* ms, long long* launches, double* flops, double* bytes);
 
+/* ------------------------------------------------------------------ measurement probes
+ * Not part of the method (the paper has no counterpart): the on-chip peaks the
+ * selection kernel's traffic is measured against, and the per-round floor of
+ * its cluster synchronisation.  Each call allocates its own buffers on the
+ * current device, runs, synchronises the device and returns the figure; use
+ * them outside timed regions.  Errors: SP_ERR_INVALID_ARG (NULL output),
+ * SP_ERR_SHAPE (sizes out of range), SP_ERR_CUDA. */
+
+/* Aggregate shared-memory read bandwidth of the device (GB/s): two CTAs per
+ * SM stream 16-byte reads over a 64 KB buffer each. */
+SP_API sp_status sp_probe_smem_gbs(double* gbs);
+
+/* Read bandwidth from an L2-resident 48 MB buffer (GB/s, all SMs, 16-byte
+ * cache-global loads). */
+SP_API sp_status sp_probe_l2_gbs(double* gbs);
+
+/* Microseconds per round of the selection loop's synchronisation alone:
+ * `episodes` clusters of `cluster_size` (8 or 16) CTAs of 256 threads, each
+ * round two DSMEM push exchanges (h floats, then a short list, into every CTA
+ * of the cluster), two cluster barriers and the block reductions, no
+ * candidate or history work.  h in 128..1024, rounds >= 1. */
+SP_API sp_status sp_probe_select_floor(int cluster_size, int h, int rounds, int episodes, double* us_per_round);
+
 #ifdef __cplusplus
 }
 #endif

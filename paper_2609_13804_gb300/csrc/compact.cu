@@ -15,11 +15,27 @@ namespace {
 
 constexpr int NT = 256;
 
+// One row, 16-byte chunks per lane; eight loads are issued before their stores
+// so a warp keeps up to 4 KB in flight instead of one chunk per round trip.
 SP_DEVINL void copy_row(const uint4* __restrict__ src, uint4* __restrict__ dst, int n16, int lane) {
-  for (int i = lane; i < n16; i += 32) dst[i] = __ldg(src + i);
+  int i = lane;
+  for (; i + 7 * 32 < n16; i += 8 * 32) {
+    uint4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = __ldg(src + i + u * 32);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) dst[i + u * 32] = v[u];
+  }
+  uint4 v[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u)
+    if (i + u * 32 < n16) v[u] = __ldg(src + i + u * 32);
+#pragma unroll
+  for (int u = 0; u < 8; ++u)
+    if (i + u * 32 < n16) dst[i + u * 32] = v[u];
 }
 
-__global__ void __launch_bounds__(NT)
+__global__ void __launch_bounds__(NT, 4)
 compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vis,
                const __nv_bfloat16* __restrict__ text, int W_txt, const int* __restrict__ idx, int k_cap,
                const int* __restrict__ count, __nv_bfloat16* __restrict__ packed, int* __restrict__ cu,
@@ -79,6 +95,9 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
     const int b = lo;
     const int local = r - s_cu[b];
     if (lane == 0) pos[r] = local;
+    const uint4* src;
+    uint4* dst;
+    int n16;
     if (local < s_cnt[b]) {
       const int j = __ldg(idx + (size_t)b * k_cap + local);
       const int n_img = bd.vis_off[b + 1] - bd.vis_off[b];
@@ -86,19 +105,21 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
         if (lane == 0) set_error(err, SP_DEVERR_INDEX);
         continue;
       }
-      const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)(bd.vis_off[b] + j) * W_vis);
+      src = reinterpret_cast<const uint4*>(X + (size_t)(bd.vis_off[b] + j) * W_vis);
+      n16 = nv16;
       if (vis_packed) {
         const int vr = s_vcu[b] + local;
         if (lane == 0) vis_row_map[vr] = r;
-        copy_row(src, reinterpret_cast<uint4*>(vis_packed + (size_t)vr * W_vis), nv16, lane);
+        dst = reinterpret_cast<uint4*>(vis_packed + (size_t)vr * W_vis);
       } else {
-        copy_row(src, reinterpret_cast<uint4*>(packed + (size_t)r * W_txt), nv16, lane);
+        dst = reinterpret_cast<uint4*>(packed + (size_t)r * W_txt);
       }
     } else {
-      const uint4* src =
-          reinterpret_cast<const uint4*>(text + (size_t)(bd.txt_off[b] + local - s_cnt[b]) * W_txt);
-      copy_row(src, reinterpret_cast<uint4*>(packed + (size_t)r * W_txt), nt16, lane);
+      src = reinterpret_cast<const uint4*>(text + (size_t)(bd.txt_off[b] + local - s_cnt[b]) * W_txt);
+      dst = reinterpret_cast<uint4*>(packed + (size_t)r * W_txt);
+      n16 = nt16;
     }
+    copy_row(src, dst, n16, lane);
   }
 }
 

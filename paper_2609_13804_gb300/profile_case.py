@@ -5,6 +5,7 @@ launches).  Shapes are those of the 16-image LLaVA-1.5-7B-shaped batch.
     python -m paper_2609_13804_gb300.profile_case gemm       # 1 decoder layer, T = 1791 (4 GEMMs)
     python -m paper_2609_13804_gb300.profile_case select     # selection from a given memory H
     python -m paper_2609_13804_gb300.profile_case compact    # compaction of the batch
+    python -m paper_2609_13804_gb300.profile_case compact_full  # every visual token kept (50 MB)
     python -m paper_2609_13804_gb300.profile_case attention  # 1 decoder layer, like gemm
 
 Each case runs its stage twice (the second launch set is the one to capture
@@ -68,6 +69,15 @@ def main(case: str):
         for _ in range(2):
             r = B.sp_select(selector, w.n_vis, w.n_txt, H=Hd, stop_bias=bias, k_max=w.k_max, traces=False, ws=ws)
             ws = r["_ws"]
+        torch.cuda.synchronize()
+    elif case == "compact_full":
+        # every visual token kept: the bandwidth-sized compaction (50 MB moved)
+        X = B.dev_bf16(S.bf16_round(S.normal(w.seed, "X", (sum(w.n_vis), 1024))), dev)
+        E = B.dev_bf16(S.bf16_round(S.normal(w.seed, "E", (sum(w.n_txt), 4096), 0.02)), dev)
+        idx = torch.arange(576, dtype=torch.int32, device=dev).repeat(w.B, 1).contiguous()
+        cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
+        for _ in range(2):
+            B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=cnt, k_cap=576, projector_mode=True)
         torch.cuda.synchronize()
     elif case == "compact":
         X = B.dev_bf16(S.bf16_round(S.normal(w.seed, "X", (sum(w.n_vis), 1024))), dev)

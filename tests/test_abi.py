@@ -23,7 +23,7 @@ def L():
 def declared_symbols():
     with open(os.path.join(ROOT, "include", "stepprune.h")) as f:
         src = f.read()
-    return sorted(set(re.findall(r"^SP_API [^(]*?\b(sp_[a-z_]+)\(", src, flags=re.M)))
+    return sorted(set(re.findall(r"^SP_API [^(]*?\b(sp_[a-z0-9_]+)\(", src, flags=re.M)))
 
 
 def test_header_and_binding_agree():
