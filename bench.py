@@ -392,25 +392,28 @@ def run_ours(args):
     sel_report = selection_report(B, w, selector, X, E, bias, prof["select"]["ms"] / args.steps, dev)
     comp = {}
 
-    def do_compact(idx, count, kc):
-        comp["o"] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
-                                 projector_mode=True)
+    def do_compact(idx, count, kc, reuse=False):
+        prev = comp.get(kc) if reuse else None
+        comp["o"] = comp[kc] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
+                                            projector_mode=True, out=prev)
 
-    def kernel_ms(fn, kind, reps=5):
-        # device time of the launches of one kind (events around each launch on
-        # its stream): a spin kernel ahead of them keeps the GPU busy while the
-        # host enqueues the calls, so no launch waits on the host inside a pair
-        # of events
+    def kernel_ms(fn, reps=5):
+        # device time per call of a one-launch call: a spin kernel ahead of the
+        # calls keeps the GPU busy while the host enqueues them, so they run
+        # back to back between one pair of events (no host gap, no per-launch
+        # events inside)
         fn()
         torch.cuda.synchronize()
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda._sleep(4_000_000)
-        B.sp_profile_begin(reps * 16)
+        a.record()
         for _ in range(reps):
             fn()
+        b_.record()
         torch.cuda.synchronize()
-        return B.sp_profile_end()[kind]["ms"] / reps
+        return a.elapsed_time(b_) / reps
 
-    compact_ms = kernel_ms(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap), "compact")
+    compact_ms = kernel_ms(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap, reuse=True))
     comp_bytes = 2.0 * (K_sum * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
 
     def prefill_stage(idx, count, kc):
@@ -427,7 +430,7 @@ def run_ours(args):
     full_cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
     full_ms = timed(lambda: prefill_stage(full_idx, full_cnt, 576), reps=3)
     # compaction at a bandwidth-sized case: every visual token kept (the full prefix)
-    full_compact_ms = kernel_ms(lambda: do_compact(full_idx, full_cnt, 576), "compact")
+    full_compact_ms = kernel_ms(lambda: do_compact(full_idx, full_cnt, 576, reuse=True))
     full_T = sum(w.n_vis) + sum(w.n_txt)
     full_comp_bytes = 2.0 * (sum(w.n_vis) * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + full_T)
 

@@ -333,7 +333,10 @@ def sp_select(sel: Selector, n_vis, n_txt, *, stop_bias, X=None, E_text=None, H=
 
 # ----------------------------------------------------------------------------- compaction
 
-def sp_compact(n_vis, n_txt, *, X, text, idx, count, k_cap, projector_mode=False, stream=None) -> Dict:
+def sp_compact(n_vis, n_txt, *, X, text, idx, count, k_cap, projector_mode=False, stream=None,
+               out: Optional[Dict] = None) -> Dict:
+    """Compaction into new zero-filled outputs, or into `out` (a dict a
+    previous call returned for the same sizes) without touching it first."""
     torch = _torch()
     dev = X.device
     keep: List = []
@@ -342,6 +345,17 @@ def sp_compact(n_vis, n_txt, *, X, text, idx, count, k_cap, projector_mode=False
     W_vis, W_txt = X.shape[1], text.shape[1]
     T_cap = sp_packed_cap(n_vis, n_txt, k_cap)
     rows_cap = sum(min(n, k_cap) for n in n_vis)
+    if out is not None:
+        if out["T_cap"] != T_cap or (projector_mode and out.get("rows_cap") != rows_cap):
+            raise ValueError("sp_compact: `out` was made for other sizes")
+        ci = sp_compact_in(len(n_vis), C.cast(nv, IP), C.cast(nt, IP), ptr(X), int(W_vis), ptr(text), int(W_txt),
+                           ptr(idx), int(k_cap), ptr(count))
+        co = sp_compact_out(ptr(out["packed"]), ptr(out["cu_seqlens"]), ptr(out["pos"]),
+                            ptr(out.get("vis_packed") if projector_mode else None),
+                            ptr(out.get("vis_row_map") if projector_mode else None),
+                            ptr(out.get("vis_cu") if projector_mode else None), ptr(out["err"]))
+        _check(lib().sp_compact(C.byref(ci), C.byref(co), _stream(stream)), "sp_compact")
+        return out
     out = {"packed": torch.zeros((max(T_cap, 1), W_txt), dtype=torch.bfloat16, device=dev),
            "cu_seqlens": torch.zeros(len(n_vis) + 1, dtype=torch.int32, device=dev),
            "pos": torch.full((max(T_cap, 1),), -1, dtype=torch.int32, device=dev),
