@@ -28,6 +28,9 @@ Parity status of each function:
   restore / compact                     pinned (hand-worked golden fixture; invariants)
   rope                                  pinned (rotation closed form, relative-position property)
   round_bf16                            pinned (torch's float32 -> bfloat16 conversion)
+  decode_step, cache_from_prefill       pinned (equals the prefill over the extended
+                                        sequences at the new positions, with and
+                                        without bf16 storage)
   projector, prefill_layer, prefill     pinned through their parts plus special cases
                                         (acc='fp32' variant: pinned against acc='fp64'
                                         to fp32 precision)
@@ -431,7 +434,7 @@ def _mm(a, b, acc: str) -> np.ndarray:
 
 
 def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = None,
-                  acc: str = "fp64") -> np.ndarray:
+                  acc: str = "fp64", kv_out: Optional[list] = None) -> np.ndarray:
     """One pre-norm decoder layer of the frozen LM over the packed sequences:
     h += Wo Attn(RoPE(Wq x), RoPE(Wk x), Wv x), x = RMSNorm(h);
     h += Wdown (SiLU(Wg x') * Wu x'), x' = RMSNorm(h).  Attention is causal and
@@ -440,7 +443,9 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
     inputs, rotated q / k, v, attention output, SwiGLU output) are rounded to
     bf16 where they are stored.  acc='fp32' computes the four projections in
     fp32 instead of fp64 (used only to size how far two exact bf16 prefills
-    drift apart through rounding decisions alone)."""
+    drift apart through rounding decisions alone).  kv_out, if given, receives
+    this layer's (rotated keys, values) of every packed row: the cache a
+    generation step reads."""
     h = _f(h).copy()
     Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
     x = _store(rms_norm(h, m.rms_eps, L.get("attn_norm")), store)
@@ -448,6 +453,8 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
     q = _store(rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta), store)
     k = _store(rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta), store)
     v = _store(qkv[:, (Hq + Hkv) * dh:], store)
+    if kv_out is not None:
+        kv_out.append((k.copy(), v.copy()))
     o = np.zeros((h.shape[0], Hq * dh), dtype=F64)
     for b in range(len(cu) - 1):
         s, e = int(cu[b]), int(cu[b + 1])
@@ -467,11 +474,57 @@ def final_norm(h, m, gain=None) -> np.ndarray:
 
 
 def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None, store: Optional[str] = None,
-            acc: str = "fp64") -> np.ndarray:
+            acc: str = "fp64", kv_out: Optional[list] = None) -> np.ndarray:
     h = _f(x)
     for L in layers:
-        h = prefill_layer(h, L, m, cu, pos, store, acc)
+        h = prefill_layer(h, L, m, cu, pos, store, acc, kv_out)
     return final_norm(h, m, final_gain)
+
+
+def cache_from_prefill(kv_rows, cu) -> List[List[tuple]]:
+    """Per layer, per sequence (K, V): the prefill's packed cache rows split at
+    the sequence boundaries."""
+    out = []
+    for k, v in kv_rows:
+        out.append([(k[int(cu[b]):int(cu[b + 1])].copy(), v[int(cu[b]):int(cu[b + 1])].copy())
+                    for b in range(len(cu) - 1)])
+    return out
+
+
+def decode_step(x_new, layers: Sequence[Dict], m, cache: List[List[tuple]], final_gain=None,
+                store: Optional[str] = None):
+    """One generation step after the prefill over the pruned prefix (the decode
+    the paper's per-token and end-to-end latencies include): sequence b's new
+    token x_new[b] takes position len_b = cache rows of b and attends to the
+    cached rotated keys / values 0..len_b-1 and to itself.  The layer is the
+    prefill's layer applied to that one row.  Returns the normalised hidden
+    state of the new tokens [B, d] and the cache with their keys / values
+    appended."""
+    h = _f(x_new).copy()
+    B = h.shape[0]
+    Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
+    lens = [cache[0][b][0].shape[0] for b in range(B)]
+    pos = np.array(lens, dtype=F64)
+    new_cache = []
+    for L, layer_cache in zip(layers, cache):
+        x = _store(rms_norm(h, m.rms_eps, L.get("attn_norm")), store)
+        qkv = x @ _f(L["Wqkv"]).T
+        q = _store(rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta), store)
+        k = _store(rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta), store)
+        v = _store(qkv[:, (Hq + Hkv) * dh:], store)
+        o = np.zeros((B, Hq * dh), dtype=F64)
+        grown = []
+        for b in range(B):
+            Kb = np.concatenate([layer_cache[b][0], k[b:b + 1]])
+            Vb = np.concatenate([layer_cache[b][1], v[b:b + 1]])
+            grown.append((Kb, Vb))
+            o[b] = attention(q[b:b + 1], Kb, Vb, Hq, Hkv, causal=False)[0]
+        new_cache.append(grown)
+        h = h + _store(o, store) @ _f(L["Wo"]).T
+        x2 = _store(rms_norm(h, m.rms_eps, L.get("mlp_norm")), store)
+        gu = x2 @ _f(L["Wgu"]).T
+        h = h + _store(silu(gu[:, :F]) * gu[:, F:], store) @ _f(L["Wdown"]).T
+    return final_norm(h, m, final_gain), new_cache
 
 
 # ----------------------------------------------------------------------------

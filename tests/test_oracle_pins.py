@@ -380,6 +380,37 @@ def test_prefill_fp32_accumulation_variant_is_fp32_close():
     assert np.abs(b - a).max() > 0.0
 
 
+@pytest.mark.parametrize("store", [None, "bf16"])
+def test_decode_step_equals_prefill_over_the_extended_sequences(store):
+    """A generation step over the prefill's cache gives, for every sequence, the
+    hidden state the prefill itself computes at that position when the new
+    token is appended to the packed sequence (and the cache grows by exactly
+    that position's keys / values)."""
+    w, L = _tiny_lm(17, hq=4, hkv=2)
+    m = w.model
+    layers = [L, _tiny_lm(18, hq=4, hkv=2)[1]]
+    lens = [5, 1, 9]
+    x = S.normal(17, "x", (sum(lens), m.d)).astype(np.float64)
+    x_new = S.normal(17, "x_new", (len(lens), m.d)).astype(np.float64)
+    cu = np.r_[0, np.cumsum(lens)]
+    pos = np.concatenate([np.arange(n) for n in lens])
+    kv = []
+    O.prefill(x, layers, m, cu, pos, store=store, kv_out=kv)
+    cache = O.cache_from_prefill(kv, cu)
+    got, grown = O.decode_step(x_new, layers, m, cache, store=store)
+    # the same tokens as one longer prefill
+    ext = np.concatenate([np.concatenate([x[cu[b]:cu[b + 1]], x_new[b:b + 1]]) for b in range(len(lens))])
+    cu2 = np.r_[0, np.cumsum([n + 1 for n in lens])]
+    pos2 = np.concatenate([np.arange(n + 1) for n in lens])
+    kv2 = []
+    full = O.prefill(ext, layers, m, cu2, pos2, store=store, kv_out=kv2)
+    np.testing.assert_allclose(got, full[cu2[1:] - 1], rtol=0, atol=1e-10)
+    for l in range(len(layers)):
+        for b in range(len(lens)):
+            np.testing.assert_allclose(grown[l][b][0], kv2[l][0][cu2[b]:cu2[b + 1]], atol=1e-12)
+            np.testing.assert_allclose(grown[l][b][1], kv2[l][1][cu2[b]:cu2[b + 1]], atol=1e-12)
+
+
 def test_projector_forms():
     w = S.tiny_workload(15, [4], [2], D=12, d=20)
     head = S.make_model_head(w)
