@@ -434,6 +434,37 @@ def run_ours(args):
     full_T = sum(w.n_vis) + sum(w.n_txt)
     full_comp_bytes = 2.0 * (sum(w.n_vis) * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + full_T)
 
+    # ---- generation over the pruned prefix vs the full prefix (one token per
+    #      sequence per step, 32 layers; the cache contents do not change the
+    #      work, so a zeroed cache with the prefix lengths stands in)
+    def decode_ms(lens, steps=5):
+        S_cap = max(lens) + steps + 8
+        kv = B.kv_cache(model, w.B, S_cap)
+        x_new = (torch.randn((w.B, m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+        lens_d = torch.tensor(lens, dtype=torch.int32, device=dev)
+        o = B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap)
+        ws_d = o["_ws"]
+        lens_d.copy_(torch.tensor(lens, dtype=torch.int32, device=dev))
+        torch.cuda.synchronize()
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws_d)
+        b_.record()
+        torch.cuda.synchronize()
+        del kv
+        return a.elapsed_time(b_) / steps
+
+    pruned_lens = np.diff(pipe.cu.cpu().numpy()).astype(int).tolist()
+    full_lens = [n + t for n, t in zip(w.n_vis, w.n_txt)]
+    dec_pruned_ms = decode_ms(pruned_lens)
+    dec_full_ms = decode_ms(full_lens)
+    qkv_w = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
+    weight_bytes = 2.0 * m.n_layers * (m.d * qkv_w + m.n_heads * m.head_dim * m.d + 3 * m.d * m.ffn)
+
+    def cache_bytes(lens):
+        return 2.0 * 2 * m.n_layers * m.n_kv_heads * m.head_dim * sum(n + 1 for n in lens)
+
     # ---- end to end from host buffers (copies inside the timed region)
     Xh = X.cpu().pin_memory()
     Eh = E.cpu().pin_memory()
@@ -493,6 +524,12 @@ def run_ours(args):
             "speedup_with_selection": full_ms / (pruned_ms + select_ms),
             "token_ratio": (sum(w.n_vis) + sum(w.n_txt)) / T,
             "kept_counts": counts.tolist(),
+            "decode": {"ms_per_step_pruned_prefix": dec_pruned_ms, "ms_per_step_full_prefix": dec_full_ms,
+                       "speedup": dec_full_ms / dec_pruned_ms, "sequences": w.B,
+                       "hbm_gbs_pruned": (weight_bytes + cache_bytes(pruned_lens)) / (dec_pruned_ms * 1e-3) / 1e9,
+                       "hbm_frac_pruned": (weight_bytes + cache_bytes(pruned_lens)) / (dec_pruned_ms * 1e-3) / 1e9
+                       / pk["hbm_gbs"],
+                       "bytes_note": "weights of the 32 layers + the cache rows read, per step"},
         }
         print(json.dumps(line), flush=True)
     if dist:

@@ -343,7 +343,12 @@ SP_API sp_status sp_project(const sp_model* m, const sp_project_io* io, void* wo
  * (cu_seqlens), rotary positions pos, pre-RMSNorm Llama-style layers, and the
  * final RMSNorm.  hidden rows t < T = cu_seqlens[B] are written; rows >= T are
  * untouched.  residual (optional) receives the last residual stream (fp32,
- * before the final norm).
+ * before the final norm).  kv (optional) receives the key / value cache the
+ * generation that follows reads (sp_decode): per layer l, sequence b and
+ * position p = pos[row] the rotated key at
+ *   kv + (((l * 2 + 0) * B + b) * kv_S_cap + p) * (n_kv_heads * head_dim)
+ * and the value at the same offset with 1 in place of 0 (bf16).  Positions
+ * must be < kv_S_cap (else SP_DEVERR_INDEX).
  */
 typedef struct {
   int B;
@@ -355,11 +360,40 @@ typedef struct {
   float* hidden;            /* DEVICE [T_cap, d] fp32 output */
   float* residual;          /* DEVICE [T_cap, d] fp32 or NULL */
   int* err;
+  void* kv;                 /* DEVICE [n_layers][2][B][kv_S_cap][n_kv_heads * head_dim] bf16, or NULL */
+  int kv_S_cap;             /* positions per sequence in kv */
 } sp_prefill_io;
 
 SP_API size_t sp_prefill_workspace(const sp_model* m, int T_cap, int max_seqlen_cap);
 SP_API sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* workspace,
                      size_t workspace_bytes, sp_stream stream);
+
+/*
+ * One generation step after the prefill (the decode whose per-token latency
+ * the pruned prefix lowers): every sequence b appends one token x[b] at
+ * position lens[b], which attends to the cached keys / values 0..lens[b]-1
+ * (written by sp_prefill's kv, or by earlier steps) and to itself; the layers
+ * are the prefill's, applied to that one row.  The step writes the new
+ * token's rotated key / value into the cache at position lens[b], the final
+ * RMSNorm of its last residual into hidden[b], and then increments lens[b]
+ * (on the device, so steps chain without a host round trip).
+ * Errors: a position >= kv_S_cap sets SP_DEVERR_INDEX (nothing is written
+ * for that sequence's cache row).
+ */
+typedef struct {
+  int B;                    /* sequences, as in the prefill that wrote kv */
+  const void* x;            /* DEVICE [B, d] bf16: the new token of each sequence */
+  int* lens;                /* DEVICE [B] int32: cached positions per sequence; incremented */
+  void* kv;                 /* DEVICE cache, layout of sp_prefill_io.kv */
+  int kv_S_cap;             /* positions per sequence in kv */
+  int max_len_cap;          /* bound on lens[b] + 1 (sizes the attention launch) */
+  float* hidden;            /* DEVICE [B, d] fp32 output */
+  int* err;
+} sp_decode_io;
+
+SP_API size_t sp_decode_workspace(const sp_model* m, int B);
+SP_API sp_status sp_decode(const sp_model* m, const sp_decode_io* io, void* workspace, size_t workspace_bytes,
+                           sp_stream stream);
 
 /* ------------------------------------------------------------------------ */
 /* The whole path: select -> compact -> project -> prefill.                  */

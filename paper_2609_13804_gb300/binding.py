@@ -33,7 +33,7 @@ EXPORTS = [
     "sp_model_destroy", "sp_project_workspace", "sp_project", "sp_prefill_workspace", "sp_prefill",
     "sp_pipeline_workspace", "sp_pipeline", "sp_pipeline_host_workspace", "sp_pipeline_host",
     "sp_profile_begin", "sp_profile_end", "sp_select_noalloc", "sp_probe_smem_gbs", "sp_probe_l2_gbs",
-    "sp_probe_select_floor",
+    "sp_probe_select_floor", "sp_decode_workspace", "sp_decode",
 ]
 SP_SELECT_NOALLOC_SCRATCH_BYTES = 64 << 20
 
@@ -97,7 +97,12 @@ class sp_project_io(C.Structure):
 
 class sp_prefill_io(C.Structure):
     _fields_ = [("B", C.c_int), ("T_cap", C.c_int), ("max_seqlen_cap", C.c_int), ("x", P), ("cu_seqlens", P),
-                ("pos", P), ("hidden", P), ("residual", P), ("err", P)]
+                ("pos", P), ("hidden", P), ("residual", P), ("err", P), ("kv", P), ("kv_S_cap", C.c_int)]
+
+
+class sp_decode_io(C.Structure):
+    _fields_ = [("B", C.c_int), ("x", P), ("lens", P), ("kv", P), ("kv_S_cap", C.c_int), ("max_len_cap", C.c_int),
+                ("hidden", P), ("err", P)]
 
 
 class sp_pipeline_io(C.Structure):
@@ -138,6 +143,8 @@ def lib():
         "sp_project": (C.c_int, [P, C.POINTER(sp_project_io), P, C.c_size_t, P]),
         "sp_prefill_workspace": (C.c_size_t, [P, C.c_int, C.c_int]),
         "sp_prefill": (C.c_int, [P, C.POINTER(sp_prefill_io), P, C.c_size_t, P]),
+        "sp_decode_workspace": (C.c_size_t, [P, C.c_int]),
+        "sp_decode": (C.c_int, [P, C.POINTER(sp_decode_io), P, C.c_size_t, P]),
         "sp_pipeline_workspace": (C.c_size_t, [P, P, C.POINTER(sp_pipeline_io)]),
         "sp_pipeline": (C.c_int, [P, P, C.POINTER(sp_pipeline_io), P, C.c_size_t, P]),
         "sp_pipeline_host_workspace": (C.c_size_t, [P, P, C.POINTER(sp_pipeline_host_io)]),
@@ -434,18 +441,42 @@ def sp_project(model: Model, *, vis_packed, vis_row_map, vis_cu, packed, rows_ca
     return err
 
 
+def kv_cache(model: Model, B: int, S_cap: int, device=None):
+    """A zeroed key / value cache [n_layers, 2, B, S_cap, n_kv_heads * head_dim] bf16."""
+    torch = _torch()
+    m = model.shape
+    return torch.zeros((m.n_layers, 2, B, S_cap, m.n_kv_heads * m.head_dim), dtype=torch.bfloat16,
+                       device=device or model.device)
+
+
 def sp_prefill(model: Model, *, x, cu_seqlens, pos, B, T_cap, max_seqlen_cap, residual=None, stream=None,
-               ws=None, hidden=None):
+               ws=None, hidden=None, kv=None):
     torch = _torch()
     dev = x.device
     if hidden is None:
         hidden = torch.zeros((max(T_cap, 1), model.shape.d), dtype=torch.float32, device=dev)
     err = torch.zeros(1, dtype=torch.int32, device=dev)
     io = sp_prefill_io(int(B), int(T_cap), int(max_seqlen_cap), ptr(x), ptr(cu_seqlens), ptr(pos), ptr(hidden),
-                       ptr(residual), ptr(err))
+                       ptr(residual), ptr(err), ptr(kv), int(kv.shape[3]) if kv is not None else 0)
     if ws is None:
         ws = workspace(lib().sp_prefill_workspace(model.handle, int(T_cap), int(max_seqlen_cap)), dev)
     _check(lib().sp_prefill(model.handle, C.byref(io), ptr(ws), ws.numel(), _stream(stream)), "sp_prefill")
+    return {"hidden": hidden, "err": err, "_ws": ws}
+
+
+def sp_decode(model: Model, *, x, lens, kv, max_len_cap, stream=None, ws=None, hidden=None) -> Dict:
+    """One generation step: x [B, d] bf16 new tokens, lens [B] int32 cached lengths
+    (incremented on the device), kv the cache of kv_cache() / sp_prefill."""
+    torch = _torch()
+    dev = x.device
+    B = int(x.shape[0])
+    if hidden is None:
+        hidden = torch.zeros((B, model.shape.d), dtype=torch.float32, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    io = sp_decode_io(B, ptr(x), ptr(lens), ptr(kv), int(kv.shape[3]), int(max_len_cap), ptr(hidden), ptr(err))
+    if ws is None:
+        ws = workspace(lib().sp_decode_workspace(model.handle, B), dev)
+    _check(lib().sp_decode(model.handle, C.byref(io), ptr(ws), ws.numel(), _stream(stream)), "sp_decode")
     return {"hidden": hidden, "err": err, "_ws": ws}
 
 

@@ -817,8 +817,10 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
     return fail(SP_ERR_SHAPE, "sp_prefill: bad B / T_cap / max_seqlen_cap");
   if (io->max_seqlen_cap > c.max_pos) return fail(SP_ERR_SHAPE, "sp_prefill: max_seqlen_cap %d > max_pos %d", io->max_seqlen_cap, c.max_pos);
   if (!io->x || !io->cu_seqlens || !io->pos || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_prefill: x, cu_seqlens, pos, hidden required");
-  if (!al16(io->x) || !al16(io->hidden) || (io->residual && !al16(io->residual)))
+  if (!al16(io->x) || !al16(io->hidden) || (io->residual && !al16(io->residual)) || (io->kv && !al16(io->kv)))
     return fail(SP_ERR_ALIGN, "sp_prefill: buffers must be 16-byte aligned");
+  if (io->kv && io->kv_S_cap < io->max_seqlen_cap)
+    return fail(SP_ERR_SHAPE, "sp_prefill: kv_S_cap %d < max_seqlen_cap %d", io->kv_S_cap, io->max_seqlen_cap);
   if (io->T_cap == 0) return SP_OK;
   Carve cv(ws);
   PrefillParts p;
@@ -852,6 +854,11 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
     SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->qkv[l], qkvw, eq, io->err, st, &gs), "qkv");
+    if (io->kv) {
+      void* kv_l = static_cast<uint16_t*>(io->kv) + (size_t)l * 2 * io->B * io->kv_S_cap * c.n_kv_heads * c.head_dim;
+      SP_CUDA(kv_store(p.qkv, io->cu_seqlens, io->pos, io->B, T_cap, c.n_heads, c.n_kv_heads, c.head_dim, kv_l,
+                       io->kv_S_cap, io->err, st), "kv cache");
+    }
     SP_CUDA(attention_varlen(p.qkv, p.ob, io->cu_seqlens, io->B, io->max_seqlen_cap, T_cap, c.n_heads, c.n_kv_heads,
                              c.head_dim, true, io->err, st), "attention");
     GemmEpi er;
@@ -874,6 +881,91 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
 
 sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* ws, size_t ws_bytes, sp_stream stream) {
   return prefill_impl(m, io, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ decode
+
+static size_t decode_ws(const sp_model* m, int B, Carve& cv, PrefillParts* p) {
+  // the prefill's buffers at B rows (the single-CTA GEMM path: no stream-K scratch)
+  const sp_model_cfg& c = m->cfg;
+  const size_t R = (size_t)std::max(B, 1);
+  PrefillParts q;
+  q.h32 = cv.take<float>(R * c.d);
+  q.xb = cv.take<uint16_t>(R * c.d);
+  q.qkv = cv.take<uint16_t>(R * (c.n_heads + 2 * c.n_kv_heads) * c.head_dim);
+  q.ob = cv.take<uint16_t>(R * c.n_heads * c.head_dim);
+  q.act = cv.take<uint16_t>(R * c.ffn);
+  q.gsk = nullptr;
+  if (p) *p = q;
+  return cv.off;
+}
+
+size_t sp_decode_workspace(const sp_model* m, int B) {
+  if (!m || B < 1) return 0;
+  Carve cv(nullptr);
+  return decode_ws(m, B, cv, nullptr) + 256;
+}
+
+static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws, size_t ws_bytes, cudaStream_t st) {
+  if (!m || !io) return fail(SP_ERR_INVALID_ARG, "sp_decode: NULL argument");
+  const sp_model_cfg& c = m->cfg;
+  if (io->B < 1 || io->B > SP_MAX_BATCH || io->kv_S_cap < 1 || io->max_len_cap < 1 || io->max_len_cap > io->kv_S_cap)
+    return fail(SP_ERR_SHAPE, "sp_decode: bad B / kv_S_cap / max_len_cap");
+  if (io->max_len_cap > c.max_pos) return fail(SP_ERR_SHAPE, "sp_decode: max_len_cap %d > max_pos %d", io->max_len_cap, c.max_pos);
+  if (!io->x || !io->lens || !io->kv || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_decode: x, lens, kv, hidden required");
+  if (!al16(io->x) || !al16(io->kv) || !al16(io->hidden)) return fail(SP_ERR_ALIGN, "sp_decode: buffers must be 16-byte aligned");
+  Carve cv(ws);
+  PrefillParts p;
+  const size_t need = decode_ws(m, io->B, cv, &p) + 256;
+  if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_decode: workspace %zu < %zu bytes", ws_bytes, need);
+  if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_decode: workspace must be 16-byte aligned");
+  const int B = io->B;
+  const int dq = c.n_heads * c.head_dim, qkvw = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim;
+  const size_t layer_elems = (size_t)2 * B * io->kv_S_cap * c.n_kv_heads * c.head_dim;
+  std::string msg;
+  CUtensorMap tX, tO, tA;
+  if (!encode_tmap_bf16(&tX, p.xb, B, c.d, 128, &msg) || !encode_tmap_bf16(&tO, p.ob, B, dq, 128, &msg) ||
+      !encode_tmap_bf16(&tA, p.act, B, c.ffn, 128, &msg))
+    return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  SP_CUDA(bf16_to_f32(io->x, p.h32, B, nullptr, c.d, st), "embed");
+  for (int l = 0; l < c.n_layers; ++l) {
+    void* kv_l = static_cast<uint16_t*>(io->kv) + (size_t)l * layer_elems;
+    SP_CUDA(rmsnorm_f32_to_bf16(p.h32, m->w.attn_norm[l], p.xb, B, nullptr, c.d, c.rms_eps, st), "attn norm");
+    GemmEpi eq;
+    eq.kind = EPI_BF16_ROPE;
+    eq.out = p.qkv;
+    eq.ldo = qkvw;
+    eq.rope = m->rope;
+    eq.pos = io->lens;  // the new token's position is the cached length
+    eq.max_pos = c.max_pos;
+    eq.head_dim = c.head_dim;
+    eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
+    SP_CUDA(gemm_bf16(tX, B, nullptr, m->qkv[l], qkvw, eq, io->err, st), "qkv");
+    SP_CUDA(kv_append(p.qkv, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim, kv_l, io->kv_S_cap, io->err, st),
+            "kv append");
+    SP_CUDA(decode_attention(p.qkv, kv_l, io->kv_S_cap, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim, p.ob, st),
+            "decode attention");
+    GemmEpi er;
+    er.kind = EPI_F32_ACC;
+    er.out = p.h32;
+    er.ldo = c.d;
+    SP_CUDA(gemm_bf16(tO, B, nullptr, m->o[l], c.d, er, io->err, st), "o");
+    SP_CUDA(rmsnorm_f32_to_bf16(p.h32, m->w.mlp_norm[l], p.xb, B, nullptr, c.d, c.rms_eps, st), "mlp norm");
+    GemmEpi eg;
+    eg.kind = EPI_SWIGLU_BF16;
+    eg.out = p.act;
+    eg.ldo = c.ffn;
+    eg.up_off = c.ffn;
+    SP_CUDA(gemm_bf16(tX, B, nullptr, m->gu[l], 2 * c.ffn, eg, io->err, st), "gate/up");
+    SP_CUDA(gemm_bf16(tA, B, nullptr, m->down[l], c.d, er, io->err, st), "down");
+  }
+  SP_CUDA(rmsnorm_f32_to_f32(p.h32, m->w.final_norm, io->hidden, B, nullptr, c.d, c.rms_eps, st), "final norm");
+  SP_CUDA(lens_increment(io->lens, B, io->kv_S_cap, st), "lens");
+  return SP_OK;
+}
+
+sp_status sp_decode(const sp_model* m, const sp_decode_io* io, void* ws, size_t ws_bytes, sp_stream stream) {
+  return decode_impl(m, io, ws, ws_bytes, (cudaStream_t)stream);
 }
 
 // ------------------------------------------------------------------ pipeline

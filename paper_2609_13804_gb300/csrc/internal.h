@@ -132,6 +132,16 @@ cudaError_t gather_memory(const BatchDesc& bd, const float* R, const float* H, c
                           const float* s_start, float* Mall, int D, cudaStream_t st);
 cudaError_t write_enc_cu(const BatchDesc& bd, int* cu, cudaStream_t st);
 
+// ------------------------------------------------------------- key / value cache and decode
+// Cache layout: layer block [2][B][S_cap][Hkv * dh] bf16 (K then V).
+cudaError_t kv_store(const void* qkv, const int* cu, const int* pos, int B, int T_cap, int Hq, int Hkv, int dh,
+                     void* kv_l, int S_cap, int* err, cudaStream_t st);
+cudaError_t kv_append(const void* qkv, const int* lens, int B, int Hq, int Hkv, int dh, void* kv_l, int S_cap,
+                      int* err, cudaStream_t st);
+cudaError_t decode_attention(const void* qkv, const void* kv_l, int S_cap, const int* lens, int B, int Hq, int Hkv,
+                             int dh, void* out, cudaStream_t st);
+cudaError_t lens_increment(int* lens, int B, int S_cap, cudaStream_t st);
+
 // ------------------------------------------------------------- attention
 // Varlen attention over packed qkv [rows_cap, (Hq + 2 Hkv) dh] bf16 -> out [T, Hq dh] bf16
 // (rows of sequence b from cu_seqlens[b]; rows_cap bounds the buffer for TMA).

@@ -425,3 +425,74 @@ def test_prefill_llava15_b16_32layers_sampled(B):
         r = PT.hidden_close(g2, np.concatenate([ref[b] for b in picks]), f"layer {l}")
         print(f"layer-local parity, layer {l}: max-abs %.3e mean-rel %.3e" % r)
         one.close()
+
+
+# ------------------------------------------------------------------ generation over the pruned prefix
+
+def _decode_case(B, w, lens, n_layers, steps=2):
+    """The prefill's cache (parity of every cached row against the oracle's),
+    then generation steps: the first fed the oracle's own cache (stage-local),
+    the next chained on the GPU's cache."""
+    m = w.model
+    layers = [S.make_layer_weights(w, l, norm_affine=True) for l in range(n_layers)]
+    head = S.make_model_head(w, norm_affine=True)
+    model = B.Model(m, layers, head, DEV, max_pos=max(lens) + steps + 8)
+    T = int(sum(lens))
+    nb = len(lens)
+    x = S.bf16_round(S.normal(w.seed, "packed", (T, m.d), 0.5))
+    cu, pos = PT.lens_cu_pos(lens)
+    S_cap = max(lens) + steps
+    kv_rows = []
+    O.prefill(x, layers, m, cu, pos, head["final_norm"], store="bf16", kv_out=kv_rows)
+    cache = O.cache_from_prefill(kv_rows, cu)
+
+    # prefill writes the cache
+    kv = B.kv_cache(model, nb, S_cap)
+    out = B.sp_prefill(model, x=B.dev_bf16(x, DEV), cu_seqlens=torch.from_numpy(cu.astype(np.int32)).to(DEV),
+                       pos=torch.from_numpy(pos.astype(np.int32)).to(DEV), B=nb, T_cap=T, max_seqlen_cap=max(lens),
+                       kv=kv)
+    torch.cuda.synchronize()
+    assert int(out["err"].item()) == 0
+    got_kv = kv.float().cpu().numpy()
+    for l in range(n_layers):
+        for b in range(nb):
+            for j, name in ((0, "K"), (1, "V")):
+                ref = cache[l][b][j]
+                g = got_kv[l, j, b, :lens[b]]
+                err = np.abs(g - ref).max() / max(np.abs(ref).max(), 1e-6)
+                # layer 0 is one GEMM from the same bf16 input: one rounding flip at most
+                bound = 1e-2 if l == 0 else 5e-2
+                assert err <= bound, (l, b, name, err)
+            assert np.all(got_kv[l, :, b, lens[b]:] == 0)  # positions past the prefix untouched
+
+    # step 1 from the oracle's cache, then chained steps on the GPU cache
+    kv_o = B.kv_cache(model, nb, S_cap)
+    host = kv_o.float().cpu().numpy()
+    for l in range(n_layers):
+        for b in range(nb):
+            host[l, 0, b, :lens[b]] = cache[l][b][0]
+            host[l, 1, b, :lens[b]] = cache[l][b][1]
+    kv_o.copy_(torch.from_numpy(host).to(torch.bfloat16))
+    lens_d = torch.tensor(lens, dtype=torch.int32, device=DEV)
+    ws = None
+    for step in range(steps):
+        x_new = S.bf16_round(S.normal(w.seed, f"new{step}", (nb, m.d), 0.5))
+        o = B.sp_decode(model, x=B.dev_bf16(x_new, DEV), lens=lens_d, kv=kv_o, max_len_cap=S_cap, ws=ws)
+        ws = o["_ws"]
+        torch.cuda.synchronize()
+        assert int(o["err"].item()) == 0
+        ref, cache = O.decode_step(x_new, layers, m, cache, head["final_norm"], store="bf16")
+        r = PT.hidden_close(np_(o["hidden"]), ref, f"{w.name} decode step {step}")
+        print(f"decode step {step}: max-abs %.3e mean-rel %.3e" % r)
+        np.testing.assert_array_equal(lens_d.cpu().numpy(), np.array(lens) + step + 1)
+    model.close()
+
+
+def test_decode_tiny_gqa_ragged(B):
+    w = S.tiny_workload(62, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=2)
+    _decode_case(B, w, [5, 130, 1, 64], 2)
+
+
+def test_decode_llama7b_dims_1layer(B):
+    w = S.llava15_7b_b16()
+    _decode_case(B, w, [112, 240, 64, 17], 1)
