@@ -44,6 +44,16 @@ def test_struct_sizes_match_header_layout():
     assert C.sizeof(b.sp_select_out) == 8 + 8 + 8 * 8
 
 
+def test_prefill_and_decode_io_layout():
+    assert C.sizeof(b.sp_prefill_io) == 4 * 3 + 4 + 8 * 6 + 8 + 4 + 4
+    assert C.sizeof(b.sp_decode_io) == 4 + 4 + 8 * 3 + 4 * 2 + 8 * 2
+
+
+def test_decode_argument_checks_fail_before_any_launch(L):
+    assert L.sp_decode(None, None, None, 0, None) == 1
+    assert L.sp_decode_workspace(None, 4) == 0
+
+
 def test_host_arithmetic(L):
     assert b.sp_num_episodes([576] * 16, 0) == 16
     assert b.sp_num_episodes([2880] * 8, 576) == 40
