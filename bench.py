@@ -536,6 +536,93 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+# Sec. 4 scaling table (LLaVA-1.5-7B rows): input tokens, retained tokens,
+# full prefill ms, pruned-path ms, selector ms, on the paper's GPU (context only)
+PAPER_SCALING = {
+    320: (32, 29.34, 30.00, 9.65), 640: (64, 53.24, 37.14, 16.15), 960: (96, 70.86, 37.75, 20.45),
+    1280: (128, 116.89, 40.91, 24.25), 1600: (160, 142.93, 46.13, 28.85), 1920: (192, 189.83, 52.28, 34.41),
+    2240: (224, 236.55, 57.73, 39.14)}
+
+
+def run_sweep(args):
+    """Scaling with the visual-prefix length at 10% retention: one image of N
+    visual + 48 text tokens on the LLaVA-1.5-7B-shaped model, N = 320..2240.
+    Per N: the full-prefix prefill (projector on N rows + 32 layers over N + 48),
+    the pruned path (selector incl. its encoder, compaction, projector on the
+    kept rows, 32 layers over K + 48) and the selector alone, each the mean of
+    `--steps` calls after `--warmup`."""
+    import torch
+    from paper_2609_13804_gb300 import binding as B
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = S.llava15_7b_b16()
+    s, m = w.selector, w.model
+    selector = B.Selector(s, S.make_selector_weights(w), dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(w.seed)
+    layers = [device_layer_weights(m, l, dev, gen, torch) for l in range(m.n_layers)]
+    head = {"final_norm": torch.ones(m.d, device=dev),
+            "proj_W1": (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16),
+            "proj_W2": (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)}
+    model = B.Model(m, layers, head, dev, max_pos=4096)
+    L = 48
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize()
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(args.steps):
+            fn()
+        b_.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b_) / args.steps
+
+    rows = []
+    for N in sorted(PAPER_SCALING):
+        K = N // 10
+        X = (torch.randn((N, s.D), device=dev, generator=gen)).to(torch.bfloat16)
+        E = (torch.randn((L, m.d), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+        bias = torch.full((1,), -1e30, dtype=torch.float32, device=dev)  # STOP never wins: exactly K kept
+        pipe = B.Pipeline(selector, model, [N], [L], group_size=0, g=1, k_max=K)
+        pruned_ms = timed(lambda: pipe(X, E, bias))
+        sel_ws = {}
+
+        def select():
+            r = B.sp_select(selector, [N], [L], X=X, E_text=E, stop_bias=bias, group_size=0, g=1, k_max=K,
+                            traces=False, ws=sel_ws.get("ws"))
+            sel_ws["ws"] = r["_ws"]
+        selector_ms = timed(select)
+        full_idx = torch.arange(N, dtype=torch.int32, device=dev).reshape(1, N)
+        full_cnt = torch.full((1,), N, dtype=torch.int32, device=dev)
+        st = {}
+
+        def full_prefill():
+            o = B.sp_compact([N], [L], X=X, text=E, idx=full_idx, count=full_cnt, k_cap=N, projector_mode=True,
+                             out=st.get("c"))
+            st["c"] = o
+            B.sp_project(model, vis_packed=o["vis_packed"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
+                         packed=o["packed"], rows_cap=o["rows_cap"], B=1)
+            r = B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=1, T_cap=o["T_cap"],
+                             max_seqlen_cap=N + L, ws=st.get("ws"), hidden=st.get("h"))
+            st["ws"], st["h"] = r["_ws"], r["hidden"]
+        full_ms = timed(full_prefill)
+        kept = int(pipe.count[0].item())
+        pk, pf, pp, ps = PAPER_SCALING[N]
+        rows.append({"input_tokens": N, "retained": kept, "full_prefill_ms": full_ms, "stepprune_prefill_ms": pruned_ms,
+                     "selector_ms": selector_ms, "speedup": full_ms / pruned_ms,
+                     "selector_share": selector_ms / pruned_ms,
+                     "paper": {"retained": pk, "full_prefill_ms": pf, "stepprune_prefill_ms": pp, "selector_ms": ps,
+                               "speedup": pf / pp, "selector_share": ps / pp}})
+        del pipe
+    line = {"sweep": "visual-prefix length at 10% retention", "config": {"workload": "llava15-7b dims, 1 image",
+            "text_tokens": L, "layers": m.n_layers}, "steps": args.steps, "warmup": args.warmup,
+            "paper_gpu": "RTX PRO 6000 Blackwell (the paper's; context only)", "rows": rows}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -545,10 +632,14 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--launch-list", action="store_true",
                     help="set up, warm up and run one more step only (for an ncu launch list)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="scaling with the visual-prefix length at 10%% retention (one JSON line, no headline)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.sweep:
+        run_sweep(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

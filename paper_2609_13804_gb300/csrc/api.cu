@@ -721,12 +721,21 @@ void sp_model_destroy(sp_model* m) {
 
 // ------------------------------------------------------------------ projector
 
-static size_t project_ws(const sp_model* m, int rows_cap, Carve& cv, void** tmp, void** gsk = nullptr) {
+static size_t project_ws(const sp_model* m, int rows_cap, Carve& cv, void** tmp, void** gsk = nullptr,
+                         float** splitk = nullptr, size_t* splitk_floats = nullptr) {
   void* t = nullptr;
   if (m->cfg.proj_kind == SP_PROJ_MLP2_GELU) t = cv.take<uint16_t>((size_t)std::max(rows_cap, 1) * m->cfg.proj_hidden);
   void* g = m->cfg.proj_kind != SP_PROJ_NONE ? cv.take<char>(gemm_scratch_bytes()) : nullptr;
+  float* sk = nullptr;
+  size_t skf = 0;
+  if (m->cfg.proj_kind != SP_PROJ_NONE && rows_cap <= 128) {
+    skf = gemm_splitk_floats(std::max(m->cfg.proj_hidden, m->cfg.d));
+    sk = cv.take<float>(skf);
+  }
   if (tmp) *tmp = t;
   if (gsk) *gsk = g;
+  if (splitk) *splitk = sk;
+  if (splitk_floats) *splitk_floats = skf;
   return cv.off;
 }
 
@@ -748,12 +757,18 @@ static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* 
   Carve cv(ws);
   void* tmp = nullptr;
   void* gsk = nullptr;
-  const size_t need = project_ws(m, io->rows_cap, cv, &tmp, &gsk) + 256;
+  float* spk = nullptr;
+  size_t spkf = 0;
+  const size_t need = project_ws(m, io->rows_cap, cv, &tmp, &gsk, &spk, &spkf) + 256;
   const bool have_ws = ws && ws_bytes >= need;
   if (c.proj_kind == SP_PROJ_MLP2_GELU && !have_ws)
     return fail(SP_ERR_WORKSPACE, "sp_project: workspace %zu < %zu bytes", ws_bytes, need);
   // a linear projector runs without a workspace too (whole GEMM tiles only)
-  const GemmScratch gs = gemm_scratch_at(have_ws ? gsk : nullptr);
+  GemmScratch gs = gemm_scratch_at(have_ws ? gsk : nullptr);
+  if (have_ws) {
+    gs.splitk = spk;
+    gs.splitk_floats = spkf;
+  }
   SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   std::string msg;
   CUtensorMap tV;
@@ -788,7 +803,13 @@ sp_status sp_project(const sp_model* m, const sp_project_io* io, void* ws, size_
 struct PrefillParts {
   float* h32;
   void *xb, *qkv, *ob, *act, *gsk;
+  float* splitk = nullptr;  // small-M split-K planes (T_cap <= 128)
+  size_t splitk_floats = 0;
 };
+
+static size_t model_max_n(const sp_model_cfg& c) {
+  return (size_t)std::max(std::max((c.n_heads + 2 * c.n_kv_heads) * c.head_dim, c.d), 2 * c.ffn);
+}
 
 static size_t prefill_ws(const sp_model* m, int T_cap, bool own_residual, Carve& cv, PrefillParts* p) {
   const sp_model_cfg& c = m->cfg;
@@ -800,6 +821,10 @@ static size_t prefill_ws(const sp_model* m, int T_cap, bool own_residual, Carve&
   q.ob = cv.take<uint16_t>(T * c.n_heads * c.head_dim);
   q.act = cv.take<uint16_t>(T * c.ffn);
   q.gsk = cv.take<char>(gemm_scratch_bytes());
+  if (T_cap <= 128) {
+    q.splitk_floats = gemm_splitk_floats((int)model_max_n(c));
+    q.splitk = cv.take<float>(q.splitk_floats);
+  }
   if (p) *p = q;
   return cv.off;
 }
@@ -836,7 +861,9 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
   if (!encode_tmap_bf16(&tX, p.xb, T_cap, c.d, 128, &msg) || !encode_tmap_bf16(&tO, p.ob, T_cap, dq, 128, &msg) ||
       !encode_tmap_bf16(&tA, p.act, T_cap, c.ffn, 128, &msg))
     return fail(SP_ERR_CUDA, "%s", msg.c_str());
-  const GemmScratch gs = gemm_scratch_at(p.gsk);
+  GemmScratch gs = gemm_scratch_at(p.gsk);
+  gs.splitk = p.splitk;
+  gs.splitk_floats = p.splitk_floats;
   SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   SP_CUDA(bf16_to_f32(io->x, h32, T_cap, T_dev, c.d, st), "embed");
   // the attention's last key tile reads up to 63 rows past the packed length
@@ -896,6 +923,10 @@ static size_t decode_ws(const sp_model* m, int B, Carve& cv, PrefillParts* p) {
   q.ob = cv.take<uint16_t>(R * c.n_heads * c.head_dim);
   q.act = cv.take<uint16_t>(R * c.ffn);
   q.gsk = nullptr;
+  if (B <= 128) {
+    q.splitk_floats = gemm_splitk_floats((int)model_max_n(c));
+    q.splitk = cv.take<float>(q.splitk_floats);
+  }
   if (p) *p = q;
   return cv.off;
 }
@@ -927,6 +958,9 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
   if (!encode_tmap_bf16(&tX, p.xb, B, c.d, 128, &msg) || !encode_tmap_bf16(&tO, p.ob, B, dq, 128, &msg) ||
       !encode_tmap_bf16(&tA, p.act, B, c.ffn, 128, &msg))
     return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  GemmScratch gs;
+  gs.splitk = p.splitk;
+  gs.splitk_floats = p.splitk_floats;
   SP_CUDA(bf16_to_f32(io->x, p.h32, B, nullptr, c.d, st), "embed");
   for (int l = 0; l < c.n_layers; ++l) {
     void* kv_l = static_cast<uint16_t*>(io->kv) + (size_t)l * layer_elems;
@@ -940,7 +974,7 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
     eq.max_pos = c.max_pos;
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
-    SP_CUDA(gemm_bf16(tX, B, nullptr, m->qkv[l], qkvw, eq, io->err, st), "qkv");
+    SP_CUDA(gemm_bf16(tX, B, nullptr, m->qkv[l], qkvw, eq, io->err, st, &gs), "qkv");
     SP_CUDA(kv_append(p.qkv, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim, kv_l, io->kv_S_cap, io->err, st),
             "kv append");
     SP_CUDA(decode_attention(p.qkv, kv_l, io->kv_S_cap, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim, p.ob, st),
@@ -949,15 +983,15 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
     er.kind = EPI_F32_ACC;
     er.out = p.h32;
     er.ldo = c.d;
-    SP_CUDA(gemm_bf16(tO, B, nullptr, m->o[l], c.d, er, io->err, st), "o");
+    SP_CUDA(gemm_bf16(tO, B, nullptr, m->o[l], c.d, er, io->err, st, &gs), "o");
     SP_CUDA(rmsnorm_f32_to_bf16(p.h32, m->w.mlp_norm[l], p.xb, B, nullptr, c.d, c.rms_eps, st), "mlp norm");
     GemmEpi eg;
     eg.kind = EPI_SWIGLU_BF16;
     eg.out = p.act;
     eg.ldo = c.ffn;
     eg.up_off = c.ffn;
-    SP_CUDA(gemm_bf16(tX, B, nullptr, m->gu[l], 2 * c.ffn, eg, io->err, st), "gate/up");
-    SP_CUDA(gemm_bf16(tA, B, nullptr, m->down[l], c.d, er, io->err, st), "down");
+    SP_CUDA(gemm_bf16(tX, B, nullptr, m->gu[l], 2 * c.ffn, eg, io->err, st, &gs), "gate/up");
+    SP_CUDA(gemm_bf16(tA, B, nullptr, m->down[l], c.d, er, io->err, st, &gs), "down");
   }
   SP_CUDA(rmsnorm_f32_to_f32(p.h32, m->w.final_norm, io->hidden, B, nullptr, c.d, c.rms_eps, st), "final norm");
   SP_CUDA(lens_increment(io->lens, B, io->kv_S_cap, st), "lens");

@@ -57,6 +57,9 @@ struct KArgs {
   int* err;
   int a_seg;       // A k-segment remap (GemmASplit); 0: none
   uint32_t a_map;
+  int ksplit;      // single-CTA kernel: K ranges per tile (> 1: fp32 partials to tmO at row s * m_pad)
+  int m_pad;       // rows per partial plane (multiple of 32)
+  int swiglu_b;    // load B as SwiGLU gate | up halves whatever the epilogue
   float* sk_part;  // pair kernel: stream-K partial tiles [pairs][256][BN] (NULL: whole tiles only)
   int* sk_flags;   // pair kernel: [pairs][8] ready flags, zero between launches
 };
@@ -457,8 +460,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   if (M < 0) M = 0;
   const int num_m = (M + BM - 1) / BM;
   const int num_n = args.N_acc / BN;
-  const int total = num_m * num_n;
+  const int ks = args.ksplit > 1 ? args.ksplit : 1;
+  const int total = num_m * num_n * ks;  // work items: (tile, K range)
   const int KB = args.K / BK;
+  const bool swb = (EPI == EPI_SWIGLU_BF16) || args.swiglu_b;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -491,17 +496,19 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       int issued = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-        const int mb = t % num_m, nb = t / num_m;
+        const int tile = t / ks, sp = t - tile * ks;
+        const int mb = tile % num_m, nb = tile / num_m;
         const int m0 = mb * BM;
         int b0, b1;
-        if (EPI == EPI_SWIGLU_BF16) {
+        if (swb) {
           b0 = nb * (BN / 2);
           b1 = args.e.up_off + nb * (BN / 2);
         } else {
           b0 = nb * BN;
           b1 = nb * BN + BN / 2;
         }
-        for (int kb = 0; kb < KB; ++kb) {
+        const int kb0 = sp * KB / ks, kb1 = (sp + 1) * KB / ks;
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, err)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[s], C::A_BYTES + C::B_BYTES);
           tma_load_2d(sA + s * C::A_BYTES, &tmA, &full[s], a_col(args, kb * BK), m0);
@@ -537,7 +544,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (!mbar_wait(&tempty[acc], aph ^ 1u, err)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        for (int kb = 0; kb < KB; ++kb) {
+        const int sp = t % ks;
+        const int kb0 = sp * KB / ks, kb1 = (sp + 1) * KB / ks;
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full[s], ph, err)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
@@ -545,7 +554,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             umma_bf16(d_tmem, umma_desc_sw128(a0 + k * 32), umma_desc_sw128(b0 + k * 32), IDESC,
-                      (kb | k) != 0 ? 1u : 0u);
+                      (kb != kb0 || k != 0) ? 1u : 0u);
           }
           umma_commit(&empty[s]);
           if (++s == C::STAGES) { s = 0; ph ^= 1u; }
@@ -569,14 +578,21 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const uint32_t aph = (it >> 1) & 1;
       if (!mbar_wait_warp(&tfull[acc], aph, err)) break;
       tc_fence_after();
-      const int mb = t % num_m, nb = t / num_m;
+      const int tile = t / ks, sp = t - tile * ks;
+      const int mb = tile % num_m, nb = tile / num_m;
       const int row0 = mb * BM + quad * 32;
       const int row = row0 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + acc * BN;
-      if (EPI == EPI_SCATTER_BF16)
+      if (ks > 1) {
+        // a K range: its raw fp32 partial into plane sp (rows past m_pad belong to the next plane)
+        if (EPI == EPI_F32 && row0 < args.m_pad)
+          epilogue_tma<BN, EPI>(args.e, &tmO, taddr, sp * args.m_pad + row0, lane, row < M, nb, boxes, nbox, Fix(),
+                                err);
+      } else if (EPI == EPI_SCATTER_BF16) {
         epilogue_tile<BN, EPI>(args.e, taddr, row, row < M, nb, err, Fix());
-      else
+      } else {
         epilogue_tma<BN, EPI>(args.e, &tmO, taddr, row0, lane, row < M, nb, boxes, nbox, Fix(), err);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -996,6 +1012,68 @@ cudaError_t dispatch_pair(const CUtensorMap& A, const CUtensorMap& B, const CUte
   }
 }
 
+// Sum of the K-range partials of a split GEMM (planes of m_pad x N_acc fp32)
+// and the epilogue the unsplit GEMM would have fused (one block row per row).
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restrict__ part, int ks, int m_pad,
+                                                            int M_cap, const int* __restrict__ M_dev, int N_acc,
+                                                            int BN, const GemmEpi e, int* err) {
+  int M = M_cap;
+  if (M_dev) M = min(M, __ldg(M_dev));
+  const int row = blockIdx.y;
+  if (row >= M) return;
+  const size_t plane = (size_t)m_pad * N_acc;
+  const float* pr = part + (size_t)row * N_acc;
+  auto sum = [&](int c) {
+    float v = 0.f;
+    for (int s = 0; s < ks; ++s) v += __ldcg(pr + s * plane + c);
+    return v;
+  };
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e.kind == EPI_SWIGLU_BF16) {
+    if (c >= N_acc / 2) return;
+    const int nb = c / (BN / 2), j = c - nb * (BN / 2);
+    const float g = sum(nb * BN + j), u = sum(nb * BN + BN / 2 + j);
+    reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)row * e.ldo + c] = __float2bfloat16_rn(silu(g) * u);
+    return;
+  }
+  if (c >= N_acc) return;
+  if (e.kind == EPI_BF16_ROPE) {
+    const int dh = e.head_dim, half = dh >> 1;
+    const int hb = (c / dh) * dh, i = c - hb;
+    __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(e.out) + (size_t)row * e.ldo;
+    if (hb < e.rope_cols) {
+      if (i >= half) return;  // the pair's first element writes both
+      const int p = __ldg(e.pos + row);
+      const bool pos_ok = p >= 0 && p < e.max_pos;
+      if (!pos_ok) set_error(err, SP_DEVERR_INDEX);
+      const float2 r = __ldg(e.rope + (size_t)(pos_ok ? p : 0) * half + i);
+      const float a = sum(c), b = sum(c + half);
+      o[c] = __float2bfloat16_rn(a * r.x - b * r.y);
+      o[c + half] = __float2bfloat16_rn(b * r.x + a * r.y);
+    } else {
+      o[c] = __float2bfloat16_rn(sum(c));
+    }
+    return;
+  }
+  const float v = sum(c);
+  if (e.kind == EPI_F32) {
+    reinterpret_cast<float*>(e.out)[(size_t)row * e.ldo + c] = v;
+  } else if (e.kind == EPI_F32_ACC) {
+    reinterpret_cast<float*>(e.out)[(size_t)row * e.ldo + c] += v;
+  } else if (e.kind == EPI_GELU_BF16) {
+    reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)row * e.ldo + c] = __float2bfloat16_rn(gelu_erf(v));
+  } else if (e.kind == EPI_SCATTER_BF16) {
+    const int orow = __ldg(e.row_map + row);
+    if (orow < 0) {
+      set_error(err, SP_DEVERR_INDEX);
+      return;
+    }
+    reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)orow * e.ldo + c] = __float2bfloat16_rn(v);
+  } else {
+    reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)row * e.ldo + c] = __float2bfloat16_rn(v);
+  }
+}
+
 template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& O, const KArgs& a, int grid,
                        cudaStream_t st) {
@@ -1069,6 +1147,13 @@ GemmScratch gemm_scratch_at(void* p) {
   return g;
 }
 
+size_t gemm_splitk_floats(int max_n_acc) {
+  // split count <= ceil(SMs / tiles) with tiles >= N / 256 and <= 16: planes x N_acc
+  // stays below (SMs + N / 128) x 256 per row, 128 rows per plane at most
+  const size_t per_row = ((size_t)device_sm_count() + (size_t)max_n_acc / 128 + 1) * 256;
+  return per_row * BM;
+}
+
 cudaError_t gemm_scratch_clear(const GemmScratch& g, cudaStream_t st) {
   if (!g.flags) return cudaSuccess;
   return cudaMemsetAsync(g.flags, 0, (size_t)g.slots * 8 * sizeof(int), st);
@@ -1108,6 +1193,9 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
   a.sk_flags = nullptr;
   a.a_seg = 0;
   a.a_map = 0;
+  a.ksplit = 1;
+  a.m_pad = 0;
+  a.swiglu_b = 0;
   if (as && as->seg > 0) {
     if (as->seg % BK != 0 || B.K > 8 * as->seg) return cudaErrorInvalidValue;
     a.a_seg = as->seg;
@@ -1139,12 +1227,44 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
     prof_end_launch(st, SP_K_GEMM, 2.0 * (double)M_cap * (double)N_acc * (double)B.K, 0.0);
     return r;
   }
-  const int tiles = mt * (N_acc / (use256 ? 256 : 128));
+  const int bn = use256 ? 256 : 128;
+  const int tiles = mt * (N_acc / bn);
+  double flops = 2.0 * (double)M_cap * (double)N_acc * (double)B.K;
+  // Small M (<= 128 rows: generation steps, one short sequence): too few tiles
+  // to stream the weights with every SM; split K into ranges over the idle SMs,
+  // fp32 partials to the caller's scratch, then one reduce + epilogue pass.
+  const int KB = B.K / BK;
+  if (sk && sk->splitk && M_cap <= BM && tiles < sms && KB >= 8) {
+    int kspl = std::min(std::min((sms + tiles - 1) / tiles, KB / 4), 16);
+    const int m_pad = (M_cap + 31) / 32 * 32;
+    while (kspl > 1 && (size_t)kspl * m_pad * N_acc > sk->splitk_floats) --kspl;
+    if (kspl > 1) {
+      CUtensorMap tmP;
+      if (!encode_tmap_2d(&tmP, sk->splitk, true, (uint64_t)kspl * m_pad, (uint64_t)N_acc, 32, 32, nullptr))
+        return cudaErrorInvalidValue;
+      KArgs ap = a;
+      ap.e.kind = EPI_F32;
+      ap.ksplit = kspl;
+      ap.m_pad = m_pad;
+      ap.swiglu_b = e.kind == EPI_SWIGLU_BF16 ? 1 : 0;
+      const int grid = std::max(1, std::min(tiles * kspl, sms));
+      prof_begin_launch(st);
+      r = use256 ? launch_one<256, EPI_F32>(A, B.map256, tmP, ap, grid, st)
+                 : launch_one<128, EPI_F32>(A, B.map128, tmP, ap, grid, st);
+      prof_end_launch(st, SP_K_GEMM, flops, 0.0);
+      if (r != cudaSuccess) return r;
+      const int cols = e.kind == EPI_SWIGLU_BF16 ? N_acc / 2 : N_acc;
+      dim3 rg((cols + 255) / 256, M_cap);
+      prof_begin_launch(st);
+      splitk_reduce_kernel<<<rg, 256, 0, st>>>(sk->splitk, kspl, m_pad, M_cap, M_dev, N_acc, bn, e, err);
+      prof_end_launch(st, SP_K_MISC, 0.0, 4.0 * kspl * (double)m_pad * N_acc);
+      return cudaGetLastError();
+    }
+  }
   const int grid = std::max(1, std::min(tiles, sms));
   prof_begin_launch(st);
   r = use256 ? dispatch<256>(A, B.map256, tmO, a, grid, st)
              : dispatch<128>(A, B.map128, tmO, a, grid, st);
-  double flops = 2.0 * (double)M_cap * (double)N_acc * (double)B.K;
   prof_end_launch(st, SP_K_GEMM, flops, 0.0);
   return r;
 }

@@ -84,8 +84,12 @@ struct GemmScratch {
   float* part = nullptr;
   int* flags = nullptr;
   int slots = 0;
+  float* splitk = nullptr;   // small-M split-K partial planes (NULL: no split)
+  size_t splitk_floats = 0;
 };
 size_t gemm_scratch_bytes();
+// fp32 scratch that lets small-M GEMMs (M <= 128) of width <= max_n_acc split K.
+size_t gemm_splitk_floats(int max_n_acc);
 GemmScratch gemm_scratch_at(void* p);  // p: gemm_scratch_bytes() bytes, 256-byte aligned (or NULL)
 cudaError_t gemm_scratch_clear(const GemmScratch& g, cudaStream_t st);
 

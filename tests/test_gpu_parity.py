@@ -189,15 +189,15 @@ def test_compaction_bit_exact(B, projector_mode):
 
 # ------------------------------------------------------------------ projector
 
-@pytest.mark.parametrize("kind", ["linear", "mlp2"])
-def test_projector_scatter(B, kind):
+@pytest.mark.parametrize("kind,rows", [("linear", 300), ("mlp2", 300), ("mlp2", 100)])
+def test_projector_scatter(B, kind, rows):
+    # rows <= 128: the split-K path (GELU and row-scatter epilogues in the reduce pass)
     w = S.tiny_workload(51, [300], [1], D=1024, d=1024, n_heads=8, n_kv_heads=8, head_dim=128, ffn=1024,
                         n_layers=1, proj_kind=kind)
     w.model.proj_hidden = 2048
     head = S.make_model_head(w)
     L = S.make_layer_weights(w, 0)
     model = B.Model(w.model, [L], head, DEV, max_pos=512)
-    rows = 300
     vis = S.bf16_round(S.normal(51, "vis", (rows, 1024)))
     T = rows + 50
     rmap = np.random.default_rng(51).permutation(T)[:rows].astype(np.int32)
@@ -298,6 +298,14 @@ def test_prefill_llama7b_dims_2layers(B):
     bound = max(PT.HID_MAX_ABS, 1.5 * drift)
     print(f"2-layer prefill: max-abs {mx:.3e} (bound {bound:.3e}, fp32/fp64 drift {drift:.3e}) mean-rel {mr:.3e}")
     assert mx <= bound and mr <= PT.HID_MEAN_REL, (mx, bound, mr)
+
+
+def test_prefill_short_batch_split_k(B):
+    # T <= 128 packed rows: the GEMMs split K over the SMs and reduce the partials
+    # with the fused epilogues (RoPE, residual, SwiGLU) in a second pass
+    _prefill_case(B, S.llava15_7b_b16(), [40, 7, 60], 1)
+    w = S.tiny_workload(63, [1], [1], D=128, d=128, n_heads=2, n_kv_heads=1, head_dim=64, ffn=256, n_layers=2)
+    _prefill_case(B, w, [5, 30, 1, 64], 2)
 
 
 def test_prefill_qwen_gqa_dims(B):
