@@ -79,6 +79,14 @@ def test_select_tiny_stop_extremes(B):
     assert int(gpu["count"][2]) == 3 and int(gpu["rounds"][2]) == 4  # exhausted: only STOP left
 
 
+def test_select_max_batch(B):
+    # SP_MAX_BATCH images of 1..40 candidates, text 0..3, cap 8
+    n_vis = [int(v) for v in S.uniform_int(24, "nv", 1, 41, 256)]
+    n_txt = [int(v) for v in S.uniform_int(24, "nt", 0, 4, 256)]
+    w = S.tiny_workload(24, n_vis, n_txt, D=128, h=128, k_max=8)
+    _run_select_case(B, w, scale=4.0)
+
+
 def test_select_groups_g5(B):
     w = S.tiny_workload(23, [300, 77, 128], [2, 2, 2], D=128, h=128, k_max=20, group_size=128, g=5)
     _run_select_case(B, w, scale=4.0)
@@ -185,6 +193,34 @@ def test_compaction_bit_exact(B, projector_mode):
         text_rows = np.setdiff1d(np.arange(T), rmap)
         np.testing.assert_array_equal(got[text_rows], packed[text_rows])
         np.testing.assert_array_equal(np_(out["vis_cu"]), np.concatenate([[0], np.cumsum(count)]))
+
+
+def test_compaction_max_batch(B):
+    # SP_MAX_BATCH images: kept counts 0..n (none, some, all), text 0..3 rows
+    rng = np.random.default_rng(42)
+    n_vis = [int(v) for v in rng.integers(1, 33, 256)]
+    n_txt = [int(v) for v in rng.integers(0, 4, 256)]
+    W = 256
+    X = S.bf16_round(S.normal(42, "X", (sum(n_vis), W)))
+    text = S.bf16_round(S.normal(42, "T", (max(sum(n_txt), 1), W)))
+    k_cap = 32
+    idx_list = []
+    for b, n in enumerate(n_vis):
+        k = [0, n, int(rng.integers(0, n + 1))][b % 3]
+        idx_list.append(np.sort(rng.choice(n, k, replace=False)))
+    idx = np.full((256, k_cap), -1, np.int32)
+    for b, l in enumerate(idx_list):
+        idx[b, :len(l)] = l
+    count = np.array([len(l) for l in idx_list], np.int32)
+    out = B.sp_compact(n_vis, n_txt, X=B.dev_bf16(X, DEV), text=B.dev_bf16(text, DEV), idx=torch.from_numpy(idx).to(DEV),
+                       count=torch.from_numpy(count).to(DEV), k_cap=k_cap)
+    torch.cuda.synchronize()
+    assert int(out["err"].item()) == 0
+    packed, cu, pos = O.compact(X, n_vis, idx_list, text[:sum(n_txt)], n_txt)
+    T = int(cu[-1])
+    np.testing.assert_array_equal(np_(out["cu_seqlens"]), cu)
+    np.testing.assert_array_equal(np_(out["pos"])[:T], pos)
+    np.testing.assert_array_equal(np_(out["packed"])[:T], packed)
 
 
 # ------------------------------------------------------------------ projector
@@ -306,6 +342,12 @@ def test_prefill_short_batch_split_k(B):
     _prefill_case(B, S.llava15_7b_b16(), [40, 7, 60], 1)
     w = S.tiny_workload(63, [1], [1], D=128, d=128, n_heads=2, n_kv_heads=1, head_dim=64, ffn=256, n_layers=2)
     _prefill_case(B, w, [5, 30, 1, 64], 2)
+
+
+def test_prefill_empty_sequences(B):
+    # zero-length sequences between non-empty ones (repeated cu_seqlens entries)
+    w = S.tiny_workload(64, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=2)
+    _prefill_case(B, w, [0, 5, 0, 130, 1, 0], 2)
 
 
 def test_prefill_qwen_gqa_dims(B):
@@ -465,6 +507,8 @@ def _decode_case(B, w, lens, n_layers, steps=2):
     for l in range(n_layers):
         for b in range(nb):
             for j, name in ((0, "K"), (1, "V")):
+                if lens[b] == 0:
+                    continue
                 ref = cache[l][b][j]
                 g = got_kv[l, j, b, :lens[b]]
                 err = np.abs(g - ref).max() / max(np.abs(ref).max(), 1e-6)
@@ -499,6 +543,12 @@ def _decode_case(B, w, lens, n_layers, steps=2):
 def test_decode_tiny_gqa_ragged(B):
     w = S.tiny_workload(62, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=2)
     _decode_case(B, w, [5, 130, 1, 64], 2)
+
+
+def test_decode_empty_prefix(B):
+    # a sequence with no cached positions attends to its new token alone
+    w = S.tiny_workload(65, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=2)
+    _decode_case(B, w, [0, 7, 1], 2)
 
 
 def test_decode_llama7b_dims_1layer(B):
