@@ -281,6 +281,16 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   const size_t trace = (size_t)e * (k_max + 1);
   __syncthreads();
 
+  // the per-element vectors of a round (residual, merged attention output,
+  // LN2 output) are held DPT consecutive elements per thread
+  auto el = [&](int d) { return tid * DPT + d; };
+  // LN2 affine parameters, read once for the whole episode
+  float g2[DPT], b2[DPT];
+#pragma unroll
+  for (int d = 0; d < DPT; ++d) {
+    g2[d] = (a.ln2_g && el(d) < h) ? __ldg(a.ln2_g + el(d)) : 1.f;
+    b2[d] = (a.ln2_b && el(d) < h) ? __ldg(a.ln2_b + el(d)) : 0.f;
+  }
   // query / residual rows of the last history position, loaded one round ahead
   float zr[DPT];
   float4 q[HV];
@@ -289,7 +299,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     const float* zrow = a.Z + (size_t)row * a.ldz;
     shift = __ldg(zrow);  // common shift of the LN moments (any value near the data)
 #pragma unroll
-    for (int d = 0; d < DPT; ++d) zr[d] = (tid + d * NT < h) ? __ldg(zrow + tid + d * NT) : 0.f;
+    for (int d = 0; d < DPT; ++d) zr[d] = (el(d) < h) ? __ldg(zrow + el(d)) : 0.f;
     const float4* qrow = reinterpret_cast<const float4*>(a.QS + (size_t)row * a.ldqs);
 #pragma unroll
     for (int k = 0; k < HV; ++k) q[k] = __ldg(qrow + lane + 32 * k);
@@ -381,14 +391,25 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
 #pragma unroll
       for (int w = 0; w < NW; ++w) cw[w] = __shfl_sync(0xffffffffu, cwl, w);
       float* slot = all_o + ((size_t)buf * C + rank) * h;
+      if (el(0) < h) {
+        float acc[DPT];
 #pragma unroll
-      for (int d = 0; d < DPT; ++d) {
-        const int i = tid + d * NT;
-        if (i >= h) continue;
-        float acc = 0.f;
+        for (int d = 0; d < DPT; ++d) {
+          acc[d] = 0.f;
 #pragma unroll
-        for (int w = 0; w < NW; ++w) acc += cw[w] * wpart_o[w * h + i];
-        for (int r = 0; r < C; ++r) cluster.map_shared_rank(slot, r)[i] = acc;
+          for (int w = 0; w < NW; ++w) acc[d] += cw[w] * wpart_o[w * h + el(d)];
+        }
+        // one vector store per peer (DPT consecutive elements)
+        for (int r = 0; r < C; ++r) {
+          float* dst = cluster.map_shared_rank(slot, r) + el(0);
+          if (DPT == 4)
+            *reinterpret_cast<float4*>(dst) = make_float4(acc[0], acc[DPT > 1 ? 1 : 0], acc[DPT > 2 ? 2 : 0],
+                                                          acc[DPT > 3 ? 3 : 0]);
+          else if (DPT == 2)
+            *reinterpret_cast<float2*>(dst) = make_float2(acc[0], acc[DPT > 1 ? 1 : 0]);
+          else
+            dst[0] = acc[0];
+        }
       }
       if (tid < C) {
         float* ml = cluster.map_shared_rank(all_ml + ((size_t)buf * C + rank) * 2, tid);
@@ -414,7 +435,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     float mom[2] = {0.f, 0.f};
 #pragma unroll
     for (int d = 0; d < DPT; ++d) {
-      const int i = tid + d * NT;
+      const int i = el(d);
       uv[d] = 0.f;
       if (i >= h) continue;
       float o = 0.f;
@@ -432,12 +453,9 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     const float rstd = rsqrtf(fmaxf(mom[1] / (float)h - m1 * m1, 0.f) + a.ln_eps);
 #pragma unroll
     for (int d = 0; d < DPT; ++d) {
-      const int i = tid + d * NT;
+      const int i = el(d);
       if (i >= h) continue;
-      float x = (uv[d] - mean) * rstd;
-      if (a.ln2_g) x *= __ldg(a.ln2_g + i);
-      if (a.ln2_b) x += __ldg(a.ln2_b + i);
-      xp_s[i] = x;
+      xp_s[i] = (uv[d] - mean) * rstd * g2[d] + b2[d];
     }
     __syncthreads();
 
