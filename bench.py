@@ -39,7 +39,7 @@ UNIT = "ms/batch"
 # (one 7B-dims layer at T = 1,792 rows, the benchmark's packed length within
 # 0.5%).  The figure belongs to the kernel sources with this digest; once they
 # change it is reported as null until a new capture replaces it.
-GEMM_TRAFFIC = {"bytes_per_launch": 165.6e6, "sources_sha256_16": "13a67d04a743e2a2"}
+GEMM_TRAFFIC = {"bytes_per_launch": 163.6e6, "sources_sha256_16": "8820f8545daa90b6"}
 GEMM_SOURCES = ("paper_2609_13804_gb300/csrc/gemm_tc.cu", "paper_2609_13804_gb300/csrc/common.cuh")
 
 
@@ -199,8 +199,10 @@ def cpu_oracle_sample(w, n_images=1, n_layers=1):
 def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
     """The selection kernel against its on-chip roofline: algorithmic bytes per
     round per episode are the folded pointer keys of its candidates, (N_e + 1) h
-    fp32 from shared memory, plus the history rows the round's attention reads,
-    2 t h fp32 from L2 (t = history length); the kernel's time is the longest
+    fp32 from shared memory, the history rows the round's attention reads, 2 t h
+    fp32 (t = history length) from the TMEM cache, and from L2 the rows that
+    enter the round (the last position's query and residual rows, the key and
+    value rows of the positions appended); the kernel's time is the longest
     episode's rounds.  Peaks and the synchronisation floor come from the
     library's probes."""
     r = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bias, group_size=w.group_size, g=w.g,
@@ -210,14 +212,18 @@ def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
     rounds = r["rounds"].cpu().numpy().astype(int)
     h = w.selector.h
     eps = w.episodes()
-    smem_b = l2_b = 0.0
+    n_max = max(n for (_, _, n) in eps)
+    C = 8 if (n_max + 7) // 8 + 1 <= 128 else 16
+    cached = C * 256 // (h // 128)  # history positions the TMEM cache of an episode holds
+    smem_b = tmem_b = l2_b = 0.0
     for (_, _, n_e), R in zip(eps, rounds):
         for t_round in range(int(R)):
             t = min(1 + w.g * t_round, w.k_max)
+            t_new = 1 if t_round == 0 else min(w.g, t - 1)
             smem_b += (n_e + 1) * h * 4.0
-            l2_b += 2.0 * t * h * 4.0
-    n_max = max(n for (_, _, n) in eps)
-    C = 8 if (n_max + 7) // 8 + 1 <= 128 else 16
+            in_tmem = max(0, min(t, cached) - t_new)
+            tmem_b += 2.0 * in_tmem * h * 4.0
+            l2_b += 2.0 * (t - in_tmem) * h * 4.0 + 2.0 * h * 4.0
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     smem_peak = B.probe_smem_gbs()
     l2_peak = B.probe_l2_gbs()
@@ -225,12 +231,15 @@ def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
     floor_us = B.probe_select_floor(C, h, max(r_max, 1), len(eps))
     ks = kernel_ms * 1e-3
     used = min(len(eps) * C, sms) / sms
+    onchip = smem_b + tmem_b + l2_b
     return {"kernel_ms": kernel_ms, "episodes": len(eps), "cluster_size": C, "max_rounds": r_max,
             "us_per_round": kernel_ms * 1e3 / max(r_max, 1), "floor_us_per_round": floor_us,
-            "smem_bytes": smem_b, "l2_bytes": l2_b,
-            "smem_gbs": smem_b / ks / 1e9, "l2_gbs": l2_b / ks / 1e9,
+            "smem_bytes": smem_b, "tmem_bytes": tmem_b, "l2_bytes": l2_b,
+            "smem_gbs": smem_b / ks / 1e9, "tmem_gbs": tmem_b / ks / 1e9, "l2_gbs": l2_b / ks / 1e9,
+            "onchip_gbs": onchip / ks / 1e9,
             "smem_peak_gbs": smem_peak, "smem_peak_used_sms_gbs": smem_peak * used, "l2_peak_gbs": l2_peak,
-            "smem_frac_of_used_sms": smem_b / ks / 1e9 / (smem_peak * used), "l2_frac": l2_b / ks / 1e9 / l2_peak,
+            "onchip_frac_of_smem_peak_used_sms": onchip / ks / 1e9 / (smem_peak * used),
+            "l2_frac": l2_b / ks / 1e9 / l2_peak,
             "note": "latency-bound dependent chain: compare us_per_round with floor_us_per_round"}
 
 

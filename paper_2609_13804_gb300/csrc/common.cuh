@@ -253,6 +253,100 @@ SP_DEVINL void tmem_st_32x32b_x32(uint32_t taddr, const float (&r)[32]) {
 
 SP_DEVINL void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+// TMEM <-> registers for N = 4, 8, 16 or 32 consecutive columns of this thread's
+// lane (32x32b shape); complete with tmem_ld_wait / tmem_st_wait.
+template <int N>
+SP_DEVINL void tmem_ld_cols(uint32_t taddr, float* r);
+template <>
+SP_DEVINL void tmem_ld_cols<4>(uint32_t taddr, float* r) {
+  uint32_t* u = reinterpret_cast<uint32_t*>(r);
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]) : "r"(taddr));
+}
+template <>
+SP_DEVINL void tmem_ld_cols<8>(uint32_t taddr, float* r) {
+  uint32_t* u = reinterpret_cast<uint32_t*>(r);
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]), "=r"(u[7])
+               : "r"(taddr));
+}
+template <>
+SP_DEVINL void tmem_ld_cols<16>(uint32_t taddr, float* r) {
+  uint32_t* u = reinterpret_cast<uint32_t*>(r);
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+               "%12, %13, %14, %15}, [%16];"
+               : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]), "=r"(u[7]),
+                 "=r"(u[8]), "=r"(u[9]), "=r"(u[10]), "=r"(u[11]), "=r"(u[12]), "=r"(u[13]), "=r"(u[14]),
+                 "=r"(u[15])
+               : "r"(taddr));
+}
+template <int N>
+SP_DEVINL void tmem_st_cols(uint32_t taddr, const float* r);
+template <>
+SP_DEVINL void tmem_st_cols<4>(uint32_t taddr, const float* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr),
+               "r"(__float_as_uint(r[0])), "r"(__float_as_uint(r[1])), "r"(__float_as_uint(r[2])),
+               "r"(__float_as_uint(r[3]))
+               : "memory");
+}
+template <>
+SP_DEVINL void tmem_st_cols<8>(uint32_t taddr, const float* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+               "r"(__float_as_uint(r[0])), "r"(__float_as_uint(r[1])), "r"(__float_as_uint(r[2])),
+               "r"(__float_as_uint(r[3])), "r"(__float_as_uint(r[4])), "r"(__float_as_uint(r[5])),
+               "r"(__float_as_uint(r[6])), "r"(__float_as_uint(r[7]))
+               : "memory");
+}
+template <>
+SP_DEVINL void tmem_st_cols<16>(uint32_t taddr, const float* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, "
+               "%13, %14, %15, %16};" ::"r"(taddr),
+               "r"(__float_as_uint(r[0])), "r"(__float_as_uint(r[1])), "r"(__float_as_uint(r[2])),
+               "r"(__float_as_uint(r[3])), "r"(__float_as_uint(r[4])), "r"(__float_as_uint(r[5])),
+               "r"(__float_as_uint(r[6])), "r"(__float_as_uint(r[7])), "r"(__float_as_uint(r[8])),
+               "r"(__float_as_uint(r[9])), "r"(__float_as_uint(r[10])), "r"(__float_as_uint(r[11])),
+               "r"(__float_as_uint(r[12])), "r"(__float_as_uint(r[13])), "r"(__float_as_uint(r[14])),
+               "r"(__float_as_uint(r[15]))
+               : "memory");
+}
+template <>
+SP_DEVINL void tmem_ld_cols<32>(uint32_t taddr, float* r) {
+  tmem_ld_32x32b_x32(taddr, *reinterpret_cast<float(*)[32]>(r));
+}
+template <>
+SP_DEVINL void tmem_st_cols<32>(uint32_t taddr, const float* r) {
+  tmem_st_32x32b_x32(taddr, *reinterpret_cast<const float(*)[32]>(r));
+}
+
+// An h-vector slice held as HV float4 per lane <-> 4 HV consecutive TMEM columns
+// of the lane (column 4k + c holds component c of r[k]).
+template <int HV>
+SP_DEVINL void tmem_ld_f4(uint32_t taddr, float4 (&r)[HV]) {
+  float t[4 * HV];
+  tmem_ld_cols<4 * HV>(taddr, t);
+#pragma unroll
+  for (int k = 0; k < HV; ++k) r[k] = make_float4(t[4 * k], t[4 * k + 1], t[4 * k + 2], t[4 * k + 3]);
+}
+template <int HV>
+SP_DEVINL void tmem_st_f4(uint32_t taddr, const float4 (&r)[HV]) {
+  float t[4 * HV];
+#pragma unroll
+  for (int k = 0; k < HV; ++k) {
+    t[4 * k] = r[k].x;
+    t[4 * k + 1] = r[k].y;
+    t[4 * k + 2] = r[k].z;
+    t[4 * k + 3] = r[k].w;
+  }
+  tmem_st_cols<4 * HV>(taddr, t);
+}
+// Orders later uses of registers written by tcgen05.ld after the tcgen05.wait::ld
+// that precedes this call (an empty volatile asm that reads and rewrites them).
+template <int HV>
+SP_DEVINL void reg_fence_f4(float4 (&r)[HV]) {
+#pragma unroll
+  for (int k = 0; k < HV; ++k) asm volatile("" : "+f"(r[k].x), "+f"(r[k].y), "+f"(r[k].z), "+f"(r[k].w));
+}
+
 // ---------------------------------------------------------------- CTA pairs (cta_group::2)
 
 SP_DEVINL uint32_t cluster_ctarank() {

@@ -212,7 +212,7 @@ SP_DEVINL void warp_merge_lists(const float* vin, const int* iin, int tot, int p
 // (g + 1 <= GL).  P = history positions a warp loads at once.
 template <int HV, int GL>
 __global__ void __launch_bounds__(NT, 1)
-select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in_smem) {
+select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in_smem, int tm_cols) {
   constexpr int P = (16 / HV) > 0 ? 16 / HV : 1;
   constexpr int DPT = (HV * 128) / NT > 0 ? (HV * 128) / NT : 1;  // dims per thread in the merges
   constexpr int U = 4;                                          // candidates per warp iteration
@@ -260,6 +260,19 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   float* red = misc;                                  // [0, 16)  NW x 2
   float* gtop_v = misc + 64;                          // [64, 81)
   int* gtop_i = reinterpret_cast<int*>(misc + 96);    // [96, 113)
+  uint32_t* tm_slot = reinterpret_cast<uint32_t*>(misc + 124);
+
+  // TMEM cache of the history rows this CTA attends over (tm_cols columns; 0 =
+  // off): a key / value row is read from L2 once, in the round its position
+  // joins the history, and from TMEM in every later round.  Warp w owns lanes
+  // 32 (w % 4) .. +31 of columns [(w / 4) tm_cols / 2, +tm_cols / 2): ppw
+  // positions of 8 HV columns each (key row, then value row, in the float4 lane
+  // layout of the loads below).  The host sizes tm_cols so that every CTA that
+  // can be resident on an SM gets its share of the 512 columns.
+  if (tm_cols > 0 && warp == 0) {
+    tmem_alloc(tm_slot, (uint32_t)tm_cols);
+    tmem_relinquish();
+  }
 
   // stage this CTA's slice of the folded keys and the STOP key
   const float* KT = a.KT;
@@ -279,7 +292,13 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   if (tid == 0) hist[0] = a.start_row;
   const float bias = __ldg(a.stop_bias + e);
   const size_t trace = (size_t)e * (k_max + 1);
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const int ppw = tm_cols / (16 * HV);  // cached positions per warp
+  const uint32_t tm_base = tm_cols > 0 ? *tm_slot : 0u;
+  const uint32_t tm_warp = tm_base + (((uint32_t)(warp & 3) * 32u) << 16) + (uint32_t)(warp >> 2) * (uint32_t)(tm_cols / 2);
+  int np_cached = 0;  // history positions of this CTA already in TMEM
 
   // the per-element vectors of a round (residual, merged attention output,
   // LN2 output) are held DPT consecutive elements per thread
@@ -328,18 +347,38 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     float4 o_w[HV];
 #pragma unroll
     for (int k = 0; k < HV; ++k) o_w[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k0 = warp * P; k0 < np; k0 += NW * P) {
+    for (int jj = 0, k0 = warp * P; k0 < np; ++jj, k0 += NW * P) {
       float4 kr[P][HV], vr[P][HV];
+      bool fresh[P];  // read from L2 this round, to be kept in TMEM
 #pragma unroll
       for (int pp = 0; pp < P; ++pp) {
+        const int o = jj * P + pp;  // warp-uniform, like k0 and np
+        fresh[pp] = false;
         if (k0 + pp < np) {
-          const int row = hist[rank + (k0 + pp) * C];
-          const float4* ks = reinterpret_cast<const float4*>(a.KS + (size_t)row * a.ldks);
-          const float4* vt = reinterpret_cast<const float4*>(a.VT + (size_t)row * a.ldvt);
+          if (o < ppw && k0 + pp < np_cached) {
+            const uint32_t ta = tm_warp + (uint32_t)(o * 8 * HV);
+            tmem_ld_f4<HV>(ta, kr[pp]);
+            tmem_ld_f4<HV>(ta + 4 * HV, vr[pp]);
+          } else {
+            const int row = hist[rank + (k0 + pp) * C];
+            const float4* ks = reinterpret_cast<const float4*>(a.KS + (size_t)row * a.ldks);
+            const float4* vt = reinterpret_cast<const float4*>(a.VT + (size_t)row * a.ldvt);
 #pragma unroll
-          for (int k = 0; k < HV; ++k) {
-            kr[pp][k] = __ldg(ks + lane + 32 * k);
-            vr[pp][k] = __ldg(vt + lane + 32 * k);
+            for (int k = 0; k < HV; ++k) {
+              kr[pp][k] = __ldg(ks + lane + 32 * k);
+              vr[pp][k] = __ldg(vt + lane + 32 * k);
+            }
+            fresh[pp] = o < ppw;
+          }
+        }
+      }
+      if (ppw > 0) {
+        tmem_ld_wait();
+#pragma unroll
+        for (int pp = 0; pp < P; ++pp) {
+          if (k0 + pp < np && jj * P + pp < ppw && k0 + pp < np_cached) {
+            reg_fence_f4<HV>(kr[pp]);
+            reg_fence_f4<HV>(vr[pp]);
           }
         }
       }
@@ -371,7 +410,17 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           m_w = mn;
         }
       }
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        if (fresh[pp]) {
+          const uint32_t ta = tm_warp + (uint32_t)((jj * P + pp) * 8 * HV);
+          tmem_st_f4<HV>(ta, kr[pp]);
+          tmem_st_f4<HV>(ta + 4 * HV, vr[pp]);
+        }
+      }
     }
+    if (ppw > 0) tmem_st_wait();  // this round's rows are in TMEM before the next round reads them
+    np_cached = np;
 #pragma unroll
     for (int k = 0; k < HV; ++k) reinterpret_cast<float4*>(wpart_o + warp * h)[lane + 32 * k] = o_w[k];
     if (lane == 0) {
@@ -647,7 +696,12 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     if (a.ep_count) a.ep_count[e] = nsel;
     if (a.rounds) a.rounds[e] = round;
   }
+  tc_fence_before();
   cluster.sync();  // no CTA leaves while a peer may still write into it
+  if (tm_cols > 0 && warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tm_base, (uint32_t)tm_cols);
+  }
 }
 
 // Algorithm 1 step 4: per image, the union of its episodes' selections in
@@ -745,7 +799,7 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
   }
   const int n_loc = (n_max + C - 1) / C;
   const SelSmem L = sel_layout(a.h, n_loc, a.k_max, C, keys_in_smem);
-  void (*kern)(const BatchDesc, const SelectArgs, int, int) = nullptr;
+  void (*kern)(const BatchDesc, const SelectArgs, int, int, int) = nullptr;
   const int gl = a.g + 1 <= 2 ? 2 : (a.g + 1 <= 6 ? 6 : 17);
 #define SP_SEL_CASE(HV_)                                                                                   \
   case HV_:                                                                                                \
@@ -765,6 +819,15 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
     r = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (r != cudaSuccess) return r;
   }
+  // TMEM history cache: 512 columns shared by the CTAs of this kernel that fit on
+  // one SM (so an allocation never waits on another cluster's CTA), at least
+  // one position (16 HV columns for the two rows) per warp, else off
+  int per_sm = 0;
+  r = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT, L.total);
+  if (r != cudaSuccess) return r;
+  int tm_cols = 512;
+  while (per_sm > 1 && tm_cols * per_sm > 512) tm_cols >>= 1;
+  if (per_sm < 1 || tm_cols < 32 || tm_cols < 16 * (a.h / 128)) tm_cols = 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(n_episodes * C, 1, 1);
   cfg.blockDim = dim3(NT, 1, 1);
@@ -778,7 +841,7 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   prof_begin_launch(st);
-  r = cudaLaunchKernelEx(&cfg, kern, bd, a, n_loc, keys_in_smem ? 1 : 0);
+  r = cudaLaunchKernelEx(&cfg, kern, bd, a, n_loc, keys_in_smem ? 1 : 0, tm_cols);
   prof_end_launch(st, SP_K_SELECT, 0.0, 0.0);
   return r;
 }
