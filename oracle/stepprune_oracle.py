@@ -10,6 +10,9 @@ A plain, slow, fp64 restatement of what the inference path of StepPrune
   * Algorithm 1: loop, restore to native order, gather  (Algorithm 1; Sec. 3.3, last paragraph)
   * frozen projector and LM prefill over the packed prefix (Sec. 3.3-3.4; LM dims of the
     evaluated backbones, Sec. 4.1)
+  * the training-time continuous pathway, forward only: trajectory aggregation,
+    soft count, SoftTopK polarisation, variance-preserving noise gate (Sec. 3.3,
+    Eqs. 5-9)
 
 Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline leg may import
 this module.  It shares no code with the CUDA library and imports nothing from
@@ -28,6 +31,16 @@ Parity status of each function:
   restore / compact                     pinned (hand-worked golden fixture; invariants)
   rope                                  pinned (rotation closed form, relative-position property)
   round_bf16                            pinned (torch's float32 -> bfloat16 conversion)
+  trajectory_aggregate                  pinned (closed forms of Eqs. 5-7 for a constant
+                                        STOP probability; Sum_i s_i = Kbar at beta = 1)
+  trajectory_episode                    pinned (its hard rollout equals select_episode
+                                        with g = 1; scratch = incremental; tau -> 0 gives
+                                        Kbar = hard count, s = beta^t at the chosen step)
+  soft_topk                             pinned (the two-anchor transport has the closed
+                                        form sigmoid((s_i - theta) 2 / tau) with
+                                        Sum alpha = k, found by bisection; n = 2, k = 1
+                                        logistic; tau -> 0 hard top-k)
+  vp_gate                               pinned (alpha = 1 / 0 ends; variance preserved)
   decode_step, cache_from_prefill       pinned (equals the prefill over the extended
                                         sequences at the new positions, with and
                                         without bf16 storage)
@@ -364,6 +377,200 @@ def select_image(H_b, dec: Dict, *, k_max: int, g: int, group_size: int,
         eps_out.append(r)
         idx.extend(s + i for i in r["order"])
     return {"idx": restore(idx), "count": len(idx), "episodes": eps_out}
+
+
+# ----------------------------------------------------------------------------
+# training-time continuous pathway, forward only (Sec. 3.3: Eqs. 5-9)
+# ----------------------------------------------------------------------------
+#
+# Reading (rollout): the hard rollout is Eq. 4 exactly as at inference with one
+# token per step (the grouped rounds of Sec. 3.5 are an inference device): it
+# ends at the first hard STOP, at K_max kept tokens, or with only STOP left.
+# p_t = softmax(l_t / tau) is taken at every evaluated step (masked slots get
+# probability 0, STOP is the last slot, stop_bias enters l_t(STOP) as at
+# inference: pass 0 for the paper's training), and the sums of Eqs. 6-7 run over
+# those steps; steps after the end of the rollout contribute nothing.
+
+
+def trajectory_aggregate(P, beta: float) -> Dict:
+    """Eqs. 5-7 over the evaluated steps of one rollout.
+
+    P: [T, N+1] pointer distributions of steps t = 1..T (STOP in the last column).
+      A_1 = 1,  A_t = prod_{u<t} (1 - p_u(STOP))                     (Eq. 5)
+      s_i = sum_t A_t p_t(i) beta^t                                   (Eq. 6)
+      Kbar = sum_t A_t (1 - p_t(STOP))                                (Eq. 7)
+    """
+    P = _f(P)
+    T, n1 = P.shape
+    s = np.zeros(n1 - 1, dtype=F64)
+    kbar = 0.0
+    A = 1.0
+    alive = []
+    for t in range(1, T + 1):
+        p = P[t - 1]
+        alive.append(A)
+        s += A * p[:-1] * beta ** t
+        kbar += A * (1.0 - p[-1])
+        A *= 1.0 - p[-1]
+    return {"s": s, "kbar": kbar, "alive": np.asarray(alive)}
+
+
+def trajectory_episode(H, dec: Dict, *, k_max: int, tau: float, beta: float, stop_bias: float = 0.0,
+                       eps: float = 1e-5, mode: str = "incremental",
+                       force: Optional[Sequence[int]] = None, force_stop: Optional[bool] = None) -> Dict:
+    """The training-time rollout of one episode (Eq. 4 with g = 1) and its
+    aggregates (Eqs. 5-7).
+
+    Each step: l_t = PtrAttn(q_t, M) + Mask_t (+ stop_bias on STOP),
+    p_t = softmax(l_t / tau), a_t = argmax_j l_t(j) (lowest index on ties, so
+    STOP, the last slot, wins only when strictly above every available visual
+    logit); a visual a_t is masked and M[a_t] (the forward value of M^T p~_t)
+    joins the causal history.
+
+    force / force_stop: teacher forcing -- the actions taken are force[0..] and
+    then STOP iff force_stop (a rollout of another implementation replayed to
+    compare the distributions along it); the argmax is not consulted.
+    """
+    H = _f(H)
+    N = H.shape[0]
+    M = np.concatenate([H, _f(dec["s_stop"])[None, :]], axis=0)
+    stop = N
+    taken = np.zeros(N, dtype=bool)
+    S: List[int] = []
+    P: List[np.ndarray] = []
+    stopped = False
+    history = [_f(dec["s_start"])]
+    inc = None
+    if mode == "incremental":
+        inc = _IncrementalDecoder(M, dec, eps)
+        inc.append(history[0])
+    elif mode != "scratch":
+        raise ValueError(mode)
+    while len(S) < k_max:
+        if force is not None and len(S) == len(force) and not force_stop:
+            break
+        raw = inc.logits() if inc is not None else pointer_logits_from_scratch(np.stack(history), M, dec, eps)
+        logits = raw.copy()
+        logits[stop] += stop_bias
+        logits[:N][taken] = NEG_INF
+        P.append(softmax(logits / tau))
+        avail = np.flatnonzero(~taken)
+        if avail.size == 0:
+            stopped = True
+            break
+        if force is not None:
+            if len(S) == len(force):
+                stopped = True
+                break
+            a = int(force[len(S)])
+            if taken[a]:
+                raise ValueError("forced action already taken")
+        else:
+            best = avail[np.argmax(logits[avail])]  # argmax returns the lowest index among equals
+            if logits[stop] > logits[best]:
+                stopped = True
+                break
+            a = int(best)
+        S.append(a)
+        taken[a] = True
+        if inc is not None:
+            inc.append(M[a])
+        else:
+            history.append(M[a])
+    agg = trajectory_aggregate(np.stack(P), beta) if P else {"s": np.zeros(N), "kbar": 0.0, "alive": np.zeros(0)}
+    return {"order": S, "count": len(S), "stopped": stopped, "rounds": len(P), "P": np.stack(P) if P else None,
+            "s": agg["s"], "kbar": agg["kbar"], "alive": agg["alive"]}
+
+
+def soft_topk(s, k: float, tau: float, tol: float = 1e-13, max_iter: int = 1_000_000) -> np.ndarray:
+    """Eq. 8's SoftTopK_{k,tau}(s), which the paper only cites (the optimal-
+    transport top-k of Xie et al., 2020).
+
+    Reading: the entropic optimal transport of the n scores (mass 1/n each) onto
+    two anchors y = (0, 1) with masses ((n - k)/n, k/n), cost (s_i - y_j)^2 and
+    entropic regularisation tau; alpha_i = n Gamma_i,2, the share of token i sent
+    to the "kept" anchor.  Solved here by Sinkhorn's alternating scaling in the
+    log domain until the row marginals are met to `tol` (the column marginals
+    are exact after each column update).  k <= 0 gives all zeros and k >= n all
+    ones (the transport plan is then fixed by the marginals alone).
+    """
+    s = _f(s).ravel()
+    n = s.size
+    if n == 0:
+        return np.zeros(0)
+    if k <= 0:
+        return np.zeros(n)
+    if k >= n:
+        return np.ones(n)
+    y = np.array([0.0, 1.0])
+    C = (s[:, None] - y[None, :]) ** 2
+    log_mu = np.full(n, -math.log(n))
+    log_nu = np.log(np.array([(n - k) / n, k / n]))
+
+    def lse(x, axis):
+        m = np.max(x, axis=axis, keepdims=True)
+        return (m + np.log(np.sum(np.exp(x - m), axis=axis, keepdims=True))).squeeze(axis)
+
+    f = np.zeros(n)
+    g = np.zeros(2)
+    for _ in range(max_iter):
+        f = tau * (log_mu - lse((g[None, :] - C) / tau, axis=1))
+        g = tau * (log_nu - lse((f[:, None] - C) / tau, axis=0))
+        G = np.exp((f[:, None] + g[None, :] - C) / tau)
+        if np.max(np.abs(G.sum(axis=1) * n - 1.0)) < tol:
+            break
+    else:
+        raise RuntimeError("Sinkhorn did not converge")
+    return n * G[:, 1]
+
+
+def vp_gate(x, alpha, noise) -> np.ndarray:
+    """Eq. 9: x~_i = sqrt(alpha_i) x_i + sqrt(1 - alpha_i) eps_i, one alpha per
+    token (row); the Gaussian draws eps are an input."""
+    a = _f(alpha)[:, None]
+    return np.sqrt(a) * _f(x) + np.sqrt(1.0 - a) * _f(noise)
+
+
+def train_forward(H, n_vis: Sequence[int], dec: Dict, *, k_max: int, group_size: int, tau: float,
+                  beta: float, topk_tau: float, stop_bias: Sequence[float], X=None, noise=None,
+                  eps: float = 1e-5, mode: str = "incremental", forced: Optional[Sequence] = None) -> Dict:
+    """The continuous training pathway over a batch, forward only.
+
+    Per episode (an image, or one candidate group of it): trajectory_episode.
+    Per image: s = its episodes' scores at image positions, Kbar_b = the sum of
+    its episodes' soft counts.  Eq. 8: k = the batch mean of Kbar_b (detached;
+    the same k for every image, clamped to [0, N_b] per image), alpha_b =
+    SoftTopK_{k, topk_tau}(s_b).  Eq. 9 when X and noise are given.
+    forced: per episode (order, stopped) to replay instead of the argmax.
+    """
+    H = _f(H)
+    offs = np.concatenate([[0], np.cumsum(n_vis)]).astype(int)
+    s_all = np.zeros(offs[-1])
+    kbar_ep, kbar_img, eps_out = [], [], []
+    e = 0
+    for b, n in enumerate(n_vis):
+        gs = group_size if group_size > 0 else n
+        kb = 0.0
+        for c0 in range(0, n, gs):
+            f = forced[e] if forced is not None else (None, None)
+            r = trajectory_episode(H[offs[b] + c0: offs[b] + min(c0 + gs, n)], dec, k_max=k_max, tau=tau,
+                                   beta=beta, stop_bias=float(stop_bias[e]), eps=eps, mode=mode,
+                                   force=f[0], force_stop=f[1])
+            s_all[offs[b] + c0: offs[b] + c0 + len(r["s"])] = r["s"]
+            kbar_ep.append(r["kbar"])
+            kb += r["kbar"]
+            eps_out.append(r)
+            e += 1
+        kbar_img.append(kb)
+    k = float(np.mean(kbar_img))
+    alpha = np.zeros(offs[-1])
+    for b, n in enumerate(n_vis):
+        alpha[offs[b]:offs[b + 1]] = soft_topk(s_all[offs[b]:offs[b + 1]], min(max(k, 0.0), n), topk_tau)
+    out = {"s": s_all, "kbar": np.asarray(kbar_ep), "kbar_image": np.asarray(kbar_img), "k": k,
+           "alpha": alpha, "episodes": eps_out}
+    if X is not None and noise is not None:
+        out["x_gated"] = vp_gate(X, alpha, noise)
+    return out
 
 
 # ----------------------------------------------------------------------------
