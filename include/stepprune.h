@@ -227,6 +227,66 @@ SP_API sp_status sp_select_noalloc(const sp_selector* s, const sp_select_in* in,
                                    sp_stream stream);
 
 /* ------------------------------------------------------------------------ */
+/* Training-time continuous pathway, forward only (Sec. 3.3, Eqs. 5-9).      */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * The trajectory aggregates of Eqs. 5-7, accumulated along the hard rollout:
+ * at every evaluated step t of an episode, p_t = softmax(l_t / tau) over its
+ * available candidates and STOP (l_t as in sp_select, stop_bias included:
+ * pass zeros for the paper's training), and
+ *   A_1 = 1,  A_{t+1} = A_t (1 - p_t(STOP))                       (Eq. 5)
+ *   s_i  += A_t p_t(i) beta^t                                      (Eq. 6)
+ *   Kbar += A_t (1 - p_t(STOP))                                    (Eq. 7)
+ * The rollout is sp_select's (Eq. 4, hard argmax): it ends at the first hard
+ * STOP, at k_max kept tokens or with only STOP left; later steps contribute
+ * nothing.
+ */
+typedef struct {
+  float tau;        /* pointer temperature, > 0 */
+  float beta;       /* discount of Eq. 6, in (0, 1] */
+  float* score;     /* DEVICE [sum N_b] fp32 out: s_i, same rows as X / H (4-byte aligned) */
+  float* kbar;      /* DEVICE [n_episodes] fp32 out: Kbar per episode */
+} sp_train_args;
+
+/*
+ * sp_select plus the aggregates above, in the same launches (same workspace
+ * size as sp_select_workspace).  Requires g = 1 (one token per step, the
+ * rollout the aggregates are defined on) and an episode size whose keys fit
+ * the selection kernel's shared memory (up to 2,032 candidates per episode);
+ * otherwise SP_ERR_UNSUPPORTED before any launch.  SP_ERR_INVALID_ARG for a
+ * NULL score / kbar or tau <= 0 or beta outside (0, 1].
+ */
+SP_API sp_status sp_select_train(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
+                                 const sp_train_args* train, void* workspace, size_t workspace_bytes,
+                                 sp_stream stream);
+
+/*
+ * Eq. 8: alpha = SoftTopK_{k,tau}(s) per image, k = the batch mean of the
+ * images' soft counts (an image's count is the sum of its episodes' Kbar),
+ * detached, clamped to [0, N_b].  SoftTopK is the entropic optimal transport
+ * of an image's scores (mass 1/N_b each) onto the anchors 0 and 1 with masses
+ * (N_b - k, k) / N_b, cost (s_i - y)^2, regularisation tau; alpha_i is N_b
+ * times token i's mass sent to anchor 1, which equals
+ * sigmoid(2 (s_i - theta) / tau) with sum_i alpha_i = k (theta is solved for).
+ *   n_vis / group_size: HOST, as in sp_select_in (episodes image-major)
+ *   score: DEVICE [sum N_b] fp32, kbar: DEVICE [n_episodes] fp32
+ *   alpha: DEVICE [sum N_b] fp32 out;  k_out: DEVICE [1] fp32 out or NULL
+ * Errors: SP_ERR_INVALID_ARG / SP_ERR_SHAPE on bad sizes or pointers.
+ */
+SP_API sp_status sp_soft_topk(int B, const int* n_vis, int group_size, const float* score, const float* kbar,
+                              float tau, float* alpha, float* k_out, sp_stream stream);
+
+/*
+ * Eq. 9: x~ = sqrt(alpha_r) x + sqrt(1 - alpha_r) eps for every row r, fp32
+ * arithmetic, bf16 in and out.  X, noise, out: DEVICE [rows, D] bf16, 16-byte
+ * aligned, D a multiple of 8; alpha: DEVICE [rows] fp32 (clamped to [0, 1]).
+ * The Gaussian draws eps are the caller's.  out may alias X.
+ */
+SP_API sp_status sp_vp_gate(int rows, int D, const void* X, const void* noise, const float* alpha, void* out,
+                            sp_stream stream);
+
+/* ------------------------------------------------------------------------ */
 /* Compaction (Algorithm 1 step 5: X_S = Gather(X, S), then [X_S; text]).    */
 /* ------------------------------------------------------------------------ */
 
@@ -441,7 +501,7 @@ SP_API sp_status sp_pipeline_host(const sp_selector* s, const sp_model* m, const
 
 typedef enum {
   SP_K_GEMM = 0, SP_K_SGEMM = 1, SP_K_ATTN = 2, SP_K_NORM = 3, SP_K_SELECT = 4,
-  SP_K_RESTORE = 5, SP_K_COMPACT = 6, SP_K_MISC = 7, SP_K_COUNT = 8
+  SP_K_RESTORE = 5, SP_K_COMPACT = 6, SP_K_MISC = 7, SP_K_TRAIN = 8, SP_K_COUNT = 9
 } sp_kernel_kind;
 
 /* Starts (capacity > 0) or stops (0) recording launch events; host-allocated. */

@@ -24,7 +24,7 @@ SP_MAX_NVIS = 16384
 
 STATUS = {0: "SP_OK", 1: "SP_ERR_INVALID_ARG", 2: "SP_ERR_SHAPE", 3: "SP_ERR_ALIGN", 4: "SP_ERR_WORKSPACE",
           5: "SP_ERR_CUDA", 6: "SP_ERR_TIMEOUT", 7: "SP_ERR_UNSUPPORTED", 8: "SP_ERR_DEVICE"}
-KERNEL_KINDS = ["gemm", "sgemm", "attention", "norm", "select", "restore", "compact", "misc"]
+KERNEL_KINDS = ["gemm", "sgemm", "attention", "norm", "select", "restore", "compact", "misc", "train"]
 PROJ = {"none": 0, "linear": 1, "mlp2": 2}
 
 EXPORTS = [
@@ -33,7 +33,7 @@ EXPORTS = [
     "sp_model_destroy", "sp_project_workspace", "sp_project", "sp_prefill_workspace", "sp_prefill",
     "sp_pipeline_workspace", "sp_pipeline", "sp_pipeline_host_workspace", "sp_pipeline_host",
     "sp_profile_begin", "sp_profile_end", "sp_select_noalloc", "sp_probe_smem_gbs", "sp_probe_l2_gbs",
-    "sp_probe_select_floor", "sp_decode_workspace", "sp_decode",
+    "sp_probe_select_floor", "sp_decode_workspace", "sp_decode", "sp_select_train", "sp_soft_topk", "sp_vp_gate",
 ]
 SP_SELECT_NOALLOC_SCRATCH_BYTES = 64 << 20
 
@@ -66,6 +66,10 @@ class sp_select_in(C.Structure):
 class sp_select_out(C.Structure):
     _fields_ = [("idx", P), ("k_cap", C.c_int), ("count", P), ("order", P), ("ep_count", P),
                 ("margin", P), ("gap", P), ("rounds", P), ("memory", P), ("err", P)]
+
+
+class sp_train_args(C.Structure):
+    _fields_ = [("tau", C.c_float), ("beta", C.c_float), ("score", P), ("kbar", P)]
 
 
 class sp_compact_in(C.Structure):
@@ -150,6 +154,10 @@ def lib():
         "sp_pipeline_host_workspace": (C.c_size_t, [P, P, C.POINTER(sp_pipeline_host_io)]),
         "sp_pipeline_host": (C.c_int, [P, P, C.POINTER(sp_pipeline_host_io), P, C.c_size_t, P]),
         "sp_select_noalloc": (C.c_int, [P, C.POINTER(sp_select_in), C.POINTER(sp_select_out), P]),
+        "sp_select_train": (C.c_int, [P, C.POINTER(sp_select_in), C.POINTER(sp_select_out),
+                                      C.POINTER(sp_train_args), P, C.c_size_t, P]),
+        "sp_soft_topk": (C.c_int, [C.c_int, IP, C.c_int, P, P, C.c_float, P, P, P]),
+        "sp_vp_gate": (C.c_int, [C.c_int, C.c_int, P, P, P, P, P]),
         "sp_profile_begin": (C.c_int, [C.c_int]),
         "sp_profile_end": (C.c_int, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]),
@@ -300,10 +308,12 @@ def _select_in(n_vis, n_txt, X, E_text, H, stop_bias, group_size, g, k_max, keep
 
 def sp_select(sel: Selector, n_vis, n_txt, *, stop_bias, X=None, E_text=None, H=None, group_size=0, g=1,
               k_max=192, k_cap=None, traces=True, memory=False, stream=None, ws=None,
-              no_alloc=False) -> Dict:
+              no_alloc=False, train=None) -> Dict:
     """Runs sp_select; returns device tensors idx [B, k_cap], count [B] and, with
     traces, order / ep_count / margin / gap / rounds / err.  no_alloc=True calls
-    sp_select_noalloc instead (no workspace; the library's static scratch)."""
+    sp_select_noalloc instead (no workspace; the library's static scratch).
+    train=(tau, beta) calls sp_select_train and adds score [sum N_b] and
+    kbar [n_episodes] (the trajectory aggregates, Eqs. 5-7)."""
     torch = _torch()
     dev = sel.device
     keep: List = []
@@ -332,9 +342,43 @@ def sp_select(sel: Selector, n_vis, n_txt, *, stop_bias, X=None, E_text=None, H=
         return out
     if ws is None:
         ws = workspace(lib().sp_select_workspace(sel.handle, C.byref(inp)), dev)
+    if train is not None:
+        out["score"] = torch.empty(sum(n_vis), dtype=torch.float32, device=dev)
+        out["kbar"] = torch.empty(E, dtype=torch.float32, device=dev)
+        ta = sp_train_args(float(train[0]), float(train[1]), ptr(out["score"]), ptr(out["kbar"]))
+        _check(lib().sp_select_train(sel.handle, C.byref(inp), C.byref(o), C.byref(ta), ptr(ws), ws.numel(),
+                                     _stream(stream)), "sp_select_train")
+        out["k_cap"] = k_cap
+        out["_ws"] = ws
+        return out
     _check(lib().sp_select(sel.handle, C.byref(inp), C.byref(o), ptr(ws), ws.numel(), _stream(stream)), "sp_select")
     out["k_cap"] = k_cap
     out["_ws"] = ws
+    return out
+
+
+def sp_soft_topk(n_vis, *, score, kbar, tau, group_size=0, stream=None, alpha=None) -> Dict:
+    """Eq. 8 per image (k = the batch mean of the images' soft counts); returns
+    alpha [sum N_b] fp32 and k [1] fp32 (device tensors)."""
+    torch = _torch()
+    dev = score.device
+    nv = _int_array(n_vis)
+    if alpha is None:
+        alpha = torch.empty(sum(n_vis), dtype=torch.float32, device=dev)
+    k = torch.empty(1, dtype=torch.float32, device=dev)
+    _check(lib().sp_soft_topk(len(n_vis), C.cast(nv, IP), int(group_size), ptr(score), ptr(kbar), float(tau),
+                              ptr(alpha), ptr(k), _stream(stream)), "sp_soft_topk")
+    return {"alpha": alpha, "k": k}
+
+
+def sp_vp_gate(*, X, noise, alpha, out=None, stream=None):
+    """Eq. 9 on bf16 rows: out = sqrt(alpha) X + sqrt(1 - alpha) noise."""
+    torch = _torch()
+    if out is None:
+        out = torch.empty_like(X)
+    rows, D = X.shape
+    _check(lib().sp_vp_gate(int(rows), int(D), ptr(X), ptr(noise), ptr(alpha), ptr(out), _stream(stream)),
+           "sp_vp_gate")
     return out
 
 
@@ -533,7 +577,7 @@ def sp_profile_begin(capacity: int = 1 << 16):
 
 
 def sp_profile_end() -> Dict[str, Dict[str, float]]:
-    n = 8
+    n = len(KERNEL_KINDS)
     ms = (C.c_double * n)()
     la = (C.c_longlong * n)()
     fl = (C.c_double * n)()

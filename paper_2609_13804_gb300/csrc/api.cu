@@ -488,10 +488,22 @@ size_t sp_select_workspace(const sp_selector* s, const sp_select_in* in) {
 }
 
 static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const sp_select_out* out, void* ws,
-                             size_t ws_bytes, cudaStream_t st) {
+                             size_t ws_bytes, cudaStream_t st, const sp_train_args* tr = nullptr) {
   SelPlan p;
   sp_status rs = plan_select(s, in, &p);
   if (rs != SP_OK) return rs;
+  if (tr) {
+    if (!tr->score || !tr->kbar || (reinterpret_cast<uintptr_t>(tr->score) & 3) ||
+        (reinterpret_cast<uintptr_t>(tr->kbar) & 3))
+      return fail(SP_ERR_INVALID_ARG, "sp_select_train: score and kbar (4-byte aligned) are required");
+    if (!(tr->tau > 0.f) || !std::isfinite(tr->tau) || !(tr->beta > 0.f) || !(tr->beta <= 1.f))
+      return fail(SP_ERR_INVALID_ARG, "sp_select_train: need tau > 0 and beta in (0, 1]");
+    if (in->g != 1) return fail(SP_ERR_UNSUPPORTED, "sp_select_train: the rollout of Eqs. 5-7 takes g = 1");
+    bool ks = true;
+    size_t sm = 0;
+    select_cluster_size(p.bd, s->cfg.h, in->k_max, &ks, &sm);
+    if (!ks) return fail(SP_ERR_UNSUPPORTED, "sp_select_train: an episode's keys must fit shared memory");
+  }
   if (!out || !out->idx || !out->count) return fail(SP_ERR_INVALID_ARG, "sp_select: idx and count are required");
   if (!in->stop_bias) return fail(SP_ERR_INVALID_ARG, "sp_select: stop_bias is required");
   if (p.encoder && (!in->X || (p.ntxt > 0 && s->cfg.n_enc_layers > 0 && !in->E_text)))
@@ -577,6 +589,10 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   a.ep_count = out->ep_count ? out->ep_count : (int*)parts[12];
   a.margin = out->margin; a.gap = out->gap; a.rounds = out->rounds;
   a.err = err;
+  a.score = tr ? tr->score : nullptr;
+  a.kbar = tr ? tr->kbar : nullptr;
+  a.inv_tau = tr ? 1.f / tr->tau : 1.f;
+  a.beta = tr ? tr->beta : 1.f;
   bool keys_smem = true;
   size_t smem = 0;
   const int C = select_cluster_size(p.bd, h, in->k_max, &keys_smem, &smem);
@@ -588,6 +604,36 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
 sp_status sp_select(const sp_selector* s, const sp_select_in* in, const sp_select_out* out, void* ws,
                     size_t ws_bytes, sp_stream stream) {
   return select_impl(s, in, out, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+sp_status sp_select_train(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
+                          const sp_train_args* train, void* ws, size_t ws_bytes, sp_stream stream) {
+  if (!train) return fail(SP_ERR_INVALID_ARG, "sp_select_train: train arguments are required");
+  return select_impl(s, in, out, ws, ws_bytes, (cudaStream_t)stream, train);
+}
+
+sp_status sp_soft_topk(int B, const int* n_vis, int group_size, const float* score, const float* kbar, float tau,
+                       float* alpha, float* k_out, sp_stream stream) {
+  if (B < 1 || B > SP_MAX_BATCH || !n_vis) return fail(SP_ERR_INVALID_ARG, "sp_soft_topk: bad batch");
+  if (!score || !kbar || !alpha) return fail(SP_ERR_INVALID_ARG, "sp_soft_topk: score, kbar and alpha are required");
+  if (!(tau > 0.f) || !std::isfinite(tau)) return fail(SP_ERR_INVALID_ARG, "sp_soft_topk: need tau > 0");
+  std::vector<int> zeros(B, 0);
+  BatchDesc bd;
+  std::string msg;
+  if (!fill_batch_desc(&bd, B, n_vis, zeros.data(), group_size, &msg))
+    return fail(SP_ERR_SHAPE, "sp_soft_topk: %s", msg.c_str());
+  SP_CUDA(soft_topk_launch(bd, bd.ep_off[B], score, kbar, tau, alpha, k_out, (cudaStream_t)stream), "soft top-k");
+  return SP_OK;
+}
+
+sp_status sp_vp_gate(int rows, int D, const void* X, const void* noise, const float* alpha, void* out,
+                     sp_stream stream) {
+  if (rows < 0 || D <= 0 || D % 8) return fail(SP_ERR_SHAPE, "sp_vp_gate: rows >= 0 and D a multiple of 8");
+  if (rows == 0) return SP_OK;
+  if (!X || !noise || !alpha || !out) return fail(SP_ERR_INVALID_ARG, "sp_vp_gate: NULL pointer");
+  if (!al16(X) || !al16(noise) || !al16(out)) return fail(SP_ERR_ALIGN, "sp_vp_gate: X, noise, out 16-byte aligned");
+  SP_CUDA(vp_gate_launch(X, noise, alpha, out, rows, D, (cudaStream_t)stream), "vp gate");
+  return SP_OK;
 }
 
 }  // extern "C"

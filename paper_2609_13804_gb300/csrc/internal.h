@@ -167,11 +167,22 @@ struct SelectArgs {
   int h, k_max, g;
   int* order; int* ep_count; float* margin; float* gap; int* rounds;
   int* err;
+  // training-time pathway (Sec. 3.3): set score to also accumulate Eqs. 5-7
+  // along the rollout (g = 1, keys in shared memory); NULL otherwise
+  float* score;    // [sum N_b] s_i of Eq. 6, image-major rows
+  float* kbar;     // [n_episodes] Eq. 7
+  float inv_tau;   // 1 / pointer temperature
+  float beta;      // discount of Eq. 6
 };
 
 int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes);
 cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs& a,
                           int cluster, bool keys_in_smem, size_t smem_bytes, cudaStream_t st);
+// training-time pathway (train.cu)
+cudaError_t soft_topk_launch(const BatchDesc& bd, int n_episodes, const float* score, const float* kbar, float tau,
+                             float* alpha, float* k_out, cudaStream_t st);
+cudaError_t vp_gate_launch(const void* X, const void* noise, const float* alpha, void* out, int rows, int D,
+                           cudaStream_t st);
 cudaError_t restore_launch(const BatchDesc& bd, const int* order, const int* ep_count, int k_max,
                            int* idx, int k_cap, int* count, int* err, cudaStream_t st);
 

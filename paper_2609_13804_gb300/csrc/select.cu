@@ -47,7 +47,7 @@ constexpr int GMAX = 16;  // largest g; lists hold g + 1 entries
 
 struct SelSmem {
   size_t kt, lgp, stopkt, wpart_o, wpart_ml, all_o, all_ml, wtop_v, wtop_i, all_tv, all_ti, xp, taken, hist, misc,
-      total;
+      wsm, all_sm, score, total;
 };
 
 __host__ __device__ inline size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
@@ -74,6 +74,11 @@ __host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C
   L.taken = o;    o += al16((size_t)n_loc);
   L.hist = o;     o += al16((size_t)(k_max + 1) * 4);
   L.misc = o;     o += al16(128 * 4);
+  // training pathway: per-warp / per-CTA softmax partials (max, sum) and the
+  // CTA's scores of Eq. 6
+  L.wsm = o;      o += al16((size_t)NW * 2 * 4);
+  L.all_sm = o;   o += al16((size_t)2 * C * 2 * 4);
+  L.score = o;    o += al16((size_t)n_loc * 4);
   L.total = o;
   return L;
 }
@@ -210,7 +215,12 @@ SP_DEVINL void warp_merge_lists(const float* vin, const int* iin, int tot, int p
 // HV = h / 128: float4 slices per lane of an h-vector (lane holds elements
 // 4 (lane + 32 k) .. +3, k < HV).  GL = capacity of the per-round top lists
 // (g + 1 <= GL).  P = history positions a warp loads at once.
-template <int HV, int GL>
+// TRAIN: also accumulate the training pathway's aggregates along the rollout
+// (Eqs. 5-7; g = 1 and keys in shared memory only): every CTA merges the C
+// softmax partials (max, sum) of the round's available logits with STOP's in
+// rank order, adds A_t beta^t p_t(j) to the scores of its own candidates and
+// advances A_t and the soft count identically.
+template <int HV, int GL, bool TRAIN>
 __global__ void __launch_bounds__(NT, 1)
 select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in_smem, int tm_cols) {
   constexpr int P = (16 / HV) > 0 ? 16 / HV : 1;
@@ -261,6 +271,10 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   float* gtop_v = misc + 64;                          // [64, 81)
   int* gtop_i = reinterpret_cast<int*>(misc + 96);    // [96, 113)
   uint32_t* tm_slot = reinterpret_cast<uint32_t*>(misc + 124);
+  float* smx = misc + 20;                             // [20, 23) merged softmax: max, 1 / sum, p(STOP)
+  float* wsm = reinterpret_cast<float*>(sm + L.wsm);
+  float* all_sm = reinterpret_cast<float*>(sm + L.all_sm);
+  float* score_s = reinterpret_cast<float*>(sm + L.score);
 
   // TMEM cache of the history rows this CTA attends over (tm_cols columns; 0 =
   // off): a key / value row is read from L2 once, in the round its position
@@ -289,6 +303,8 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   for (int i = tid; i < h4; i += NT)
     reinterpret_cast<float4*>(stopkt)[i] = __ldg(reinterpret_cast<const float4*>(KT + (size_t)a.stop_row * a.ldkt) + i);
   for (int j = tid; j < n_loc_max; j += NT) taken[j] = 0;
+  if (TRAIN)
+    for (int j = tid; j < n_loc_max; j += NT) score_s[j] = 0.f;
   if (tid == 0) hist[0] = a.start_row;
   const float bias = __ldg(a.stop_bias + e);
   const size_t trace = (size_t)e * (k_max + 1);
@@ -325,6 +341,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   };
   load_last(a.start_row);
 
+  float alive = 1.f, disc = a.beta, kbar_acc = 0.f;  // A_t, beta^t, Eq. 7 (TRAIN)
   int nsel = 0, round = 0;
   while (nsel < k_max) {
     const int n_avail = n_e - nsel;
@@ -518,6 +535,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
 #pragma unroll
     for (int k = 0; k < GL; ++k) { tv[k] = -INFINITY; ti[k] = INT_MAX; }
     float stop_raw;
+    float vkeep = -INFINITY;  // this thread's candidate logit (keys in shared memory), -inf if unavailable
     if (keys_in_smem) {
       // dims-major keys: warp w takes a slice of the dims, lane = column
       // (candidates and, at column nl, STOP); per-warp partials are summed per
@@ -559,6 +577,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
         v = sj;
         id = j0 + tid;
       }
+      vkeep = v;
       // this warp's top g+1 (one candidate per lane)
       uint32_t key = (id == INT_MAX) ? 0u : fkey(v);
 #pragma unroll
@@ -571,6 +590,14 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           tv[r] = fkey_inv(mk);
           ti[r] = mk ? mi : INT_MAX;
           if (id == mi) { key = 0u; id = INT_MAX; }
+        }
+      }
+      if (TRAIN) {  // the warp's softmax partial relative to its best logit tv[0]
+        const float ex = (vkeep != -INFINITY) ? expf((vkeep - tv[0]) * a.inv_tau) : 0.f;
+        const float l_w = warp_sum(ex);
+        if (lane == 0) {
+          wsm[warp * 2] = tv[0];
+          wsm[warp * 2 + 1] = l_w;
         }
       }
     } else {
@@ -614,6 +641,17 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
         warp_merge_lists<GL, 1>(wtop_v, wtop_i, NW * per, per, cv, ci);
       else
         warp_merge_lists<GL, 9>(wtop_v, wtop_i, NW * per, per, cv, ci);
+      if (TRAIN) {  // the CTA's softmax partial, pushed with its list
+        const float mw = lane < NW ? wsm[lane * 2] : -INFINITY;
+        const float lw = lane < NW ? wsm[lane * 2 + 1] : 0.f;
+        const float mc = fkey_inv(__reduce_max_sync(0xffffffffu, fkey(mw)));
+        const float lc = warp_sum(mw == -INFINITY ? 0.f : lw * expf((mw - mc) * a.inv_tau));
+        if (lane < C) {
+          float* d = cluster.map_shared_rank(all_sm + ((size_t)buf * C + rank) * 2, lane);
+          d[0] = mc;
+          d[1] = lc;
+        }
+      }
       if (lane < C) {
         float* dv = cluster.map_shared_rank(all_tv + (size_t)buf * C * (GMAX + 1) + rank * per, lane);
         int* di = cluster.map_shared_rank(all_ti + (size_t)buf * C * (GMAX + 1) + rank * per, lane);
@@ -647,8 +685,28 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           }
         }
       }
+      if (TRAIN) {  // p_t = softmax(l_t / tau) over the available candidates and STOP
+        const float sl = stop_raw + bias;
+        const float mr = lane < C ? all_sm[((size_t)buf * C + lane) * 2] : -INFINITY;
+        const float lr = lane < C ? all_sm[((size_t)buf * C + lane) * 2 + 1] : 0.f;
+        const float mx = fmaxf(fkey_inv(__reduce_max_sync(0xffffffffu, fkey(mr))), sl);
+        const float zv = warp_sum(mr == -INFINITY ? 0.f : lr * expf((mr - mx) * a.inv_tau));
+        const float es = expf((sl - mx) * a.inv_tau);
+        if (lane == 0) {
+          smx[0] = mx;
+          smx[1] = 1.f / (zv + es);
+          smx[2] = es / (zv + es);
+        }
+      }
     }
     __syncthreads();
+    if (TRAIN) {  // Eqs. 5-7 at this step (identical A_t in every CTA)
+      const float ps = smx[2];
+      if (vkeep != -INFINITY) score_s[tid] += alive * disc * (expf((vkeep - smx[0]) * a.inv_tau) * smx[1]);
+      kbar_acc += alive * (1.f - ps);
+      alive *= 1.f - ps;
+      disc *= a.beta;
+    }
     const float stop_logit = stop_raw + bias;
     const float best = gtop_v[0];
     if (rank == 0 && tid == 0) {
@@ -695,6 +753,11 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   if (rank == 0 && tid == 0) {
     if (a.ep_count) a.ep_count[e] = nsel;
     if (a.rounds) a.rounds[e] = round;
+    if (TRAIN) a.kbar[e] = kbar_acc;
+  }
+  if (TRAIN) {
+    __syncthreads();
+    for (int j = tid; j < nl; j += NT) a.score[row0 + j0 + j] = score_s[j];
   }
   tc_fence_before();
   cluster.sync();  // no CTA leaves while a peer may still write into it
@@ -801,9 +864,13 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
   const SelSmem L = sel_layout(a.h, n_loc, a.k_max, C, keys_in_smem);
   void (*kern)(const BatchDesc, const SelectArgs, int, int, int) = nullptr;
   const int gl = a.g + 1 <= 2 ? 2 : (a.g + 1 <= 6 ? 6 : 17);
-#define SP_SEL_CASE(HV_)                                                                                   \
-  case HV_:                                                                                                \
-    kern = gl == 2 ? select_kernel<HV_, 2> : (gl == 6 ? select_kernel<HV_, 6> : select_kernel<HV_, 17>); \
+  const bool train = a.score != nullptr;
+  if (train && (a.g != 1 || !keys_in_smem || !a.kbar)) return cudaErrorInvalidValue;
+#define SP_SEL_CASE(HV_)                                                                             \
+  case HV_:                                                                                          \
+    kern = train ? select_kernel<HV_, 2, true>                                                       \
+                 : (gl == 2 ? select_kernel<HV_, 2, false>                                           \
+                            : (gl == 6 ? select_kernel<HV_, 6, false> : select_kernel<HV_, 17, false>)); \
     break;
   switch (a.h / 128) {
     SP_SEL_CASE(1)

@@ -96,3 +96,18 @@ def test_create_without_a_gpu_reports_instead_of_crashing(L):
     st = L.sp_selector_create(C.byref(cfg), C.byref(w), C.byref(h))
     assert st in (5, 7)  # SP_ERR_CUDA / SP_ERR_UNSUPPORTED
     assert not h.value
+
+
+def test_training_pathway_layout_and_argument_checks(L):
+    assert C.sizeof(b.sp_train_args) == 4 + 4 + 8 + 8
+    assert L.sp_select_train(None, None, None, None, None, 0, None) == 1   # no train arguments
+    nv = b._int_array([4, 3])
+    ok = C.c_void_p(256)  # never dereferenced: every call below fails on the host first
+    assert L.sp_soft_topk(0, C.cast(nv, b.IP), 0, ok, ok, 0.1, ok, None, None) == 1       # B = 0
+    assert L.sp_soft_topk(2, C.cast(nv, b.IP), 0, None, ok, 0.1, ok, None, None) == 1     # no scores
+    assert L.sp_soft_topk(2, C.cast(nv, b.IP), 0, ok, ok, 0.0, ok, None, None) == 1       # tau = 0
+    assert L.sp_soft_topk(2, C.cast(nv, b.IP), -1, ok, ok, 0.1, ok, None, None) == 2      # bad group size
+    assert L.sp_vp_gate(4, 12, ok, ok, ok, ok, None) == 2                                  # D not a multiple of 8
+    assert L.sp_vp_gate(0, 16, None, None, None, None, None) == 0                          # nothing to do
+    assert L.sp_vp_gate(4, 16, None, ok, ok, ok, None) == 1
+    assert L.sp_vp_gate(4, 16, C.c_void_p(264), ok, ok, ok, None) == 3                     # X misaligned
