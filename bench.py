@@ -474,6 +474,33 @@ def run_ours(args):
     def cache_bytes(lens):
         return 2.0 * 2 * m.n_layers * m.n_kv_heads * m.head_dim * sum(n + 1 for n in lens)
 
+    # ---- the training-time pathway's forward on the same batch (Eqs. 5-9):
+    #      the rollout with its aggregates (same STOP biases, so the same
+    #      trajectory as the timed selection), SoftTopK, the gate on X
+    def do_train_select():
+        return B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bias, group_size=w.group_size,
+                           g=1, k_max=w.k_max, traces=False, ws=sel_ws, train=(1.0, 0.99))
+
+    tr = do_train_select()
+    select_train_ms = timed(do_train_select)
+    alpha_buf = torch.empty(sum(w.n_vis), dtype=torch.float32, device=dev)
+    topk_ms = kernel_ms(lambda: B.sp_soft_topk(w.n_vis, score=tr["score"], kbar=tr["kbar"], tau=0.05,
+                                               group_size=w.group_size, alpha=alpha_buf))
+    noise = torch.randn(X.shape, device=dev, generator=gen).to(torch.bfloat16)
+    gated = torch.empty_like(X)
+    gate_ms = kernel_ms(lambda: B.sp_vp_gate(X=X, noise=noise, alpha=alpha_buf, out=gated))
+    gate_bytes = 3.0 * X.numel() * 2
+    del noise, gated
+    # bandwidth-sized gate: 256 images of 576 tokens (0.9 GB moved)
+    big_rows = 256 * 576
+    Xg = torch.randn((big_rows, s.D), device=dev, generator=gen).to(torch.bfloat16)
+    Ng = torch.randn((big_rows, s.D), device=dev, generator=gen).to(torch.bfloat16)
+    Ag = torch.rand(big_rows, device=dev, generator=gen)
+    Og = torch.empty_like(Xg)
+    gate_big_ms = kernel_ms(lambda: B.sp_vp_gate(X=Xg, noise=Ng, alpha=Ag, out=Og))
+    gate_big_bytes = 3.0 * Xg.numel() * 2
+    del Xg, Ng, Ag, Og
+
     # ---- end to end from host buffers (copies inside the timed region)
     Xh = X.cpu().pin_memory()
     Eh = E.cpu().pin_memory()
@@ -539,6 +566,14 @@ def run_ours(args):
                        "hbm_frac_pruned": (weight_bytes + cache_bytes(pruned_lens)) / (dec_pruned_ms * 1e-3) / 1e9
                        / pk["hbm_gbs"],
                        "bytes_note": "weights of the 32 layers + the cache rows read, per step"},
+            "train_forward": {
+                "select_ms": select_ms, "select_train_ms": select_train_ms,
+                "aggregates_overhead": select_train_ms / select_ms - 1.0,
+                "soft_topk_us": 1e3 * topk_ms, "vp_gate_us": 1e3 * gate_ms,
+                "vp_gate_gbs": gate_bytes / (gate_ms * 1e-3) / 1e9,
+                "vp_gate_256_images_gbs": gate_big_bytes / (gate_big_ms * 1e-3) / 1e9,
+                "vp_gate_256_images_hbm_frac": gate_big_bytes / (gate_big_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
+                "note": "tau 1.0, beta 0.99, SoftTopK tau 0.05; the gate reads X and noise, writes the gated rows"},
         }
         print(json.dumps(line), flush=True)
     if dist:
