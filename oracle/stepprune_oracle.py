@@ -9,7 +9,8 @@ A plain, slow, fp64 restatement of what the inference path of StepPrune
   * grouped execution, TopG per non-STOP round          (Sec. 3.5, Eq. 11)
   * Algorithm 1: loop, restore to native order, gather  (Algorithm 1; Sec. 3.3, last paragraph)
   * frozen projector and LM prefill over the packed prefix (Sec. 3.3-3.4; LM dims of the
-    evaluated backbones, Sec. 4.1)
+    evaluated backbones, Sec. 4.1), with 1-D RoPE or the 3-D mRoPE of the Qwen2.5-VL
+    backbone (Sec. 1)
   * the training-time continuous pathway, forward only: trajectory aggregation,
     soft count, SoftTopK polarisation, variance-preserving noise gate (Sec. 3.3,
     Eqs. 5-9)
@@ -30,6 +31,9 @@ Parity status of each function:
                                         special case, Eq. 1; invariants of Alg. 1 and Eq. 11)
   restore / compact                     pinned (hand-worked golden fixture; invariants)
   rope                                  pinned (rotation closed form, relative-position property)
+  mrope, mrope_positions                pinned (equal components -> rope; componentwise
+                                        relative positions; norm kept; pruned positions
+                                        = the full sequence's rows, by a grid walk)
   round_bf16                            pinned (torch's float32 -> bfloat16 conversion)
   trajectory_aggregate                  pinned (closed forms of Eqs. 5-7 for a constant
                                         STOP probability; Sum_i s_i = Kbar at beta = 1)
@@ -630,6 +634,53 @@ def rope(x, pos, n_heads: int, head_dim: int, theta: float) -> np.ndarray:
     return np.concatenate([a * c - b * s, b * c + a * s], axis=-1).reshape(x.shape[0], -1)
 
 
+def mrope(x, pos3, n_heads: int, head_dim: int, theta: float, section: Sequence[int]) -> np.ndarray:
+    """Three-dimensional multimodal rotary embedding (the mRoPE of the
+    Qwen2.5-VL backbone the method is evaluated on, Sec. 1 and Sec. 4.1).
+
+    Reading: the dh/2 rotation pairs of every head are cut into consecutive
+    sections of section[0], section[1], section[2] pairs (temporal, height,
+    width); pair i of section c is rotated (rotate-half, as `rope`) by angle
+    pos3[:, c] * theta^(-2i/dh), i counted over all dh/2 pairs.
+    """
+    x = _f(x).reshape(x.shape[0], n_heads, head_dim)
+    half = head_dim // 2
+    if sum(section) != half:
+        raise ValueError("mRoPE sections must cover the dh/2 pairs")
+    comp = np.repeat(np.arange(3), section)
+    inv = theta ** (-(2.0 * np.arange(half, dtype=F64)) / head_dim)
+    ang = _f(pos3)[:, comp] * inv[None, :]
+    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    a, b = x[..., :half], x[..., half:]
+    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1).reshape(x.shape[0], -1)
+
+
+def mrope_positions(kept, n_vis: int, grid_w: int, n_txt: int) -> np.ndarray:
+    """(t, h, w) positions of one packed sequence [kept visual tokens; text].
+
+    Reading (Sec. 3.3, last paragraph: the kept tokens are restored to native
+    order so the backbone's positional convention holds): the image's N tokens
+    form a grid of ceil(N / grid_w) rows of grid_w tokens at time 0; a kept
+    token keeps its grid position (0, row, column); the text after the image
+    continues, on all three components, from the largest position of the whole
+    (unpruned) image block plus one, as it would without pruning.  So every
+    row of the pruned sequence has the position it has in the full sequence.
+    """
+    kept = np.asarray(kept, dtype=np.int64)
+    gh = -(-n_vis // grid_w)
+    vis = np.stack([np.zeros_like(kept), kept // grid_w, kept % grid_w], axis=1)
+    start = max(gh, grid_w)
+    txt = np.repeat((start + np.arange(n_txt))[:, None], 3, axis=1)
+    return np.concatenate([vis, txt], axis=0).astype(F64)
+
+
+def _rotary(x, pos, n_heads: int, m) -> np.ndarray:
+    """rope for 1-D positions, mrope (the model's sections) for [rows, 3] ones."""
+    if np.ndim(pos) == 2:
+        return mrope(x, pos, n_heads, m.head_dim, m.rope_theta, m.mrope_section)
+    return rope(x, pos, n_heads, m.head_dim, m.rope_theta)
+
+
 def _mm(a, b, acc: str) -> np.ndarray:
     """a @ b with fp64 arithmetic, or (acc='fp32') with fp32 operands and an
     fp32 result, the precision of a tensor-core product's accumulator."""
@@ -657,8 +708,8 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
     Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
     x = _store(rms_norm(h, m.rms_eps, L.get("attn_norm")), store)
     qkv = _mm(x, _f(L["Wqkv"]).T, acc)
-    q = _store(rope(qkv[:, :Hq * dh], pos, Hq, dh, m.rope_theta), store)
-    k = _store(rope(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, dh, m.rope_theta), store)
+    q = _store(_rotary(qkv[:, :Hq * dh], pos, Hq, m), store)
+    k = _store(_rotary(qkv[:, Hq * dh:(Hq + Hkv) * dh], pos, Hkv, m), store)
     v = _store(qkv[:, (Hq + Hkv) * dh:], store)
     if kv_out is not None:
         kv_out.append((k.copy(), v.copy()))
@@ -699,19 +750,21 @@ def cache_from_prefill(kv_rows, cu) -> List[List[tuple]]:
 
 
 def decode_step(x_new, layers: Sequence[Dict], m, cache: List[List[tuple]], final_gain=None,
-                store: Optional[str] = None):
+                store: Optional[str] = None, rope_pos=None):
     """One generation step after the prefill over the pruned prefix (the decode
     the paper's per-token and end-to-end latencies include): sequence b's new
     token x_new[b] takes position len_b = cache rows of b and attends to the
     cached rotated keys / values 0..len_b-1 and to itself.  The layer is the
     prefill's layer applied to that one row.  Returns the normalised hidden
     state of the new tokens [B, d] and the cache with their keys / values
-    appended."""
+    appended.  rope_pos: the new tokens' rotary positions when they are not
+    len_b (after an mRoPE prefix: generated text tokens have equal components,
+    so their mRoPE is the 1-D rotation at that position)."""
     h = _f(x_new).copy()
     B = h.shape[0]
     Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
     lens = [cache[0][b][0].shape[0] for b in range(B)]
-    pos = np.array(lens, dtype=F64)
+    pos = np.array(lens if rope_pos is None else rope_pos, dtype=F64)
     new_cache = []
     for L, layer_cache in zip(layers, cache):
         x = _store(rms_norm(h, m.rms_eps, L.get("attn_norm")), store)

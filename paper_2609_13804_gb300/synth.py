@@ -96,6 +96,7 @@ class ModelShape:
     proj_kind: str          # "none" | "linear" | "mlp2"
     proj_in: int            # visual width entering the projector
     proj_hidden: int        # hidden width of the 2-layer projector
+    mrope_section: tuple = (0, 0, 0)  # rotation pairs per (t, h, w) component; zeros: 1-D RoPE
 
 
 @dataclasses.dataclass

@@ -1,6 +1,7 @@
 """Pins of the CPU oracle against things other than itself: library routines
 (torch fp64 modules), closed forms, brute force and the special cases the paper's
 definitions reduce to.  No GPU, no CUDA library."""
+import dataclasses
 import json
 import math
 import os
@@ -311,6 +312,83 @@ def test_rope_is_a_rotation_with_relative_positions():
     d1 = O.rope(q, [5], 1, dh, 1e4) @ O.rope(k, [2], 1, dh, 1e4).T
     d2 = O.rope(q, [33], 1, dh, 1e4) @ O.rope(k, [30], 1, dh, 1e4).T
     np.testing.assert_allclose(d1, d2, atol=1e-12)
+
+
+def test_mrope_reduces_to_rope_and_keeps_componentwise_relative_positions():
+    dh, H, sec = 16, 2, (2, 3, 3)
+    x = S.normal(12, "x", (6, H * dh)).astype(np.float64)
+    p1 = np.array([0, 1, 2, 7, 100, 3])
+    # equal components: the 1-D rotation
+    np.testing.assert_allclose(O.mrope(x, np.repeat(p1[:, None], 3, 1), H, dh, 1e4, sec),
+                               O.rope(x, p1, H, dh, 1e4), atol=1e-13)
+    # one section holding every pair: the 1-D rotation by that component
+    p3 = np.stack([p1, 5 * p1 + 1, 3 - p1], axis=1)
+    for c in range(3):
+        one = [0, 0, 0]
+        one[c] = dh // 2
+        np.testing.assert_allclose(O.mrope(x, p3, H, dh, 1e4, one), O.rope(x, p3[:, c], H, dh, 1e4), atol=1e-13)
+    # pair lengths are kept
+    r = O.mrope(x, p3, H, dh, 1e4, sec).reshape(6, H, dh)
+    xr = x.reshape(6, H, dh)
+    np.testing.assert_allclose(xr[..., :8] ** 2 + xr[..., 8:] ** 2, r[..., :8] ** 2 + r[..., 8:] ** 2, atol=1e-12)
+    # <R(a) q, R(b) k> depends only on a - b, component by component
+    q = S.normal(12, "q", (1, dh)).astype(np.float64)
+    k = S.normal(12, "k", (1, dh)).astype(np.float64)
+    a, b, sh = np.array([[2, 5, 9]]), np.array([[0, 1, 4]]), np.array([[11, -3, 40]])
+    d1 = O.mrope(q, a, 1, dh, 1e4, sec) @ O.mrope(k, b, 1, dh, 1e4, sec).T
+    d2 = O.mrope(q, a + sh, 1, dh, 1e4, sec) @ O.mrope(k, b + sh, 1, dh, 1e4, sec).T
+    np.testing.assert_allclose(d1, d2, atol=1e-12)
+
+
+def _full_sequence_positions(n_vis, grid_w, n_txt):
+    """The unpruned sequence's (t, h, w) rows, by walking the grid row by row."""
+    rows, top = [], 0
+    for i in range(n_vis):
+        r, c = i // grid_w, i % grid_w
+        rows.append((0, r, c))
+        top = max(top, r, c)
+    for j in range(n_txt):
+        rows.append((top + 1 + j,) * 3)
+    return np.array(rows, dtype=np.float64)
+
+
+@pytest.mark.parametrize("n,gw,nt", [(16, 4, 3), (12, 4, 5), (10, 4, 2), (576, 24, 7), (7, 7, 1)])
+def test_mrope_positions_are_the_full_sequence_rows(n, gw, nt):
+    full = _full_sequence_positions(n, gw, nt)
+    np.testing.assert_array_equal(O.mrope_positions(np.arange(n), n, gw, nt), full)
+    kept = np.sort(np.random.default_rng(n).choice(n, size=max(1, n // 3), replace=False))
+    got = O.mrope_positions(kept, n, gw, nt)
+    np.testing.assert_array_equal(got, np.concatenate([full[kept], full[n:]]))
+    assert O.mrope_positions([], n, gw, nt).shape == (nt, 3)
+
+
+def test_decode_with_rotary_positions_equals_mrope_prefill():
+    """A generated text token (equal components) at position p after an mRoPE
+    prefix: decode_step with rope_pos = p is the prefill over the extended
+    sequence with that row's 3-D position (p, p, p)."""
+    w = S.tiny_workload(13, [6, 4], [2, 3], d=32, n_heads=4, n_kv_heads=2, head_dim=16, ffn=40)
+    m = dataclasses.replace(w.model, mrope_section=(2, 3, 3))
+    layers = [S.make_layer_weights(w, l, norm_affine=True) for l in range(2)]
+    for L in layers:
+        for k in ("Wqkv", "Wo", "Wgu", "Wdown"):
+            L[k] = L[k] / 0.02 * 0.15
+    lens, grids = [8, 7], [3, 2]
+    kept = [[0, 2, 3, 5, 6, 7], [0, 1, 3, 4]]
+    n_img = [8, 5]
+    pos3 = [O.mrope_positions(k, n, gw, t) for k, n, gw, t in zip(kept, n_img, grids, [2, 3])]
+    x = S.normal(13, "x", (sum(lens), 32)).astype(np.float64)
+    cu = np.array([0, 8, 15])
+    kv = []
+    O.prefill(x, layers, m, cu, np.concatenate(pos3), kv_out=kv)
+    cache = O.cache_from_prefill(kv, cu)
+    xn = S.normal(13, "xn", (2, 32)).astype(np.float64)
+    nxt = [int(p[-1, 0]) + 1 for p in pos3]
+    hid, _ = O.decode_step(xn, layers, m, cache, rope_pos=nxt)
+    for b in range(2):
+        xs = np.concatenate([x[cu[b]:cu[b + 1]], xn[b:b + 1]])
+        ps = np.concatenate([pos3[b], [[nxt[b]] * 3]])
+        ref = O.prefill(xs, layers, m, [0, len(xs)], ps)
+        np.testing.assert_allclose(hid[b], ref[-1], atol=1e-10)
 
 
 def _tiny_lm(seed, hq=4, hkv=2):
