@@ -348,6 +348,9 @@ typedef struct {
   int proj_kind;     /* sp_proj_kind */
   int proj_in;       /* visual width entering the projector */
   int proj_hidden;   /* hidden width of SP_PROJ_MLP2_GELU */
+  int mrope_section[3]; /* 3-D mRoPE (the Qwen2.5-VL backbone, Sec. 1): rotation pairs given to the
+                           (t, h, w) position components, consecutive from pair 0; the three sum
+                           to head_dim / 2, each even.  All zero: 1-D RoPE on pos. */
 } sp_model_cfg;
 
 /*
@@ -409,6 +412,10 @@ SP_API sp_status sp_project(const sp_model* m, const sp_project_io* io, void* wo
  *   kv + (((l * 2 + 0) * B + b) * kv_S_cap + p) * (n_kv_heads * head_dim)
  * and the value at the same offset with 1 in place of 0 (bf16).  Positions
  * must be < kv_S_cap (else SP_DEVERR_INDEX).
+ * With an mRoPE model (mrope_section set), pos3 gives every row's rotary
+ * (t, h, w) position (sp_mrope_positions writes it for a pruned batch); pos is
+ * then only the row's index within its sequence (its cache slot).  A rotary
+ * position >= max_pos sets SP_DEVERR_INDEX.
  */
 typedef struct {
   int B;
@@ -422,7 +429,25 @@ typedef struct {
   int* err;
   void* kv;                 /* DEVICE [n_layers][2][B][kv_S_cap][n_kv_heads * head_dim] bf16, or NULL */
   int kv_S_cap;             /* positions per sequence in kv */
+  const int* pos3;          /* DEVICE [T_cap, 4] int32 (t, h, w, unused); required iff mRoPE, else NULL */
 } sp_prefill_io;
+
+/*
+ * mRoPE positions of a pruned batch (reading of Sec. 3.3's last paragraph: the
+ * kept tokens are restored to native order so that the backbone's positional
+ * convention holds).  Image b's N_b tokens form a grid of ceil(N_b / grid_w[b])
+ * rows of grid_w[b] tokens at time 0; a kept token idx keeps its grid position
+ * (0, idx / grid_w, idx % grid_w); the text after it continues on all three
+ * components from max(rows, grid_w[b]) (the unpruned image block's largest
+ * position + 1).  Row cu + j of sequence b (cu = sum over earlier images of
+ * count + n_txt, the packing of sp_compact) gets the j-th position.
+ *   n_vis, n_txt, grid_w: HOST [B];  idx [B, k_cap], count [B]: DEVICE (sp_select)
+ *   pos3: DEVICE [T_cap, 4] int32 out (rows >= the packed length untouched)
+ * Errors: bad sizes -> SP_ERR_SHAPE; on the device, an index outside its image
+ * or a row >= T_cap sets SP_DEVERR_INDEX (the row is skipped).
+ */
+SP_API sp_status sp_mrope_positions(int B, const int* n_vis, const int* n_txt, const int* grid_w, const int* idx,
+                                    int k_cap, const int* count, int* pos3, int T_cap, int* err, sp_stream stream);
 
 SP_API size_t sp_prefill_workspace(const sp_model* m, int T_cap, int max_seqlen_cap);
 SP_API sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* workspace,
@@ -449,6 +474,10 @@ typedef struct {
   int max_len_cap;          /* bound on lens[b] + 1 (sizes the attention launch) */
   float* hidden;            /* DEVICE [B, d] fp32 output */
   int* err;
+  int* rope_pos;            /* DEVICE [B] int32 rotary position of each new token, or NULL (= lens);
+                               incremented with lens.  After an mRoPE prefix: the position the
+                               next text token takes (on all three components, so the 1-D
+                               rotation at that position) */
 } sp_decode_io;
 
 SP_API size_t sp_decode_workspace(const sp_model* m, int B);

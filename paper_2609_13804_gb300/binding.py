@@ -34,6 +34,7 @@ EXPORTS = [
     "sp_pipeline_workspace", "sp_pipeline", "sp_pipeline_host_workspace", "sp_pipeline_host",
     "sp_profile_begin", "sp_profile_end", "sp_select_noalloc", "sp_probe_smem_gbs", "sp_probe_l2_gbs",
     "sp_probe_select_floor", "sp_decode_workspace", "sp_decode", "sp_select_train", "sp_soft_topk", "sp_vp_gate",
+    "sp_mrope_positions",
 ]
 SP_SELECT_NOALLOC_SCRATCH_BYTES = 64 << 20
 
@@ -85,7 +86,8 @@ class sp_compact_out(C.Structure):
 class sp_model_cfg(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d", C.c_int), ("n_heads", C.c_int), ("n_kv_heads", C.c_int),
                 ("head_dim", C.c_int), ("ffn", C.c_int), ("max_pos", C.c_int), ("rope_theta", C.c_float),
-                ("rms_eps", C.c_float), ("proj_kind", C.c_int), ("proj_in", C.c_int), ("proj_hidden", C.c_int)]
+                ("rms_eps", C.c_float), ("proj_kind", C.c_int), ("proj_in", C.c_int), ("proj_hidden", C.c_int),
+                ("mrope_section", C.c_int * 3)]
 
 
 class sp_model_weights(C.Structure):
@@ -101,12 +103,13 @@ class sp_project_io(C.Structure):
 
 class sp_prefill_io(C.Structure):
     _fields_ = [("B", C.c_int), ("T_cap", C.c_int), ("max_seqlen_cap", C.c_int), ("x", P), ("cu_seqlens", P),
-                ("pos", P), ("hidden", P), ("residual", P), ("err", P), ("kv", P), ("kv_S_cap", C.c_int)]
+                ("pos", P), ("hidden", P), ("residual", P), ("err", P), ("kv", P), ("kv_S_cap", C.c_int),
+                ("pos3", P)]
 
 
 class sp_decode_io(C.Structure):
     _fields_ = [("B", C.c_int), ("x", P), ("lens", P), ("kv", P), ("kv_S_cap", C.c_int), ("max_len_cap", C.c_int),
-                ("hidden", P), ("err", P)]
+                ("hidden", P), ("err", P), ("rope_pos", P)]
 
 
 class sp_pipeline_io(C.Structure):
@@ -158,6 +161,7 @@ def lib():
                                       C.POINTER(sp_train_args), P, C.c_size_t, P]),
         "sp_soft_topk": (C.c_int, [C.c_int, IP, C.c_int, P, P, C.c_float, P, P, P]),
         "sp_vp_gate": (C.c_int, [C.c_int, C.c_int, P, P, P, P, P]),
+        "sp_mrope_positions": (C.c_int, [C.c_int, IP, IP, IP, P, C.c_int, P, P, C.c_int, P, P]),
         "sp_profile_begin": (C.c_int, [C.c_int]),
         "sp_profile_end": (C.c_int, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]),
@@ -457,7 +461,8 @@ class Model:
             w.proj_w2 = keep(dev_bf16(head["proj_W2"], device))
         cfg = sp_model_cfg(len(layers), shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
                            int(max_pos), float(shape.rope_theta), float(shape.rms_eps), PROJ[shape.proj_kind],
-                           shape.proj_in, shape.proj_hidden)
+                           shape.proj_in, shape.proj_hidden,
+                           (C.c_int * 3)(*[int(v) for v in getattr(shape, "mrope_section", (0, 0, 0))]))
         h = P()
         _check(lib().sp_model_create(C.byref(cfg), C.byref(w), C.byref(h)), "sp_model_create")
         self.handle = h
@@ -494,34 +499,51 @@ def kv_cache(model: Model, B: int, S_cap: int, device=None):
 
 
 def sp_prefill(model: Model, *, x, cu_seqlens, pos, B, T_cap, max_seqlen_cap, residual=None, stream=None,
-               ws=None, hidden=None, kv=None):
+               ws=None, hidden=None, kv=None, pos3=None):
     torch = _torch()
     dev = x.device
     if hidden is None:
         hidden = torch.zeros((max(T_cap, 1), model.shape.d), dtype=torch.float32, device=dev)
     err = torch.zeros(1, dtype=torch.int32, device=dev)
     io = sp_prefill_io(int(B), int(T_cap), int(max_seqlen_cap), ptr(x), ptr(cu_seqlens), ptr(pos), ptr(hidden),
-                       ptr(residual), ptr(err), ptr(kv), int(kv.shape[3]) if kv is not None else 0)
+                       ptr(residual), ptr(err), ptr(kv), int(kv.shape[3]) if kv is not None else 0, ptr(pos3))
     if ws is None:
         ws = workspace(lib().sp_prefill_workspace(model.handle, int(T_cap), int(max_seqlen_cap)), dev)
     _check(lib().sp_prefill(model.handle, C.byref(io), ptr(ws), ws.numel(), _stream(stream)), "sp_prefill")
     return {"hidden": hidden, "err": err, "_ws": ws}
 
 
-def sp_decode(model: Model, *, x, lens, kv, max_len_cap, stream=None, ws=None, hidden=None) -> Dict:
+def sp_decode(model: Model, *, x, lens, kv, max_len_cap, stream=None, ws=None, hidden=None, rope_pos=None) -> Dict:
     """One generation step: x [B, d] bf16 new tokens, lens [B] int32 cached lengths
-    (incremented on the device), kv the cache of kv_cache() / sp_prefill."""
+    (incremented on the device), kv the cache of kv_cache() / sp_prefill;
+    rope_pos [B] int32 rotary positions (default lens), incremented with lens."""
     torch = _torch()
     dev = x.device
     B = int(x.shape[0])
     if hidden is None:
         hidden = torch.zeros((B, model.shape.d), dtype=torch.float32, device=dev)
     err = torch.zeros(1, dtype=torch.int32, device=dev)
-    io = sp_decode_io(B, ptr(x), ptr(lens), ptr(kv), int(kv.shape[3]), int(max_len_cap), ptr(hidden), ptr(err))
+    io = sp_decode_io(B, ptr(x), ptr(lens), ptr(kv), int(kv.shape[3]), int(max_len_cap), ptr(hidden), ptr(err),
+                      ptr(rope_pos))
     if ws is None:
         ws = workspace(lib().sp_decode_workspace(model.handle, B), dev)
     _check(lib().sp_decode(model.handle, C.byref(io), ptr(ws), ws.numel(), _stream(stream)), "sp_decode")
     return {"hidden": hidden, "err": err, "_ws": ws}
+
+
+def sp_mrope_positions(n_vis, n_txt, grid_w, *, idx, count, k_cap, T_cap, stream=None, pos3=None, err=None):
+    """(t, h, w) rotary positions [T_cap, 4] int32 of the packed, pruned batch."""
+    torch = _torch()
+    dev = idx.device
+    if pos3 is None:
+        pos3 = torch.zeros((max(int(T_cap), 1), 4), dtype=torch.int32, device=dev)
+    if err is None:
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+    nv, nt, gw = _int_array(n_vis), _int_array(n_txt), _int_array(grid_w)
+    _check(lib().sp_mrope_positions(len(n_vis), C.cast(nv, IP), C.cast(nt, IP), C.cast(gw, IP), ptr(idx), int(k_cap),
+                                    ptr(count), ptr(pos3), int(T_cap), ptr(err), _stream(stream)),
+           "sp_mrope_positions")
+    return {"pos3": pos3, "err": err}
 
 
 class Pipeline:

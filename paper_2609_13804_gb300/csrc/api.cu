@@ -705,6 +705,12 @@ sp_status sp_model_create(const sp_model_cfg* cfg, const sp_model_weights* w, sp
   if (c.max_pos < 1 || c.max_pos > (1 << 20)) return fail(SP_ERR_SHAPE, "max_pos out of range");
   if (!(c.rope_theta > 0.f) || !(c.rms_eps > 0.f)) return fail(SP_ERR_INVALID_ARG, "rope_theta and rms_eps must be > 0");
   if (c.proj_kind < SP_PROJ_NONE || c.proj_kind > SP_PROJ_MLP2_GELU) return fail(SP_ERR_INVALID_ARG, "bad proj_kind");
+  {
+    const int* ms = c.mrope_section;
+    const int sum = ms[0] + ms[1] + ms[2];
+    if (sum != 0 && (ms[0] < 0 || ms[1] < 0 || ms[2] < 0 || (ms[0] | ms[1] | ms[2]) & 1 || sum != c.head_dim / 2))
+      return fail(SP_ERR_SHAPE, "mrope_section: three even pair counts summing to head_dim / 2 (or all zero)");
+  }
   if (c.proj_kind != SP_PROJ_NONE) {
     if (c.proj_in <= 0 || c.proj_in % 64) return fail(SP_ERR_SHAPE, "proj_in must be a multiple of 64");
     if (!w->proj_w1) return fail(SP_ERR_INVALID_ARG, "proj_w1 required");
@@ -849,6 +855,8 @@ sp_status sp_project(const sp_model* m, const sp_project_io* io, void* ws, size_
 struct PrefillParts {
   float* h32;
   void *xb, *qkv, *ob, *act, *gsk;
+  float2* mrows = nullptr;  // mRoPE: per packed row (cos, sin) of every rotation pair
+  int* mident = nullptr;    // mRoPE: row r -> r
   float* splitk = nullptr;  // small-M split-K planes (T_cap <= 128)
   size_t splitk_floats = 0;
 };
@@ -867,6 +875,10 @@ static size_t prefill_ws(const sp_model* m, int T_cap, bool own_residual, Carve&
   q.ob = cv.take<uint16_t>(T * c.n_heads * c.head_dim);
   q.act = cv.take<uint16_t>(T * c.ffn);
   q.gsk = cv.take<char>(gemm_scratch_bytes());
+  if (c.mrope_section[0] + c.mrope_section[1] + c.mrope_section[2] > 0) {
+    q.mrows = cv.take<float2>(T * (c.head_dim / 2));
+    q.mident = cv.take<int>(T);
+  }
   if (T_cap <= 128) {
     q.splitk_floats = gemm_splitk_floats((int)model_max_n(c));
     q.splitk = cv.take<float>(q.splitk_floats);
@@ -886,12 +898,16 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
   const sp_model_cfg& c = m->cfg;
   if (io->B < 1 || io->B > SP_MAX_BATCH || io->T_cap < 0 || io->max_seqlen_cap < 0)
     return fail(SP_ERR_SHAPE, "sp_prefill: bad B / T_cap / max_seqlen_cap");
-  if (io->max_seqlen_cap > c.max_pos) return fail(SP_ERR_SHAPE, "sp_prefill: max_seqlen_cap %d > max_pos %d", io->max_seqlen_cap, c.max_pos);
+  const bool mrope = c.mrope_section[0] + c.mrope_section[1] + c.mrope_section[2] > 0;
+  if (!mrope && io->max_seqlen_cap > c.max_pos)  // (mRoPE positions are checked on the device)
+    return fail(SP_ERR_SHAPE, "sp_prefill: max_seqlen_cap %d > max_pos %d", io->max_seqlen_cap, c.max_pos);
   if (!io->x || !io->cu_seqlens || !io->pos || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_prefill: x, cu_seqlens, pos, hidden required");
   if (!al16(io->x) || !al16(io->hidden) || (io->residual && !al16(io->residual)) || (io->kv && !al16(io->kv)))
     return fail(SP_ERR_ALIGN, "sp_prefill: buffers must be 16-byte aligned");
   if (io->kv && io->kv_S_cap < io->max_seqlen_cap)
     return fail(SP_ERR_SHAPE, "sp_prefill: kv_S_cap %d < max_seqlen_cap %d", io->kv_S_cap, io->max_seqlen_cap);
+  if (mrope && (!io->pos3 || !al16(io->pos3)))
+    return fail(SP_ERR_INVALID_ARG, "sp_prefill: an mRoPE model needs pos3 (16-byte aligned)");
   if (io->T_cap == 0) return SP_OK;
   Carve cv(ws);
   PrefillParts p;
@@ -915,15 +931,19 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
   // the attention's last key tile reads up to 63 rows past the packed length
   // (weighted by zero); keep them finite: the QKV GEMMs leave them untouched
   SP_CUDA(zero_rows_after(p.qkv, (size_t)qkvw * 2, T_dev, T_cap, 64, st), "qkv tail");
+  if (mrope)
+    SP_CUDA(mrope_rows_launch(m->rope, c.max_pos, c.head_dim / 2, io->pos3, c.mrope_section[0],
+                              c.mrope_section[0] + c.mrope_section[1], T_dev, T_cap, p.mrows, p.mident, io->err, st),
+            "mrope rows");
   for (int l = 0; l < c.n_layers; ++l) {
     SP_CUDA(rmsnorm_f32_to_bf16(h32, m->w.attn_norm[l], p.xb, T_cap, T_dev, c.d, c.rms_eps, st), "attn norm");
     GemmEpi eq;
     eq.kind = EPI_BF16_ROPE;
     eq.out = p.qkv;
     eq.ldo = qkvw;
-    eq.rope = m->rope;
-    eq.pos = io->pos;
-    eq.max_pos = c.max_pos;
+    eq.rope = mrope ? p.mrows : m->rope;
+    eq.pos = mrope ? p.mident : io->pos;
+    eq.max_pos = mrope ? T_cap : c.max_pos;
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
     SP_CUDA(gemm_bf16(tX, T_cap, T_dev, m->qkv[l], qkvw, eq, io->err, st, &gs), "qkv");
@@ -954,6 +974,23 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
 
 sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* ws, size_t ws_bytes, sp_stream stream) {
   return prefill_impl(m, io, ws, ws_bytes, (cudaStream_t)stream);
+}
+
+sp_status sp_mrope_positions(int B, const int* n_vis, const int* n_txt, const int* grid_w, const int* idx, int k_cap,
+                             const int* count, int* pos3, int T_cap, int* err, sp_stream stream) {
+  BatchDesc bd;
+  std::string msg;
+  if (!fill_batch_desc(&bd, B, n_vis, n_txt, 0, &msg)) return fail(SP_ERR_SHAPE, "sp_mrope_positions: %s", msg.c_str());
+  if (!grid_w || !idx || !count || !pos3) return fail(SP_ERR_INVALID_ARG, "sp_mrope_positions: NULL argument");
+  if (k_cap < 1 || T_cap < 0) return fail(SP_ERR_SHAPE, "sp_mrope_positions: bad k_cap / T_cap");
+  if (!al16(pos3)) return fail(SP_ERR_ALIGN, "sp_mrope_positions: pos3 must be 16-byte aligned");
+  GridDesc gd;
+  for (int b = 0; b < B; ++b) {
+    if (grid_w[b] < 1 || grid_w[b] > n_vis[b]) return fail(SP_ERR_SHAPE, "sp_mrope_positions: grid_w[%d] out of 1..N_b", b);
+    gd.grid_w[b] = grid_w[b];
+  }
+  SP_CUDA(mrope_positions_launch(bd, gd, idx, k_cap, count, pos3, T_cap, err, (cudaStream_t)stream), "mrope positions");
+  return SP_OK;
 }
 
 // ------------------------------------------------------------------ decode
@@ -988,7 +1025,8 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
   const sp_model_cfg& c = m->cfg;
   if (io->B < 1 || io->B > SP_MAX_BATCH || io->kv_S_cap < 1 || io->max_len_cap < 1 || io->max_len_cap > io->kv_S_cap)
     return fail(SP_ERR_SHAPE, "sp_decode: bad B / kv_S_cap / max_len_cap");
-  if (io->max_len_cap > c.max_pos) return fail(SP_ERR_SHAPE, "sp_decode: max_len_cap %d > max_pos %d", io->max_len_cap, c.max_pos);
+  if (!io->rope_pos && io->max_len_cap > c.max_pos)  // (explicit rotary positions are checked on the device)
+    return fail(SP_ERR_SHAPE, "sp_decode: max_len_cap %d > max_pos %d", io->max_len_cap, c.max_pos);
   if (!io->x || !io->lens || !io->kv || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_decode: x, lens, kv, hidden required");
   if (!al16(io->x) || !al16(io->kv) || !al16(io->hidden)) return fail(SP_ERR_ALIGN, "sp_decode: buffers must be 16-byte aligned");
   Carve cv(ws);
@@ -1016,7 +1054,7 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
     eq.out = p.qkv;
     eq.ldo = qkvw;
     eq.rope = m->rope;
-    eq.pos = io->lens;  // the new token's position is the cached length
+    eq.pos = io->rope_pos ? io->rope_pos : io->lens;  // default: the cached length
     eq.max_pos = c.max_pos;
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
@@ -1040,7 +1078,7 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
     SP_CUDA(gemm_bf16(tA, B, nullptr, m->down[l], c.d, er, io->err, st, &gs), "down");
   }
   SP_CUDA(rmsnorm_f32_to_f32(p.h32, m->w.final_norm, io->hidden, B, nullptr, c.d, c.rms_eps, st), "final norm");
-  SP_CUDA(lens_increment(io->lens, B, io->kv_S_cap, st), "lens");
+  SP_CUDA(lens_increment(io->lens, io->rope_pos, B, io->kv_S_cap, st), "lens");
   return SP_OK;
 }
 

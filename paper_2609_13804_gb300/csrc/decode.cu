@@ -161,9 +161,12 @@ __global__ void __launch_bounds__(128) decode_attn_kernel(const __nv_bfloat16* _
   }
 }
 
-__global__ void lens_increment_kernel(int* lens, int B, int S_cap) {
+__global__ void lens_increment_kernel(int* lens, int* rope_pos, int B, int S_cap) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < B && lens[b] < S_cap) lens[b] += 1;
+  if (b < B && lens[b] < S_cap) {
+    lens[b] += 1;
+    if (rope_pos) rope_pos[b] += 1;
+  }
 }
 
 }  // namespace
@@ -212,8 +215,8 @@ cudaError_t decode_attention(const void* qkv, const void* kv_l, int S_cap, const
   return cudaGetLastError();
 }
 
-cudaError_t lens_increment(int* lens, int B, int S_cap, cudaStream_t st) {
-  lens_increment_kernel<<<(B + 127) / 128, 128, 0, st>>>(lens, B, S_cap);
+cudaError_t lens_increment(int* lens, int* rope_pos, int B, int S_cap, cudaStream_t st) {
+  lens_increment_kernel<<<(B + 127) / 128, 128, 0, st>>>(lens, rope_pos, B, S_cap);
   return cudaGetLastError();
 }
 

@@ -19,6 +19,11 @@ struct BatchDesc {
   int ep_off[SP_MAX_BATCH + 1];   // prefix of episodes per image
 };
 
+// grid width (tokens per row) of every image of a batch (mRoPE positions)
+struct GridDesc {
+  int grid_w[SP_MAX_BATCH];
+};
+
 bool fill_batch_desc(BatchDesc* d, int B, const int* n_vis, const int* n_txt, int group_size,
                      std::string* msg);
 
@@ -144,7 +149,7 @@ cudaError_t kv_append(const void* qkv, const int* lens, int B, int Hq, int Hkv, 
                       int* err, cudaStream_t st);
 cudaError_t decode_attention(const void* qkv, const void* kv_l, int S_cap, const int* lens, int B, int Hq, int Hkv,
                              int dh, void* out, cudaStream_t st);
-cudaError_t lens_increment(int* lens, int B, int S_cap, cudaStream_t st);
+cudaError_t lens_increment(int* lens, int* rope_pos, int B, int S_cap, cudaStream_t st);
 
 // ------------------------------------------------------------- attention
 // Varlen attention over packed qkv [rows_cap, (Hq + 2 Hkv) dh] bf16 -> out [T, Hq dh] bf16
@@ -178,6 +183,11 @@ struct SelectArgs {
 int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes);
 cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs& a,
                           int cluster, bool keys_in_smem, size_t smem_bytes, cudaStream_t st);
+// 3-D mRoPE (mrope.cu)
+cudaError_t mrope_positions_launch(const BatchDesc& bd, const GridDesc& gd, const int* idx, int k_cap,
+                                   const int* count, int* pos3, int T_cap, int* err, cudaStream_t st);
+cudaError_t mrope_rows_launch(const float2* rope, int max_pos, int half, const int* pos3, int s1, int s2,
+                              const int* T_dev, int T_cap, float2* rows, int* ident, int* err, cudaStream_t st);
 // training-time pathway (train.cu)
 cudaError_t soft_topk_launch(const BatchDesc& bd, int n_episodes, const float* score, const float* kbar, float tau,
                              float* alpha, float* k_out, cudaStream_t st);

@@ -45,8 +45,9 @@ def test_struct_sizes_match_header_layout():
 
 
 def test_prefill_and_decode_io_layout():
-    assert C.sizeof(b.sp_prefill_io) == 4 * 3 + 4 + 8 * 6 + 8 + 4 + 4
-    assert C.sizeof(b.sp_decode_io) == 4 + 4 + 8 * 3 + 4 * 2 + 8 * 2
+    assert C.sizeof(b.sp_prefill_io) == 4 * 3 + 4 + 8 * 6 + 8 + 4 + 4 + 8
+    assert C.sizeof(b.sp_decode_io) == 4 + 4 + 8 * 3 + 4 * 2 + 8 * 2 + 8
+    assert C.sizeof(b.sp_model_cfg) == 4 * 15
 
 
 def test_decode_argument_checks_fail_before_any_launch(L):
@@ -111,3 +112,13 @@ def test_training_pathway_layout_and_argument_checks(L):
     assert L.sp_vp_gate(0, 16, None, None, None, None, None) == 0                          # nothing to do
     assert L.sp_vp_gate(4, 16, None, ok, ok, ok, None) == 1
     assert L.sp_vp_gate(4, 16, C.c_void_p(264), ok, ok, ok, None) == 3                     # X misaligned
+
+
+def test_mrope_argument_checks(L):
+    nv, nt, gw = b._int_array([16, 9]), b._int_array([2, 3]), b._int_array([4, 3])
+    ok = C.c_void_p(256)
+    args = lambda g, kc, p: (2, C.cast(nv, b.IP), C.cast(nt, b.IP), C.cast(g, b.IP), ok, kc, ok, p, 64, None, None)  # noqa: E731
+    assert L.sp_mrope_positions(*args(gw, 0, ok)) == 2                      # k_cap 0
+    assert L.sp_mrope_positions(*args(b._int_array([4, 10]), 8, ok)) == 2  # grid wider than the image
+    assert L.sp_mrope_positions(*args(gw, 8, None)) == 1
+    assert L.sp_mrope_positions(*args(gw, 8, C.c_void_p(260))) == 3         # pos3 misaligned
