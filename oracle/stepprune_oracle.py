@@ -27,7 +27,8 @@ Parity status of each function:
   attention                             pinned (torch scaled_dot_product_attention, brute force)
   text_projection, encoder              pinned (torch.nn.TransformerEncoderLayer, fp64)
   pointer logits / select_episode       pinned (brute-force from-scratch decoder; torch
-                                        nn.MultiheadAttention decoder; history-free top-K
+                                        nn.MultiheadAttention decoder; deeper decoders against
+                                        torch nn.TransformerDecoderLayer; history-free top-K
                                         special case, Eq. 1; invariants of Alg. 1 and Eq. 11)
   restore / compact                     pinned (hand-worked golden fixture; invariants)
   rope                                  pinned (rotation closed form, relative-position property)
@@ -216,10 +217,38 @@ def encoder(X, E_tilde, sel: Dict, n_heads: int, eps: float) -> np.ndarray:
 #   In the last layer the cross-attention values and the FFN do not feed the
 #   logits, so they are not computed.  The STOP logit gets an extra per-episode
 #   stop_bias (the knob that sets the mean retained count of random-init models).
+#
+# Deeper decoders (dec["lower"], one dict per layer before the last): each such
+#   layer is a whole pre-LN decoder layer of width h (Sec. 3.2: causal
+#   self-attention over the history, cross-attention to the memory M, a
+#   feed-forward network), its output the next layer's input:
+#     a = x + Wo_s SelfAttn(LN1(x))          causal, single head, 1/sqrt h
+#     c = a + Wo_c CrossAttn(LN2(a), M)      all N+1 rows of M (the mask acts on
+#                                            the pointer logits only)
+#     x' = c + W2 GELU(W1 LN3(c))            hidden width 4h, exact-erf GELU as in
+#                                            the encoder blocks
+#   and the top-level weights describe the last layer, as for one layer.
 
 def decoder_tokens(rows, dec: Dict) -> np.ndarray:
     """Decoder input tokens y = W_in m for rows m in the D-wide memory space."""
     return _f(rows) @ _f(dec["W_in"]).T
+
+
+def decoder_full_layer(X, M, L: Dict, eps: float) -> np.ndarray:
+    """One full decoder layer (a layer before the last) over a whole history X
+    [t, h]: causal self-attention, cross-attention to every row of M, FFN."""
+    X = _f(X)
+    h = X.shape[1]
+    t = X.shape[0]
+    x1 = layer_norm(X, eps, L.get("ln1_g"), L.get("ln1_b"))
+    S = (x1 @ _f(L["Wq_s"]).T) @ (x1 @ _f(L["Wk_s"]).T).T / math.sqrt(h)
+    S[np.triu_indices(t, 1)] = NEG_INF
+    a = X + (softmax(S, axis=-1) @ (x1 @ _f(L["Wv_s"]).T)) @ _f(L["Wo_s"]).T
+    x2 = layer_norm(a, eps, L.get("ln2_g"), L.get("ln2_b"))
+    Sc = (x2 @ _f(L["Wq_c"]).T) @ (_f(M) @ _f(L["Wk_c"]).T).T / math.sqrt(h)
+    c = a + (softmax(Sc, axis=-1) @ (_f(M) @ _f(L["Wv_c"]).T)) @ _f(L["Wo_c"]).T
+    x3 = layer_norm(c, eps, L.get("ln3_g"), L.get("ln3_b"))
+    return c + gelu(x3 @ _f(L["W1"]).T) @ _f(L["W2"]).T
 
 
 def pointer_keys(M, dec: Dict) -> np.ndarray:
@@ -232,6 +261,8 @@ def pointer_logits_from_scratch(history_rows, M, dec: Dict, eps: float) -> np.nd
     decoder over the history [q_1, ..., q_t] (no cached state)."""
     h = dec["W_in"].shape[0]
     Y = decoder_tokens(history_rows, dec)
+    for L in dec.get("lower", []):
+        Y = decoder_full_layer(Y, M, L, eps)
     X1 = layer_norm(Y, eps, dec.get("ln1_g"), dec.get("ln1_b"))
     Q = X1 @ _f(dec["Wq_s"]).T
     K = X1 @ _f(dec["Wk_s"]).T
@@ -252,13 +283,37 @@ class _IncrementalDecoder:
         self.dec, self.eps = dec, eps
         self.h = dec["W_in"].shape[0]
         self.Kp = pointer_keys(M, dec)
-        self.Y: List[np.ndarray] = []
+        self.Y: List[np.ndarray] = []      # inputs of the last layer
         self.Ks: List[np.ndarray] = []
         self.Vs: List[np.ndarray] = []
+        # layers before the last: their self-attention caches and the memory's
+        # cross-attention keys / values
+        self.lower = list(dec.get("lower", []))
+        self.lK: List[List[np.ndarray]] = [[] for _ in self.lower]
+        self.lV: List[List[np.ndarray]] = [[] for _ in self.lower]
+        self.cK = [_f(M) @ _f(L["Wk_c"]).T for L in self.lower]
+        self.cV = [_f(M) @ _f(L["Wv_c"]).T for L in self.lower]
+
+    def _through_lower(self, y):
+        """The new position through every layer before the last."""
+        x, h, e = y, self.h, self.eps
+        for i, L in enumerate(self.lower):
+            x1 = layer_norm(x, e, L.get("ln1_g"), L.get("ln1_b"))
+            self.lK[i].append(x1 @ _f(L["Wk_s"]).T)
+            self.lV[i].append(x1 @ _f(L["Wv_s"]).T)
+            att = softmax(np.stack(self.lK[i]) @ (x1 @ _f(L["Wq_s"]).T) / math.sqrt(h))
+            a = x + (att @ np.stack(self.lV[i])) @ _f(L["Wo_s"]).T
+            x2 = layer_norm(a, e, L.get("ln2_g"), L.get("ln2_b"))
+            ca = softmax(self.cK[i] @ (x2 @ _f(L["Wq_c"]).T) / math.sqrt(h))
+            c = a + (ca @ self.cV[i]) @ _f(L["Wo_c"]).T
+            x3 = layer_norm(c, e, L.get("ln3_g"), L.get("ln3_b"))
+            x = c + gelu(x3 @ _f(L["W1"]).T) @ _f(L["W2"]).T
+        return x
 
     def append(self, rows):
         d = self.dec
         for y in decoder_tokens(np.atleast_2d(rows), d):
+            y = self._through_lower(y)
             x = layer_norm(y, self.eps, d.get("ln1_g"), d.get("ln1_b"))
             self.Y.append(y)
             self.Ks.append(x @ _f(d["Wk_s"]).T)

@@ -73,6 +73,7 @@ class SelectorShape:
     enc_ffn_mult: int = 4
     ln_eps: float = 1e-5
     g_text: float = 1.0
+    n_dec_layers: int = 1  # pointer-decoder layers (the last one gives the logits)
 
     @property
     def enc_heads(self) -> int:
@@ -265,6 +266,23 @@ def make_selector_weights(w: Workload, ln_affine: bool = False) -> Dict[str, obj
         out[n] = f32("sel.dec." + n, (h, h))
     out["ln2_g"], out["ln2_b"] = ln("sel.dec.ln2", h)
     out["Wk_p"] = f32("sel.dec.Wk_p", (h, D))
+    # decoder layers before the last (pointer decoders of n_dec_layers > 1);
+    # the FFN matrices are bf16-representable (the GPU stores them as bf16)
+    lower = []
+    for i in range(getattr(s, "n_dec_layers", 1) - 1):
+        L = {}
+        L["ln1_g"], L["ln1_b"] = ln(f"sel.dec{i}.ln1", h)
+        for n in ("Wq_s", "Wk_s", "Wv_s", "Wo_s", "Wq_c", "Wo_c"):
+            L[n] = f32(f"sel.dec{i}.{n}", (h, h))
+        L["Wk_c"] = f32(f"sel.dec{i}.Wk_c", (h, D))
+        L["Wv_c"] = f32(f"sel.dec{i}.Wv_c", (h, D))
+        L["ln2_g"], L["ln2_b"] = ln(f"sel.dec{i}.ln2", h)
+        L["ln3_g"], L["ln3_b"] = ln(f"sel.dec{i}.ln3", h)
+        L["W1"] = bf(f"sel.dec{i}.W1", (4 * h, h))
+        L["W2"] = bf(f"sel.dec{i}.W2", (h, 4 * h))
+        lower.append(L)
+    if lower:
+        out["lower"] = lower
     return out
 
 

@@ -156,6 +156,78 @@ def test_pointer_logits_match_torch_multihead_attention_decoder():
     np.testing.assert_allclose(d_ours, d_ref, atol=1e-10)
 
 
+def _deep_selector(seed, n_dec, N=12, D=16, h=16, scale=0.3):
+    """Tiny selector with n_dec decoder layers; every decoder matrix scaled so
+    that each layer moves its input by O(1)."""
+    w = S.tiny_workload(seed, [N], [3], D=D, h=h)
+    w.selector = dataclasses.replace(w.selector, n_dec_layers=n_dec)
+    sel = S.make_selector_weights(w, ln_affine=True)
+    def sc(a):
+        return (a / 0.02 * scale / math.sqrt(a.shape[-1])).astype(np.float32)
+    for n in ("W_in", "Wq_s", "Wk_s", "Wv_s", "Wo_s", "Wq_p", "Wk_p", "s_start", "s_stop"):
+        sel[n] = sc(sel[n])
+    for L in sel.get("lower", []):
+        for n in ("Wq_s", "Wk_s", "Wv_s", "Wo_s", "Wq_c", "Wk_c", "Wv_c", "Wo_c", "W1", "W2"):
+            L[n] = sc(L[n])
+    return sel, S.make_memory(w).astype(np.float64)
+
+
+@pytest.mark.parametrize("n_dec", [2, 3])
+def test_deep_pointer_decoder_matches_torch_transformer_decoder_layers(n_dec):
+    """Layers before the last = torch.nn.TransformerDecoderLayer (pre-norm, one
+    head, no biases, GELU, FFN 4h) over the history with memory M (D = h here,
+    the module's constraint); the last layer as in the one-layer pin."""
+    sel, H = _deep_selector(40 + n_dec, n_dec)
+    N, D = H.shape
+    h = sel["W_in"].shape[0]
+    M = np.concatenate([H, sel["s_stop"][None].astype(np.float64)])
+    hist = np.stack([sel["s_start"], M[3], M[7], M[1], M[10]]).astype(np.float64)
+    ours = O.pointer_logits_from_scratch(hist, M, sel, 1e-5)
+    t = hist.shape[0]
+    causal = torch.triu(torch.full((t, t), float("-inf")), 1)
+    with torch.no_grad():
+        y = torch.nn.functional.linear(t64(hist), t64(sel["W_in"]))[None]
+        for L in sel["lower"]:
+            layer = torch.nn.TransformerDecoderLayer(h, 1, dim_feedforward=4 * h, dropout=0.0, activation="gelu",
+                                                     batch_first=True, norm_first=True, bias=False)
+            layer.self_attn.in_proj_weight.copy_(t64(np.concatenate([L["Wq_s"], L["Wk_s"], L["Wv_s"]])))
+            layer.self_attn.out_proj.weight.copy_(t64(L["Wo_s"]))
+            layer.multihead_attn.in_proj_weight.copy_(t64(np.concatenate([L["Wq_c"], L["Wk_c"], L["Wv_c"]])))
+            layer.multihead_attn.out_proj.weight.copy_(t64(L["Wo_c"]))
+            layer.linear1.weight.copy_(t64(L["W1"]))
+            layer.linear2.weight.copy_(t64(L["W2"]))
+            for k in (1, 2, 3):  # bias=False drops the norms' biases too: give them back
+                norm = torch.nn.LayerNorm(h, eps=1e-5)
+                norm.weight.copy_(t64(L[f"ln{k}_g"]))
+                norm.bias.copy_(t64(L[f"ln{k}_b"]))
+                setattr(layer, f"norm{k}", norm)
+            y = layer(y, t64(M)[None], tgt_mask=causal)
+        sa = torch.nn.MultiheadAttention(h, 1, bias=False, batch_first=True)
+        ca = torch.nn.MultiheadAttention(h, 1, bias=False, kdim=D, vdim=D, batch_first=True)
+        sa.in_proj_weight.copy_(t64(np.concatenate([sel["Wq_s"], sel["Wk_s"], sel["Wv_s"]])))
+        sa.out_proj.weight.copy_(t64(sel["Wo_s"]))
+        # D = h: the module packs the cross-attention projections
+        ca.in_proj_weight.copy_(torch.cat([t64(sel["Wq_p"]), t64(sel["Wk_p"]), torch.randn(h, D)]))
+        x = torch.nn.functional.layer_norm(y, (h,), t64(sel["ln1_g"]), t64(sel["ln1_b"]), 1e-5)
+        u = y + sa(x, x, x, attn_mask=causal, need_weights=False)[0]
+        x2 = torch.nn.functional.layer_norm(u[:, -1:], (h,), t64(sel["ln2_g"]), t64(sel["ln2_b"]), 1e-5)
+        _, p = ca(x2, t64(M)[None], t64(M)[None], need_weights=True)
+    logp = torch.log(p[0, 0]).numpy()
+    np.testing.assert_allclose(ours - ours.max(), logp - logp.max(), atol=1e-10)
+
+
+@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("n_dec", [2, 3])
+def test_deep_decoder_incremental_equals_brute_force(seed, n_dec):
+    sel, H = _deep_selector(140 + seed, n_dec, N=10, D=24)
+    for g in (1, 3):
+        for bias in (-0.3, 0.2, -1e9):
+            a = O.select_episode(H, sel, k_max=7, g=g, stop_bias=bias)
+            b = O.select_episode(H, sel, k_max=7, g=g, stop_bias=bias, mode="scratch")
+            assert a["order"] == b["order"] and a["stopped"] == b["stopped"]
+            np.testing.assert_allclose(a["gap"], b["gap"], atol=1e-11)
+
+
 @pytest.mark.parametrize("seed", range(12))
 @pytest.mark.parametrize("g", [1, 3])
 def test_incremental_selection_equals_brute_force(seed, g):
