@@ -61,6 +61,7 @@ extern "C" {
 /* Limits checked on the host (SP_ERR_SHAPE when exceeded). */
 #define SP_MAX_BATCH 256          /* images per call */
 #define SP_MAX_ENC_LAYERS 4       /* cross-modal encoder blocks */
+#define SP_MAX_DEC_LAYERS 4       /* pointer-decoder layers */
 #define SP_MAX_LM_LAYERS 96       /* decoder layers of the LM */
 #define SP_MAX_KMAX 1024          /* per-episode cap on retained tokens */
 #define SP_MAX_NVIS 16384         /* visual tokens of one image */
@@ -103,6 +104,7 @@ typedef struct {
   int enc_ffn;       /* encoder MLP width (4 D in a ViT block) */
   float ln_eps;      /* LayerNorm epsilon */
   float g_text;      /* text gate g_text of E~ = g_text LN(W_p E) (1 at inference) */
+  int n_dec_layers;  /* pointer-decoder layers, 1..SP_MAX_DEC_LAYERS (0 is read as 1) */
 } sp_selector_cfg;
 
 /*
@@ -118,7 +120,27 @@ typedef struct {
  * Wv_s x_i with x_i = LN1(y_i); the pointer logits are the cross-attention
  * scores l_t(j) = <Wq_p LN2(u_t), Wk_p M_j>/sqrt h over the N+1 rows of
  * M = [H; s_stop], plus a per-episode stop_bias on the STOP row.
+ *
+ * With n_dec_layers = L > 1 the fields below (ln1, Wq_s .. Wo_s, ln2, Wq_p,
+ * Wk_p) describe the LAST layer, and dec_lower[0 .. L-2] the layers before it,
+ * each a whole pre-LN decoder layer of width h (Sec. 3.2: self-attention,
+ * cross-attention to the memory, feed-forward network):
+ *   a  = x + Wo_s SelfAttn(LN1(x))            causal over the history
+ *   c  = a + Wo_c CrossAttn(LN2(a), M)        all N+1 rows of M, unmasked
+ *   x' = c + W2 GELU(W1 LN3(c))               hidden width 4h, exact-erf GELU
+ * x of layer 0 is y = W_in q; x' of layer L-2 enters the last layer.
  */
+typedef struct {
+  const float* ln1_g; const float* ln1_b;  /* [h] */
+  const float* Wq_s; const float* Wk_s; const float* Wv_s; const float* Wo_s;  /* [h, h] fp32 */
+  const float* ln2_g; const float* ln2_b;  /* [h] */
+  const float* Wq_c; const float* Wo_c;    /* [h, h] fp32 */
+  const float* Wk_c; const float* Wv_c;    /* [h, D] fp32 */
+  const float* ln3_g; const float* ln3_b;  /* [h] */
+  const void* W1;                          /* [4h, h] bf16 */
+  const void* W2;                          /* [h, 4h] bf16 */
+} sp_dec_layer_weights;
+
 typedef struct {
   const void* W_p;                         /* [D, D_text] bf16 text projection */
   const float* ln_text_g; const float* ln_text_b;    /* [D] */
@@ -136,6 +158,8 @@ typedef struct {
   const float* ln2_g; const float* ln2_b;  /* [h] */
   const float* Wq_p;                       /* [h, h] pointer query */
   const float* Wk_p;                       /* [h, D] pointer key */
+  const sp_dec_layer_weights* dec_lower;   /* HOST [n_dec_layers - 1] (copied at creation; the
+                                              DEVICE pointers inside are borrowed), or NULL */
 } sp_selector_weights;
 
 typedef struct sp_selector_s sp_selector;
@@ -202,7 +226,10 @@ typedef struct {
 SP_API int sp_num_episodes(int B, const int* n_vis, int group_size);
 /* Workspace bytes sp_select needs for this batch (0 on bad arguments). */
 SP_API size_t sp_select_workspace(const sp_selector* s, const sp_select_in* in);
-/* Algorithm 1 steps 1-4 for every image of the batch (see sp_select_in). */
+/* Algorithm 1 steps 1-4 for every image of the batch (see sp_select_in).
+ * A selector with n_dec_layers > 1 takes g = 1 only (each new history position
+ * runs through every layer before the next decision; SP_ERR_UNSUPPORTED
+ * otherwise, before any launch). */
 SP_API sp_status sp_select(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
                     void* workspace, size_t workspace_bytes, sp_stream stream);
 

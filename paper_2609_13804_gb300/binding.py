@@ -45,7 +45,14 @@ IP = C.POINTER(C.c_int)
 
 class sp_selector_cfg(C.Structure):
     _fields_ = [("D", C.c_int), ("D_text", C.c_int), ("h", C.c_int), ("n_enc_layers", C.c_int),
-                ("enc_head_dim", C.c_int), ("enc_ffn", C.c_int), ("ln_eps", C.c_float), ("g_text", C.c_float)]
+                ("enc_head_dim", C.c_int), ("enc_ffn", C.c_int), ("ln_eps", C.c_float), ("g_text", C.c_float),
+                ("n_dec_layers", C.c_int)]
+
+
+class sp_dec_layer_weights(C.Structure):
+    _fields_ = [("ln1_g", P), ("ln1_b", P), ("Wq_s", P), ("Wk_s", P), ("Wv_s", P), ("Wo_s", P), ("ln2_g", P),
+                ("ln2_b", P), ("Wq_c", P), ("Wo_c", P), ("Wk_c", P), ("Wv_c", P), ("ln3_g", P), ("ln3_b", P),
+                ("W1", P), ("W2", P)]
 
 
 class sp_selector_weights(C.Structure):
@@ -56,7 +63,7 @@ class sp_selector_weights(C.Structure):
                 ("enc_ln2_g", P * SP_MAX_ENC_LAYERS), ("enc_ln2_b", P * SP_MAX_ENC_LAYERS),
                 ("s_stop", P), ("s_start", P), ("W_in", P), ("ln1_g", P), ("ln1_b", P),
                 ("Wq_s", P), ("Wk_s", P), ("Wv_s", P), ("Wo_s", P), ("ln2_g", P), ("ln2_b", P),
-                ("Wq_p", P), ("Wk_p", P)]
+                ("Wq_p", P), ("Wk_p", P), ("dec_lower", C.POINTER(sp_dec_layer_weights))]
 
 
 class sp_select_in(C.Structure):
@@ -267,8 +274,22 @@ class Selector:
         for n in ("s_stop", "s_start", "W_in", "ln1_g", "ln1_b", "Wq_s", "Wk_s", "Wv_s", "Wo_s", "ln2_g",
                   "ln2_b", "Wq_p", "Wk_p"):
             setattr(w, n, keep(dev_f32(weights[n], device)))
+        lower = weights.get("lower", [])
+        nd = getattr(shape, "n_dec_layers", 1)
+        if len(lower) != nd - 1:
+            raise ValueError(f"{nd} decoder layers need {nd - 1} lower layers, got {len(lower)}")
+        if lower:
+            arr = (sp_dec_layer_weights * len(lower))()
+            for i, L in enumerate(lower):
+                for n in ("ln1_g", "ln1_b", "Wq_s", "Wk_s", "Wv_s", "Wo_s", "ln2_g", "ln2_b", "Wq_c", "Wo_c",
+                          "Wk_c", "Wv_c", "ln3_g", "ln3_b"):
+                    setattr(arr[i], n, keep(dev_f32(L[n], device)))
+                arr[i].W1 = keep(dev_bf16(L["W1"], device))
+                arr[i].W2 = keep(dev_bf16(L["W2"], device))
+            self._keep.append(arr)
+            w.dec_lower = C.cast(arr, C.POINTER(sp_dec_layer_weights))
         cfg = sp_selector_cfg(shape.D, shape.D_text, shape.h, nl, shape.enc_head_dim, shape.enc_ffn,
-                              shape.ln_eps, shape.g_text)
+                              shape.ln_eps, shape.g_text, int(nd))
         h = P()
         _check(lib().sp_selector_create(C.byref(cfg), C.byref(w), C.byref(h)), "sp_selector_create")
         self.handle = h

@@ -230,6 +230,13 @@ struct sp_selector_s {
   void* P2s = nullptr;  // [3h, 6h]
   GemmB P1, P2;
   GemmB Wp;
+  // decoders of several layers: Wcat1 also holds, per layer before the last,
+  // Wq_c^T Wk_c / sqrt(h) | Wo_c Wv_c; the runtime weights of layers >= 1
+  int n_dec = 1;
+  const float* pre_ln1_g = nullptr;  // layer 0's LN1 (applied in the precompute)
+  const float* pre_ln1_b = nullptr;
+  float* Wf = nullptr;               // [n_dec - 1][3h, h]
+  DecLayerDev* dec_dev = nullptr;    // [n_dec]
   GemmB enc_qkv[SP_MAX_ENC_LAYERS], enc_o[SP_MAX_ENC_LAYERS], enc_1[SP_MAX_ENC_LAYERS],
       enc_2[SP_MAX_ENC_LAYERS];
 };
@@ -298,22 +305,50 @@ sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weigh
   if (!(c.ln_eps > 0.f)) return fail(SP_ERR_INVALID_ARG, "ln_eps must be > 0");
   if (!w->s_stop || !w->s_start || !w->W_in || !w->Wq_s || !w->Wk_s || !w->Wv_s || !w->Wo_s || !w->Wq_p || !w->Wk_p)
     return fail(SP_ERR_INVALID_ARG, "pointer-decoder weights missing");
+  const int nd = c.n_dec_layers <= 0 ? 1 : c.n_dec_layers;
+  if (nd > SP_MAX_DEC_LAYERS) return fail(SP_ERR_SHAPE, "n_dec_layers must be in 1..SP_MAX_DEC_LAYERS");
+  if (nd > 1 && !w->dec_lower) return fail(SP_ERR_INVALID_ARG, "dec_lower is required with n_dec_layers > 1");
+  for (int l = 0; l + 1 < nd; ++l) {
+    const sp_dec_layer_weights& L = w->dec_lower[l];
+    if (!L.Wq_s || !L.Wk_s || !L.Wv_s || !L.Wo_s || !L.Wq_c || !L.Wo_c || !L.Wk_c || !L.Wv_c || !L.W1 || !L.W2)
+      return fail(SP_ERR_INVALID_ARG, "decoder layer %d weights missing", l);
+    if ((reinterpret_cast<uintptr_t>(L.W1) | reinterpret_cast<uintptr_t>(L.W2)) & 15)
+      return fail(SP_ERR_ALIGN, "decoder layer %d: W1 / W2 must be 16-byte aligned", l);
+  }
 
   sp_selector* s = new (std::nothrow) sp_selector_s();
   if (!s) return fail(SP_ERR_INVALID_ARG, "out of host memory");
   s->cfg = c;
   s->w = *w;
   const int h = c.h, D = c.D;
+  const sp_dec_layer_weights* low = nd > 1 ? w->dec_lower : nullptr;
+  s->n_dec = nd;
+  // layer 0's self-attention (the precomputed candidate rows)
+  const float* q0 = low ? low[0].Wq_s : w->Wq_s;
+  const float* k0 = low ? low[0].Wk_s : w->Wk_s;
+  const float* v0 = low ? low[0].Wv_s : w->Wv_s;
+  const float* o0 = low ? low[0].Wo_s : w->Wo_s;
+  s->pre_ln1_g = low ? low[0].ln1_g : w->ln1_g;
+  s->pre_ln1_b = low ? low[0].ln1_b : w->ln1_b;
+  const int r1 = 2 * nd;  // row blocks of h in Wcat1
   float *Wcat1 = nullptr, *Wcat2 = nullptr;
-  cudaError_t e = cudaMalloc(&Wcat1, (size_t)2 * h * D * sizeof(float));
+  cudaError_t e = cudaMalloc(&Wcat1, (size_t)r1 * h * D * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&Wcat2, (size_t)3 * h * h * sizeof(float));
-  if (e == cudaSuccess) e = cudaMalloc(&s->P1s, (size_t)2 * h * 6 * D * sizeof(uint16_t));
+  if (e == cudaSuccess) e = cudaMalloc(&s->P1s, (size_t)r1 * h * 6 * D * sizeof(uint16_t));
   if (e == cudaSuccess) e = cudaMalloc(&s->P2s, (size_t)3 * h * 6 * h * sizeof(uint16_t));
+  if (e == cudaSuccess && nd > 1) e = cudaMalloc(&s->Wf, (size_t)(nd - 1) * 3 * h * h * sizeof(float));
+  if (e == cudaSuccess && nd > 1) e = cudaMalloc(&s->dec_dev, (size_t)nd * sizeof(DecLayerDev));
   const float rs = 1.0f / std::sqrt((float)h);
   if (e == cudaSuccess) e = cudaMemcpy2D(Wcat1, D * sizeof(float), w->W_in, D * sizeof(float), D * sizeof(float), h, cudaMemcpyDeviceToDevice);
   // Wq_p^T Wk_p / sqrt(h): (i, j) = sum_k Wq_p[k, i] Wk_p[k, j]
   if (e == cudaSuccess) e = fold_matmul(w->Wq_p, 1, h, w->Wk_p, D, 1, Wcat1 + (size_t)h * D, D, h, D, h, rs, 0);
-  // Wq_s / sqrt(h), as Wq_s times the identity through the same fold kernel
+  // the layers before the last: Wq_c^T Wk_c / sqrt(h) and Wo_c Wv_c
+  for (int l = 0; e == cudaSuccess && l + 1 < nd; ++l) {
+    e = fold_matmul(low[l].Wq_c, 1, h, low[l].Wk_c, D, 1, Wcat1 + (size_t)(2 + 2 * l) * h * D, D, h, D, h, rs, 0);
+    if (e == cudaSuccess)
+      e = fold_matmul(low[l].Wo_c, h, 1, low[l].Wv_c, D, 1, Wcat1 + (size_t)(3 + 2 * l) * h * D, D, h, D, h, 1.f, 0);
+  }
+  // Wq / sqrt(h), as Wq times the identity through the same fold kernel
   std::vector<float> eye;
   float* dI = nullptr;
   if (e == cudaSuccess) {
@@ -322,11 +357,36 @@ sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weigh
     e = cudaMalloc(&dI, (size_t)h * h * sizeof(float));
     if (e == cudaSuccess) e = cudaMemcpy(dI, eye.data(), eye.size() * sizeof(float), cudaMemcpyHostToDevice);
   }
-  if (e == cudaSuccess) e = fold_matmul(w->Wq_s, h, 1, dI, h, 1, Wcat2, h, h, h, h, rs, 0);
-  if (e == cudaSuccess) e = cudaMemcpy(Wcat2 + (size_t)h * h, w->Wk_s, (size_t)h * h * sizeof(float), cudaMemcpyDeviceToDevice);
-  // Wo_s Wv_s: (i, j) = sum_k Wo_s[i, k] Wv_s[k, j]
-  if (e == cudaSuccess) e = fold_matmul(w->Wo_s, h, 1, w->Wv_s, h, 1, Wcat2 + (size_t)2 * h * h, h, h, h, h, 1.f, 0);
-  if (e == cudaSuccess) e = split6_weights(Wcat1, 2 * h, D, s->P1s, 0);
+  // [Wq / sqrt(h); Wk; Wo Wv] of one self-attention into dst [3h, h]
+  auto fold_self = [&](const float* Wq, const float* Wk, const float* Wv, const float* Wo, float* dst) {
+    cudaError_t r = fold_matmul(Wq, h, 1, dI, h, 1, dst, h, h, h, h, rs, 0);
+    if (r == cudaSuccess) r = cudaMemcpy(dst + (size_t)h * h, Wk, (size_t)h * h * sizeof(float), cudaMemcpyDeviceToDevice);
+    // Wo Wv: (i, j) = sum_k Wo[i, k] Wv[k, j]
+    if (r == cudaSuccess) r = fold_matmul(Wo, h, 1, Wv, h, 1, dst + (size_t)2 * h * h, h, h, h, h, 1.f, 0);
+    return r;
+  };
+  if (e == cudaSuccess) e = fold_self(q0, k0, v0, o0, Wcat2);
+  std::vector<DecLayerDev> dd(nd);
+  for (int l = 0; e == cudaSuccess && l < nd; ++l) {
+    DecLayerDev& L = dd[l];
+    memset(&L, 0, sizeof(L));
+    const bool last = l == nd - 1;
+    if (l >= 1) {
+      L.Wf = s->Wf + (size_t)(l - 1) * 3 * h * h;
+      e = last ? fold_self(w->Wq_s, w->Wk_s, w->Wv_s, w->Wo_s, const_cast<float*>(L.Wf))
+               : fold_self(low[l].Wq_s, low[l].Wk_s, low[l].Wv_s, low[l].Wo_s, const_cast<float*>(L.Wf));
+      L.ln1_g = last ? w->ln1_g : low[l].ln1_g;
+      L.ln1_b = last ? w->ln1_b : low[l].ln1_b;
+    }
+    if (!last) {
+      L.ln2_g = low[l].ln2_g; L.ln2_b = low[l].ln2_b;
+      L.ln3_g = low[l].ln3_g; L.ln3_b = low[l].ln3_b;
+      L.W1 = static_cast<const __nv_bfloat16*>(low[l].W1);
+      L.W2 = static_cast<const __nv_bfloat16*>(low[l].W2);
+    }
+  }
+  if (e == cudaSuccess && nd > 1) e = cudaMemcpy(s->dec_dev, dd.data(), nd * sizeof(DecLayerDev), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = split6_weights(Wcat1, r1 * h, D, s->P1s, 0);
   if (e == cudaSuccess) e = split6_weights(Wcat2, 3 * h, h, s->P2s, 0);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (dI) cudaFree(dI);
@@ -337,7 +397,7 @@ sp_status sp_selector_create(const sp_selector_cfg* cfg, const sp_selector_weigh
     return cuda_fail(e, "sp_selector_create (fold)");
   }
   std::string msg;
-  bool ok = make_gemm_b(&s->P1, s->P1s, 2 * h, 6 * D, &msg) && make_gemm_b(&s->P2, s->P2s, 3 * h, 6 * h, &msg);
+  bool ok = make_gemm_b(&s->P1, s->P1s, r1 * h, 6 * D, &msg) && make_gemm_b(&s->P2, s->P2s, 3 * h, 6 * h, &msg);
   if (ok && c.n_enc_layers > 0) {
     ok = make_gemm_b(&s->Wp, w->W_p, D, c.D_text, &msg);
     for (int i = 0; ok && i < c.n_enc_layers; ++i) {
@@ -359,6 +419,8 @@ void sp_selector_destroy(sp_selector* s) {
   if (!s) return;
   if (s->P1s) cudaFree(s->P1s);
   if (s->P2s) cudaFree(s->P2s);
+  if (s->Wf) cudaFree(s->Wf);
+  if (s->dec_dev) cudaFree(s->dec_dev);
   delete s;
 }
 
@@ -366,7 +428,7 @@ namespace {
 
 struct SelPlan {
   BatchDesc bd;
-  int E = 0, nvis = 0, ntxt = 0, T_enc = 0, max_enc = 0, rows = 0;
+  int E = 0, nvis = 0, ntxt = 0, T_enc = 0, max_enc = 0, rows = 0, k_max = 0;
   bool encoder = false;
 };
 
@@ -378,6 +440,7 @@ sp_status plan_select(const sp_selector* s, const sp_select_in* in, SelPlan* p) 
   if (in->g < 1 || in->g > 16) return fail(SP_ERR_SHAPE, "g must be in 1..16");
   if (in->k_max < 1 || in->k_max > SP_MAX_KMAX) return fail(SP_ERR_SHAPE, "k_max must be in 1..SP_MAX_KMAX");
   p->E = p->bd.ep_off[in->B];
+  p->k_max = in->k_max;
   p->nvis = p->bd.vis_off[in->B];
   p->ntxt = p->bd.txt_off[in->B];
   p->rows = p->nvis + 2;
@@ -408,16 +471,18 @@ size_t select_ws(const sp_selector* s, const SelPlan& p, const sp_select_out* ou
     R = cv.take<float>((size_t)p.T_enc * D);
   }
   Mall = cv.take<float>((size_t)p.rows * D);
-  ZK = cv.take<float>((size_t)p.rows * 2 * h);
+  ZK = cv.take<float>((size_t)p.rows * 2 * s->n_dec * h);
   XL = cv.take<float>((size_t)p.rows * h);
   QKVs = cv.take<float>((size_t)p.rows * 3 * h);
   void* Asp = cv.take<uint16_t>((size_t)p.rows * 3 * std::max(D, h));  // split operand of the precompute GEMMs
   int* order = (out && out->order) ? nullptr : cv.take<int>((size_t)p.E * SP_MAX_KMAX);
   int* epc = (out && out->ep_count) ? nullptr : cv.take<int>((size_t)p.E);
+  // self-attention rows of decoder layers >= 1, per episode and history position
+  float* dcache = s->n_dec > 1 ? cv.take<float>((size_t)p.E * (s->n_dec - 1) * (p.k_max + 1) * 2 * h) : nullptr;
   if (parts) {
     parts[0] = P; parts[1] = R; parts[2] = Abf; parts[3] = QKV; parts[4] = O; parts[5] = F1;
     parts[6] = enc_cu; parts[7] = Mall; parts[8] = ZK; parts[9] = XL; parts[10] = QKVs;
-    parts[11] = order; parts[12] = epc; parts[13] = gsk; parts[14] = Asp;
+    parts[11] = order; parts[12] = epc; parts[13] = gsk; parts[14] = Asp; parts[15] = dcache;
   }
   return cv.off;
 }
@@ -492,6 +557,9 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   SelPlan p;
   sp_status rs = plan_select(s, in, &p);
   if (rs != SP_OK) return rs;
+  if (s->n_dec > 1 && (in->g != 1 || tr))
+    return fail(SP_ERR_UNSUPPORTED, "sp_select: a decoder of %d layers takes g = 1 (and no training aggregates)",
+                s->n_dec);
   if (tr) {
     if (!tr->score || !tr->kbar || (reinterpret_cast<uintptr_t>(tr->score) & 3) ||
         (reinterpret_cast<uintptr_t>(tr->kbar) & 3))
@@ -519,7 +587,7 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   }
   if (out->k_cap < need_cap) return fail(SP_ERR_SHAPE, "sp_select: k_cap %d < largest possible count %d", out->k_cap, need_cap);
   Carve cv(ws);
-  void* parts[15];
+  void* parts[16];
   const size_t need = select_ws(s, p, out, cv, parts) + 256;
   if (!ws || ws_bytes < need) return fail(SP_ERR_WORKSPACE, "sp_select: workspace %zu < %zu bytes", ws_bytes, need);
   if (!al16(ws)) return fail(SP_ERR_ALIGN, "sp_select: workspace must be 16-byte aligned");
@@ -560,11 +628,12 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
     GemmEpi e1;
     e1.kind = EPI_F32;
     e1.out = ZK;
-    e1.ldo = 2 * h;
+    e1.ldo = 2 * s->n_dec * h;
     const GemmASplit a1 = split3_a_map(D), a2 = split3_a_map(h);
     SP_CUDA(split3_bf16(Mall, D, p.rows, D, Asp, st), "precompute split 1");
-    SP_CUDA(gemm_bf16(t1, p.rows, nullptr, s->P1, 2 * h, e1, err, st, nullptr, &a1), "precompute 1");
-    SP_CUDA(layernorm_f32(ZK, 2 * h, s->w.ln1_g, s->w.ln1_b, XL, nullptr, h, p.rows, h, s->cfg.ln_eps, 1.f, st), "ln1");
+    SP_CUDA(gemm_bf16(t1, p.rows, nullptr, s->P1, 2 * s->n_dec * h, e1, err, st, nullptr, &a1), "precompute 1");
+    SP_CUDA(layernorm_f32(ZK, 2 * s->n_dec * h, s->pre_ln1_g, s->pre_ln1_b, XL, nullptr, h, p.rows, h, s->cfg.ln_eps,
+                          1.f, st), "ln1");
     GemmEpi e2;
     e2.kind = EPI_F32;
     e2.out = QKVs;
@@ -574,8 +643,8 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   }
 
   SelectArgs a;
-  a.Z = ZK; a.ldz = 2 * h;
-  a.KT = ZK + h; a.ldkt = 2 * h;
+  a.Z = ZK; a.ldz = 2 * s->n_dec * h;
+  a.KT = ZK + h; a.ldkt = 2 * s->n_dec * h;
   a.QS = QKVs; a.ldqs = 3 * h;
   a.KS = QKVs + h; a.ldks = 3 * h;
   a.VT = QKVs + 2 * h; a.ldvt = 3 * h;
@@ -593,9 +662,14 @@ static sp_status select_impl(const sp_selector* s, const sp_select_in* in, const
   a.kbar = tr ? tr->kbar : nullptr;
   a.inv_tau = tr ? 1.f / tr->tau : 1.f;
   a.beta = tr ? tr->beta : 1.f;
+  a.n_dec = s->n_dec;
+  a.dec = s->dec_dev;
+  a.KC = ZK + 2 * h;
+  a.dcache = static_cast<float*>(parts[15]);
+  a.dcache_ep = (size_t)(s->n_dec - 1) * (in->k_max + 1) * 2 * h;
   bool keys_smem = true;
   size_t smem = 0;
-  const int C = select_cluster_size(p.bd, h, in->k_max, &keys_smem, &smem);
+  const int C = select_cluster_size(p.bd, h, in->k_max, &keys_smem, &smem, s->n_dec > 1);
   SP_CUDA(select_launch(p.bd, p.E, a, C, keys_smem, smem, st), "selection");
   SP_CUDA(restore_launch(p.bd, a.order, a.ep_count, in->k_max, out->idx, out->k_cap, out->count, err, st), "restore");
   return SP_OK;

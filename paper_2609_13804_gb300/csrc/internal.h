@@ -1,6 +1,7 @@
 // Host-side interfaces between the translation units of libstepprune.
 #pragma once
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -159,6 +160,18 @@ cudaError_t attention_varlen(const void* qkv, void* out, const int* cu_seqlens, 
                              int* err, cudaStream_t st);
 
 // ------------------------------------------------------------- selection
+// A pointer-decoder layer's runtime weights (decoders of several layers).
+// Layer 0's self-attention rows and every layer's folded cross-attention rows
+// are precomputed per candidate; what depends on the history is applied here.
+struct DecLayerDev {
+  const float* Wf;                       // [3h, h]: [Wq_s / sqrt h; Wk_s; Wo_s Wv_s] (layers >= 1)
+  const float* ln1_g; const float* ln1_b;  // (layers >= 1)
+  const float* ln2_g; const float* ln2_b;  // before the cross-attention (layers before the last)
+  const float* ln3_g; const float* ln3_b;  // before the FFN (layers before the last)
+  const __nv_bfloat16* W1;               // [4h, h]
+  const __nv_bfloat16* W2;               // [h, 4h]
+};
+
 struct SelectArgs {
   const float* Z;  int ldz;     // decoder tokens y = W_in m
   const float* KT; int ldkt;    // folded pointer keys
@@ -178,9 +191,16 @@ struct SelectArgs {
   float* kbar;     // [n_episodes] Eq. 7
   float inv_tau;   // 1 / pointer temperature
   float beta;      // discount of Eq. 6
+  // pointer decoders of n_dec > 1 layers (g = 1)
+  int n_dec;
+  const DecLayerDev* dec;   // [n_dec] device array
+  const float* KC;          // layer l's folded cross-attention keys at KC + 2 l h, values at + h (row stride ldz)
+  float* dcache;            // self-attention rows (k | Wo Wv x) of layers 1..n_dec-1 per episode and position
+  size_t dcache_ep;         // floats per episode: (n_dec - 1) (k_max + 1) 2h
 };
 
-int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes);
+int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes,
+                        bool multi = false);
 cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs& a,
                           int cluster, bool keys_in_smem, size_t smem_bytes, cudaStream_t st);
 // 3-D mRoPE (mrope.cu)

@@ -47,14 +47,15 @@ constexpr int GMAX = 16;  // largest g; lists hold g + 1 entries
 
 struct SelSmem {
   size_t kt, lgp, stopkt, wpart_o, wpart_ml, all_o, all_ml, wtop_v, wtop_i, all_tv, all_ti, xp, taken, hist, misc,
-      wsm, all_sm, score, total;
+      wsm, all_sm, score, mx, ma, mc, mn, v3, hb, xo, total;
 };
 
 __host__ __device__ inline size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
 
 // Shared-memory layout.  The all_* slots receive, per round parity, one entry
 // per CTA of the cluster, written remotely by that CTA (push exchange).
-__host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C, bool keys_in_smem) {
+__host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C, bool keys_in_smem,
+                                              bool multi = false) {
   SelSmem L;
   size_t o = 0;
   // keys in shared memory: dims-major, (n_loc + 1) columns (the last one is
@@ -79,6 +80,17 @@ __host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C
   L.wsm = o;      o += al16((size_t)NW * 2 * 4);
   L.all_sm = o;   o += al16((size_t)2 * C * 2 * 4);
   L.score = o;    o += al16((size_t)n_loc * 4);
+  // decoders of several layers: the new position's residual / attention /
+  // cross-attention outputs and a normalised input (h each), and the pushed
+  // matrix-vector products (3h q|k|v, 4h FFN hidden, h FFN output)
+  const size_t hm = multi ? (size_t)h : 0;
+  L.mx = o;       o += al16(hm * 4);
+  L.ma = o;       o += al16(hm * 4);
+  L.mc = o;       o += al16(hm * 4);
+  L.mn = o;       o += al16(hm * 4);
+  L.v3 = o;       o += al16(3 * hm * 4);
+  L.hb = o;       o += al16(4 * hm * 4);
+  L.xo = o;       o += al16(hm * 4);
   L.total = o;
   return L;
 }
@@ -220,7 +232,7 @@ SP_DEVINL void warp_merge_lists(const float* vin, const int* iin, int tot, int p
 // softmax partials (max, sum) of the round's available logits with STOP's in
 // rank order, adds A_t beta^t p_t(j) to the scores of its own candidates and
 // advances A_t and the soft count identically.
-template <int HV, int GL, bool TRAIN>
+template <int HV, int GL, bool TRAIN, bool MULTI>
 __global__ void __launch_bounds__(NT, 1)
 select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in_smem, int tm_cols) {
   constexpr int P = (16 / HV) > 0 ? 16 / HV : 1;
@@ -251,7 +263,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
   const int nl = max(0, min(j0 + n_loc, n_e) - j0);
 
   extern __shared__ __align__(16) uint8_t sm[];
-  const SelSmem L = sel_layout(h, n_loc_max, k_max, C, keys_in_smem != 0);
+  const SelSmem L = sel_layout(h, n_loc_max, k_max, C, keys_in_smem != 0, MULTI);
   float* kt_s = reinterpret_cast<float*>(sm + L.kt);
   float* lgp = reinterpret_cast<float*>(sm + L.lgp);
   float* stopkt = reinterpret_cast<float*>(sm + L.stopkt);
@@ -339,7 +351,283 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
 #pragma unroll
     for (int k = 0; k < HV; ++k) q[k] = __ldg(qrow + lane + 32 * k);
   };
-  load_last(a.start_row);
+  if (!MULTI) load_last(a.start_row);
+
+  // ---- decoders of several layers (MULTI): the layers before the last run on
+  //      the new history position at the start of every round.  Every vector
+  //      below is identical in all CTAs of the cluster (each product row is
+  //      computed by one CTA and pushed to all; merges go in rank order).
+  float* mx = reinterpret_cast<float*>(sm + L.mx);  // residual of the new position
+  float* ma = reinterpret_cast<float*>(sm + L.ma);  // after self-attention
+  float* mc = reinterpret_cast<float*>(sm + L.mc);  // after cross-attention
+  float* mn = reinterpret_cast<float*>(sm + L.mn);  // a normalised input
+  float* v3 = reinterpret_cast<float*>(sm + L.v3);  // pushed q | k | Wo Wv x
+  float* hb = reinterpret_cast<float*>(sm + L.hb);  // pushed FFN hidden
+  float* xo = reinterpret_cast<float*>(sm + L.xo);  // pushed FFN output
+  const int ldc = 2 * h;
+  float* ecache = MULTI ? a.dcache + (size_t)e * a.dcache_ep : nullptr;
+  auto lcache = [&](int l) { return ecache + (size_t)(l - 1) * (k_max + 1) * ldc; };  // layers >= 1
+
+  // LayerNorm of a shared h-vector into dst (same arithmetic in every CTA)
+  auto ln_vec = [&](const float* src, const float* g, const float* bb, float* dst) {
+    float v[DPT];
+    float mom[2] = {0.f, 0.f};
+    const float sh = src[0];
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const int i = el(d);
+      v[d] = i < h ? src[i] : 0.f;
+      if (i < h) {
+        const float c = v[d] - sh;
+        mom[0] += c;
+        mom[1] += c * c;
+      }
+    }
+    block_sum_n<2>(mom, red);
+    const float m1 = mom[0] / (float)h;
+    const float mean = sh + m1;
+    const float rstd = rsqrtf(fmaxf(mom[1] / (float)h - m1 * m1, 0.f) + a.ln_eps);
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const int i = el(d);
+      if (i < h) dst[i] = (v[d] - mean) * rstd * (g ? __ldg(g + i) : 1.f) + (bb ? __ldg(bb + i) : 0.f);
+    }
+    __syncthreads();
+  };
+  // rows [rank R / C, +R / C) of W [R, h] (fp32) times the shared vector x;
+  // half a warp per row, two rows per half-warp at a time; each result is
+  // pushed into dst[row] of every CTA
+  auto matvec_f32_push = [&](const float* W, int R, const float* x, float* dst) {
+    const int Rc = R / C, r0 = rank * Rc, hl = lane & 15, hw = lane >> 4;
+    const int cu = h / 4;  // float4 chunks per row
+    const float4* x4 = reinterpret_cast<const float4*>(x);
+    for (int rb = (warp * 2 + hw) * 2; rb < Rc; rb += NW * 4) {
+      const float4* wa = reinterpret_cast<const float4*>(W + (size_t)(r0 + rb) * h);
+      const float4* wb = reinterpret_cast<const float4*>(W + (size_t)(r0 + min(rb + 1, Rc - 1)) * h);
+      float sv[2] = {0.f, 0.f};
+#pragma unroll 4
+      for (int u = hl; u < cu; u += 16) {
+        const float4 xv = x4[u];
+        sv[0] += dot4(xv, __ldg(wa + u));
+        sv[1] += dot4(xv, __ldg(wb + u));
+      }
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) {
+        sv[0] += __shfl_xor_sync(0xffffffffu, sv[0], o);
+        sv[1] += __shfl_xor_sync(0xffffffffu, sv[1], o);
+      }
+      if (hl < C) {
+        *cluster.map_shared_rank(dst + r0 + rb, hl) = sv[0];
+        if (rb + 1 < Rc) *cluster.map_shared_rank(dst + r0 + rb + 1, hl) = sv[1];
+      }
+    }
+  };
+  // the same for W [R, K] in bf16, optionally through the exact GELU
+  auto matvec_bf16_push = [&](const __nv_bfloat16* W, int R, int K, const float* x, float* dst, bool act) {
+    const int Rc = R / C, r0 = rank * Rc, hl = lane & 15, hw = lane >> 4;
+    const int cu = K / 8;  // 8-element chunks per row
+    const float4* x4 = reinterpret_cast<const float4*>(x);
+    for (int rb = (warp * 2 + hw) * 2; rb < Rc; rb += NW * 4) {
+      const uint4* wa = reinterpret_cast<const uint4*>(W + (size_t)(r0 + rb) * K);
+      const uint4* wb = reinterpret_cast<const uint4*>(W + (size_t)(r0 + min(rb + 1, Rc - 1)) * K);
+      float sv[2] = {0.f, 0.f};
+#pragma unroll 4
+      for (int u = hl; u < cu; u += 16) {
+        const float4 xa = x4[2 * u], xb = x4[2 * u + 1];
+        const uint4 pa = __ldg(wa + u), pb = __ldg(wb + u);
+        const uint32_t qa[4] = {pa.x, pa.y, pa.z, pa.w}, qb[4] = {pb.x, pb.y, pb.z, pb.w};
+        const float xs[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float2 fa = unpack_bf16x2(qa[k]), fb = unpack_bf16x2(qb[k]);
+          sv[0] += fa.x * xs[2 * k] + fa.y * xs[2 * k + 1];
+          sv[1] += fb.x * xs[2 * k] + fb.y * xs[2 * k + 1];
+        }
+      }
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) {
+        sv[0] += __shfl_xor_sync(0xffffffffu, sv[0], o);
+        sv[1] += __shfl_xor_sync(0xffffffffu, sv[1], o);
+      }
+      if (act) {
+        sv[0] = gelu_erf(sv[0]);
+        sv[1] = gelu_erf(sv[1]);
+      }
+      if (hl < C) {
+        *cluster.map_shared_rank(dst + r0 + rb, hl) = sv[0];
+        if (rb + 1 < Rc) *cluster.map_shared_rank(dst + r0 + rb + 1, hl) = sv[1];
+      }
+    }
+  };
+
+  // this CTA's attention partial (max, sum, weighted values) from its warps'
+  // partials, pushed into slot `slot` of every CTA (as in step 1 below)
+  auto push_partial = [&](float4 (&o_w)[HV], float m_w, float l_w, int slot) {
+#pragma unroll
+    for (int k = 0; k < HV; ++k) reinterpret_cast<float4*>(wpart_o + warp * h)[lane + 32 * k] = o_w[k];
+    if (lane == 0) {
+      wpart_ml[warp * 2 + 0] = m_w;
+      wpart_ml[warp * 2 + 1] = l_w;
+    }
+    __syncthreads();
+    const float mwl = lane < NW ? wpart_ml[lane * 2] : -INFINITY;
+    const float lwl = lane < NW ? wpart_ml[lane * 2 + 1] : 0.f;
+    const float m_c = fkey_inv(__reduce_max_sync(0xffffffffu, fkey(mwl)));
+    const float cwl = (mwl == -INFINITY) ? 0.f : __expf(mwl - m_c);
+    const float l_c = warp_sum(cwl * lwl);
+    float cw[NW];
+#pragma unroll
+    for (int w = 0; w < NW; ++w) cw[w] = __shfl_sync(0xffffffffu, cwl, w);
+    float* sl = all_o + ((size_t)slot * C + rank) * h;
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const int i = el(d);
+      if (i >= h) continue;
+      float acc = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) acc += cw[w] * wpart_o[w * h + i];
+      for (int r = 0; r < C; ++r) *cluster.map_shared_rank(sl + i, r) = acc;
+    }
+    if (tid < C) {
+      float* ml = cluster.map_shared_rank(all_ml + ((size_t)slot * C + rank) * 2, tid);
+      ml[0] = m_c;
+      ml[1] = l_c;
+    }
+  };
+  // o / l of the C partials in slot `slot`, merged in rank order (DPT per thread)
+  auto merge_slot = [&](int slot, float (&out)[DPT]) {
+    const float mrl = lane < C ? all_ml[(slot * C + lane) * 2] : -INFINITY;
+    const float lrl = lane < C ? all_ml[(slot * C + lane) * 2 + 1] : 0.f;
+    const float m = fkey_inv(__reduce_max_sync(0xffffffffu, fkey(mrl)));
+    const float wrl = (mrl == -INFINITY) ? 0.f : __expf(mrl - m);
+    const float inv = 1.f / warp_sum(wrl * lrl);
+    float wr[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) wr[r] = __shfl_sync(0xffffffffu, wrl, r);
+#pragma unroll
+    for (int d = 0; d < DPT; ++d) {
+      const int i = el(d);
+      out[d] = 0.f;
+      if (i >= h) continue;
+      float o = 0.f;
+#pragma unroll
+      for (int r = 0; r < 16; ++r)
+        if (r < C) o += wr[r] * all_o[((size_t)slot * C + r) * h + i];
+      out[d] = o * inv;
+    }
+  };
+  // online-softmax update of a warp's partial with P scored rows
+  auto absorb = [&](const float (&sc)[P], const float4 (&vr)[P][HV], int valid, float& m_w, float& l_w,
+                    float4 (&o_w)[HV]) {
+#pragma unroll
+    for (int pp = 0; pp < P; ++pp) {
+      if (pp < valid) {
+        const float sv = sc[pp];
+        const float mn2 = fmaxf(m_w, sv);
+        const float cw = (m_w == -INFINITY) ? 0.f : __expf(m_w - mn2);
+        const float ps = __expf(sv - mn2);
+        l_w = l_w * cw + ps;
+#pragma unroll
+        for (int k = 0; k < HV; ++k) {
+          o_w[k].x = o_w[k].x * cw + ps * vr[pp][k].x;
+          o_w[k].y = o_w[k].y * cw + ps * vr[pp][k].y;
+          o_w[k].z = o_w[k].z * cw + ps * vr[pp][k].z;
+          o_w[k].w = o_w[k].w * cw + ps * vr[pp][k].w;
+        }
+        m_w = mn2;
+      }
+    }
+  };
+  // layer l's causal self-attention of the new position (query qv) over this
+  // CTA's history positions rank, rank + C, ... < t; layer 0 reads the
+  // candidates' precomputed rows, deeper layers the episode's cache
+  auto self_attn_partial = [&](int l, const float4 (&qv)[HV], int t_len, int slot) {
+    const int np2 = (rank < t_len) ? (t_len - 1 - rank) / C + 1 : 0;
+    float m_w = -INFINITY, l_w = 0.f;
+    float4 o_w[HV];
+#pragma unroll
+    for (int k = 0; k < HV; ++k) o_w[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k0 = warp * P; k0 < np2; k0 += NW * P) {
+      float4 kr[P][HV], vr[P][HV];
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        if (k0 + pp < np2) {
+          const int pos = rank + (k0 + pp) * C;
+          if (l == 0) {
+            const int row = hist[pos];
+            const float4* ks = reinterpret_cast<const float4*>(a.KS + (size_t)row * a.ldks);
+            const float4* vt = reinterpret_cast<const float4*>(a.VT + (size_t)row * a.ldvt);
+#pragma unroll
+            for (int k = 0; k < HV; ++k) {
+              kr[pp][k] = __ldg(ks + lane + 32 * k);
+              vr[pp][k] = __ldg(vt + lane + 32 * k);
+            }
+          } else {
+            const float4* cr = reinterpret_cast<const float4*>(lcache(l) + (size_t)pos * ldc);
+#pragma unroll
+            for (int k = 0; k < HV; ++k) {
+              kr[pp][k] = __ldcg(cr + lane + 32 * k);
+              vr[pp][k] = __ldcg(cr + h / 4 + lane + 32 * k);
+            }
+          }
+        }
+      }
+      float sc[P];
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        sc[pp] = 0.f;
+        if (k0 + pp < np2) {
+#pragma unroll
+          for (int k = 0; k < HV; ++k) sc[pp] += dot4(qv[k], kr[pp][k]);
+        }
+      }
+      warp_sum_n<P>(sc);
+      absorb(sc, vr, np2 - k0, m_w, l_w, o_w);
+    }
+    push_partial(o_w, m_w, l_w, slot);
+  };
+  // layer l's cross-attention of the normalised input mn over every row of the
+  // episode's memory (this CTA's candidate slice; rank 0 adds the STOP row),
+  // with the folded keys (Wq_c^T Wk_c m / sqrt h) and values (Wo_c Wv_c m)
+  auto cross_partial = [&](int l, int slot) {
+    float4 xv[HV];
+#pragma unroll
+    for (int k = 0; k < HV; ++k) xv[k] = reinterpret_cast<const float4*>(mn)[lane + 32 * k];
+    const float* KCl = a.KC + (size_t)2 * l * h;
+    const int ncand = nl + (rank == 0 ? 1 : 0);
+    float m_w = -INFINITY, l_w = 0.f;
+    float4 o_w[HV];
+#pragma unroll
+    for (int k = 0; k < HV; ++k) o_w[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k0 = warp * P; k0 < ncand; k0 += NW * P) {
+      float4 kr[P][HV], vr[P][HV];
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        if (k0 + pp < ncand) {
+          const int jj = k0 + pp;
+          const int row = jj < nl ? row0 + j0 + jj : a.stop_row;
+          const float4* kc = reinterpret_cast<const float4*>(KCl + (size_t)row * a.ldz);
+#pragma unroll
+          for (int k = 0; k < HV; ++k) {
+            kr[pp][k] = __ldg(kc + lane + 32 * k);
+            vr[pp][k] = __ldg(kc + h / 4 + lane + 32 * k);
+          }
+        }
+      }
+      float sc[P];
+#pragma unroll
+      for (int pp = 0; pp < P; ++pp) {
+        sc[pp] = 0.f;
+        if (k0 + pp < ncand) {
+#pragma unroll
+          for (int k = 0; k < HV; ++k) sc[pp] += dot4(xv[k], kr[pp][k]);
+        }
+      }
+      warp_sum_n<P>(sc);
+      absorb(sc, vr, ncand - k0, m_w, l_w, o_w);
+    }
+    push_partial(o_w, m_w, l_w, slot);
+  };
 
   float alive = 1.f, disc = a.beta, kbar_acc = 0.f;  // A_t, beta^t, Eq. 7 (TRAIN)
   int nsel = 0, round = 0;
@@ -355,6 +643,81 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     }
     const int buf = round & 1;
     const int t = nsel + 1;
+
+    if constexpr (MULTI) {
+      // ---- 0. the new history position (candidate row hist[t - 1]) through
+      //      the layers before the last, then the last layer's q | k | Wo Wv x
+      //      for it (exchange slots: self-attention 0, cross-attention 1; the
+      //      pushed products are read before the next barrier and rewritten only
+      //      after several more)
+      const int p = t - 1;
+      const int rn = hist[p];
+      const int owner = p % C;  // the CTA whose share of positions holds p
+      for (int i = tid; i < h; i += NT) mx[i] = __ldg(a.Z + (size_t)rn * a.ldz + i);
+      __syncthreads();
+      for (int l = 0; l + 1 < a.n_dec; ++l) {
+        const DecLayerDev dl = a.dec[l];
+        float4 qv[HV];
+        if (l == 0) {
+          const float4* qr = reinterpret_cast<const float4*>(a.QS + (size_t)rn * a.ldqs);
+#pragma unroll
+          for (int k = 0; k < HV; ++k) qv[k] = __ldg(qr + lane + 32 * k);
+        } else {
+          ln_vec(mx, dl.ln1_g, dl.ln1_b, mn);
+          matvec_f32_push(dl.Wf, 3 * h, mn, v3);
+          cluster.sync();
+#pragma unroll
+          for (int k = 0; k < HV; ++k) qv[k] = reinterpret_cast<const float4*>(v3)[lane + 32 * k];
+          if (rank == owner) {
+            float* dst = lcache(l) + (size_t)p * ldc;
+            for (int i = tid; i < 2 * h; i += NT) dst[i] = v3[h + i];
+          }
+          __syncthreads();
+        }
+        self_attn_partial(l, qv, t, 0);
+        cluster.sync();
+        {
+          float o[DPT];
+          merge_slot(0, o);
+#pragma unroll
+          for (int d = 0; d < DPT; ++d)
+            if (el(d) < h) ma[el(d)] = mx[el(d)] + o[d];
+        }
+        __syncthreads();
+        ln_vec(ma, dl.ln2_g, dl.ln2_b, mn);
+        cross_partial(l, 1);
+        cluster.sync();
+        {
+          float o[DPT];
+          merge_slot(1, o);
+#pragma unroll
+          for (int d = 0; d < DPT; ++d)
+            if (el(d) < h) mc[el(d)] = ma[el(d)] + o[d];
+        }
+        __syncthreads();
+        ln_vec(mc, dl.ln3_g, dl.ln3_b, mn);
+        matvec_bf16_push(dl.W1, 4 * h, h, mn, hb, true);
+        cluster.sync();
+        matvec_bf16_push(dl.W2, h, 4 * h, hb, xo, false);
+        cluster.sync();
+        for (int i = tid; i < h; i += NT) mx[i] = mc[i] + xo[i];
+        __syncthreads();
+      }
+      const DecLayerDev dl = a.dec[a.n_dec - 1];
+      ln_vec(mx, dl.ln1_g, dl.ln1_b, mn);
+      matvec_f32_push(dl.Wf, 3 * h, mn, v3);
+      cluster.sync();
+#pragma unroll
+      for (int k = 0; k < HV; ++k) q[k] = reinterpret_cast<const float4*>(v3)[lane + 32 * k];
+      shift = mx[0];
+#pragma unroll
+      for (int d = 0; d < DPT; ++d) zr[d] = (el(d) < h) ? mx[el(d)] : 0.f;
+      if (rank == owner) {
+        float* dst = lcache(a.n_dec - 1) + (size_t)p * ldc;
+        for (int i = tid; i < 2 * h; i += NT) dst[i] = v3[h + i];
+      }
+      __syncthreads();
+    }
 
     // ---- 1. partial causal self-attention of the last position (its query and
     //      residual rows were loaded at the end of the previous round); every
@@ -376,6 +739,15 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
             const uint32_t ta = tm_warp + (uint32_t)(o * 8 * HV);
             tmem_ld_f4<HV>(ta, kr[pp]);
             tmem_ld_f4<HV>(ta + 4 * HV, vr[pp]);
+          } else if (MULTI) {  // the last layer's rows of the episode cache, by position
+            const float4* cr =
+                reinterpret_cast<const float4*>(lcache(a.n_dec - 1) + (size_t)(rank + (k0 + pp) * C) * ldc);
+#pragma unroll
+            for (int k = 0; k < HV; ++k) {
+              kr[pp][k] = __ldcg(cr + lane + 32 * k);
+              vr[pp][k] = __ldcg(cr + h / 4 + lane + 32 * k);
+            }
+            fresh[pp] = o < ppw;
           } else {
             const int row = hist[rank + (k0 + pp) * C];
             const float4* ks = reinterpret_cast<const float4*>(a.KS + (size_t)row * a.ldks);
@@ -745,7 +1117,7 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     }
     {  // rows of the next round's last position
       const int jl = gtop_i[take - 1];
-      load_last((jl >= 0 && jl < n_e) ? row0 + jl : a.start_row);
+      if (!MULTI) load_last((jl >= 0 && jl < n_e) ? row0 + jl : a.start_row);
     }
     nsel += take;
     __syncthreads();
@@ -831,7 +1203,7 @@ restore_kernel(const BatchDesc bd, const int* __restrict__ order, const int* __r
 
 }  // namespace
 
-int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes) {
+int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_smem, size_t* smem_bytes, bool multi) {
   int n_max = 0;
   for (int b = 0; b < bd.B; ++b) {
     const int n = bd.vis_off[b + 1] - bd.vis_off[b];
@@ -840,7 +1212,7 @@ int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_sme
   const size_t budget = 225 * 1024;
   for (int C : {8, 16}) {
     const int n_loc = (n_max + C - 1) / C;
-    const size_t need = sel_layout(h, n_loc, k_max, C, true).total;
+    const size_t need = sel_layout(h, n_loc, k_max, C, true, multi).total;
     if (n_loc + 1 <= 128 && need <= budget) {  // the dims-major logits take <= 128 columns
       *keys_in_smem = true;
       *smem_bytes = need;
@@ -848,7 +1220,7 @@ int select_cluster_size(const BatchDesc& bd, int h, int k_max, bool* keys_in_sme
     }
   }
   *keys_in_smem = false;
-  *smem_bytes = sel_layout(h, (n_max + 15) / 16, k_max, 16, false).total;
+  *smem_bytes = sel_layout(h, (n_max + 15) / 16, k_max, 16, false, multi).total;
   return 16;
 }
 
@@ -861,16 +1233,20 @@ cudaError_t select_launch(const BatchDesc& bd, int n_episodes, const SelectArgs&
     n_max = std::max(n_max, bd.group_size > 0 ? std::min(bd.group_size, n) : n);
   }
   const int n_loc = (n_max + C - 1) / C;
-  const SelSmem L = sel_layout(a.h, n_loc, a.k_max, C, keys_in_smem);
+  const SelSmem L = sel_layout(a.h, n_loc, a.k_max, C, keys_in_smem, a.n_dec > 1);
   void (*kern)(const BatchDesc, const SelectArgs, int, int, int) = nullptr;
   const int gl = a.g + 1 <= 2 ? 2 : (a.g + 1 <= 6 ? 6 : 17);
   const bool train = a.score != nullptr;
   if (train && (a.g != 1 || !keys_in_smem || !a.kbar)) return cudaErrorInvalidValue;
-#define SP_SEL_CASE(HV_)                                                                             \
-  case HV_:                                                                                          \
-    kern = train ? select_kernel<HV_, 2, true>                                                       \
-                 : (gl == 2 ? select_kernel<HV_, 2, false>                                           \
-                            : (gl == 6 ? select_kernel<HV_, 6, false> : select_kernel<HV_, 17, false>)); \
+  const bool multi = a.n_dec > 1;
+  if (multi && (a.g != 1 || train || !a.dec || !a.dcache || !a.KC)) return cudaErrorInvalidValue;
+#define SP_SEL_CASE(HV_)                                                                                    \
+  case HV_:                                                                                                 \
+    kern = multi ? select_kernel<HV_, 2, false, true>                                                       \
+                 : train ? select_kernel<HV_, 2, true, false>                                               \
+                         : (gl == 2 ? select_kernel<HV_, 2, false, false>                                   \
+                                    : (gl == 6 ? select_kernel<HV_, 6, false, false>                        \
+                                               : select_kernel<HV_, 17, false, false>));                    \
     break;
   switch (a.h / 128) {
     SP_SEL_CASE(1)

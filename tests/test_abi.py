@@ -38,7 +38,9 @@ def test_library_exports_every_declared_symbol(L):
 
 def test_struct_sizes_match_header_layout():
     # pointer arrays sized by the header limits; a mismatch shifts every later field
-    assert C.sizeof(b.sp_selector_weights) == 8 * (3 + 8 * b.SP_MAX_ENC_LAYERS + 13)
+    assert C.sizeof(b.sp_selector_weights) == 8 * (3 + 8 * b.SP_MAX_ENC_LAYERS + 13 + 1)
+    assert C.sizeof(b.sp_selector_cfg) == 4 * 9
+    assert C.sizeof(b.sp_dec_layer_weights) == 8 * 16
     assert C.sizeof(b.sp_model_weights) == 8 * (6 * b.SP_MAX_LM_LAYERS + 3)
     assert C.sizeof(b.sp_select_in) == 4 + 4 + 8 * 6 + 4 * 3 + 4
     assert C.sizeof(b.sp_select_out) == 8 + 8 + 8 * 8
