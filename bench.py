@@ -15,6 +15,7 @@ Prints one JSON line (rank 0).  `value` is ms per batch over the whole job
 workload instead.
 """
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -501,6 +502,25 @@ def run_ours(args):
     gate_big_bytes = 3.0 * Xg.numel() * 2
     del Xg, Ng, Ag, Og
 
+    # ---- pointer decoders of one and of two layers on the same shapes (every
+    #      episode runs its 192 rounds: STOP disabled; memory H given)
+    Hm = B.dev_f32(S.make_memory(w), dev)
+    nostop = B.dev_f32(np.full(w.B, -1e30), dev)
+    deep = {}
+    for nd in (1, 2):
+        shp = dataclasses.replace(s, n_enc_layers=0, n_dec_layers=nd)
+        dsel = B.Selector(shp, S.make_selector_weights(dataclasses.replace(w, selector=shp)), dev)
+        dws = [None]
+
+        def run_deep():
+            r = B.sp_select(dsel, w.n_vis, w.n_txt, H=Hm, stop_bias=nostop, g=1, k_max=w.k_max, traces=False,
+                            ws=dws[0])
+            dws[0] = r["_ws"]
+
+        deep[nd] = timed(run_deep)
+        dsel.close()
+    del Hm
+
     # ---- end to end from host buffers (copies inside the timed region)
     Xh = X.cpu().pin_memory()
     Eh = E.cpu().pin_memory()
@@ -574,6 +594,10 @@ def run_ours(args):
                 "vp_gate_256_images_gbs": gate_big_bytes / (gate_big_ms * 1e-3) / 1e9,
                 "vp_gate_256_images_hbm_frac": gate_big_bytes / (gate_big_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
                 "note": "tau 1.0, beta 0.99, SoftTopK tau 0.05; the gate reads X and noise, writes the gated rows"},
+            "deep_decoder": {
+                "select_1_layer_ms": deep[1], "select_2_layers_ms": deep[2], "rounds": w.k_max,
+                "us_per_round_1_layer": 1e3 * deep[1] / w.k_max, "us_per_round_2_layers": 1e3 * deep[2] / w.k_max,
+                "note": "16 episodes x 192 rounds from a given memory H (precompute GEMMs included)"},
         }
         print(json.dumps(line), flush=True)
     if dist:
