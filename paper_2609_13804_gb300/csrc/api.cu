@@ -10,6 +10,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -169,6 +170,14 @@ void prof_end_launch(cudaStream_t st, int kind, double flops, double bytes) {
 }
 
 // ------------------------------------------------------------------ batches
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("SP_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
 
 bool fill_batch_desc(BatchDesc* d, int B, const int* n_vis, const int* n_txt, int group_size,
                      std::string* msg) {

@@ -76,6 +76,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   uint64_t* mma_done = bar + 15;  //     every MMA of the CTA complete
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bar + 16);
 
+  pdl_wait();  // programmatic launch: the previous kernel's outputs are visible from here
+  pdl_trigger();
   const int b = blockIdx.z, h = blockIdx.y;
   const int s0 = __ldg(cu + b);
   const int len = __ldg(cu + b + 1) - s0;
@@ -316,9 +318,8 @@ cudaError_t launch_attn_tc(const void* qkv, void* out, const int* cu, int B, int
       !encode_tmap_2d(&tkv, qkv, false, (uint64_t)rows_cap, (uint64_t)ld_qkv, 64, tca::BKV, nullptr))
     return cudaErrorInvalidValue;
   dim3 grid((max_len + tca::BQ - 1) / tca::BQ, Hq, B);
-  tca::attn_tc_kernel<DH><<<grid, tca::NTHR, C::SMEM, st>>>(tq, tkv, reinterpret_cast<__nv_bfloat16*>(out), cu, Hq,
-                                                           Hkv, Hq * DH, causal ? 1 : 0, scale_log2, err);
-  return cudaGetLastError();
+  return launch_pdl(tca::attn_tc_kernel<DH>, grid, dim3(tca::NTHR), C::SMEM, st, tq, tkv,
+                    reinterpret_cast<__nv_bfloat16*>(out), cu, Hq, Hkv, Hq * DH, causal ? 1 : 0, scale_log2, err);
 }
 
 cudaError_t attention_varlen(const void* qkv, void* out, const int* cu_seqlens, int B,

@@ -32,6 +32,8 @@ __global__ void __launch_bounds__(256) kv_store_kernel(const __nv_bfloat16* __re
                                                        const int* __restrict__ pos, int B, int T_cap,
                                                        __nv_bfloat16* __restrict__ kv_l, int S_cap, int* err) {
   __shared__ int s_cu[SP_MAX_BATCH + 1];
+  pdl_wait();
+  pdl_trigger();
   for (int i = threadIdx.x; i <= B; i += blockDim.x) s_cu[i] = __ldg(cu + i);
   __syncthreads();
   const int T = min(s_cu[B], T_cap);
@@ -177,11 +179,11 @@ cudaError_t kv_store(const void* qkv, const int* cu, const int* pos, int B, int 
   const int ld = (Hq + 2 * Hkv) * dh;
   const int grid = std::max(1, std::min((T_cap + 7) / 8, device_sm_count() * 8));
   prof_begin_launch(st);
-  kv_store_kernel<<<grid, 256, 0, st>>>(reinterpret_cast<const __nv_bfloat16*>(qkv), ld, Hq * dh, (Hq + Hkv) * dh,
-                                       Hkv * dh, cu, pos, B, T_cap, reinterpret_cast<__nv_bfloat16*>(kv_l), S_cap,
-                                       err);
+  const cudaError_t r = launch_pdl(kv_store_kernel, dim3(grid), dim3(256), 0, st,
+                                   reinterpret_cast<const __nv_bfloat16*>(qkv), ld, Hq * dh, (Hq + Hkv) * dh, Hkv * dh,
+                                   cu, pos, B, T_cap, reinterpret_cast<__nv_bfloat16*>(kv_l), S_cap, err);
   prof_end_launch(st, SP_K_MISC, 0.0, 4.0 * T_cap * Hkv * dh * 2);
-  return cudaGetLastError();
+  return r;
 }
 
 cudaError_t kv_append(const void* qkv, const int* lens, int B, int Hq, int Hkv, int dh, void* kv_l, int S_cap,

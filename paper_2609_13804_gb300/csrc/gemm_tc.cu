@@ -455,16 +455,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int lane = threadIdx.x & 31;
   int* err = args.err;
 
-  int M = args.M_cap;
-  if (args.M_dev) M = min(M, __ldg(args.M_dev));
-  if (M < 0) M = 0;
-  const int num_m = (M + BM - 1) / BM;
-  const int num_n = args.N_acc / BN;
-  const int ks = args.ksplit > 1 ? args.ksplit : 1;
-  const int total = num_m * num_n * ks;  // work items: (tile, K range)
-  const int KB = args.K / BK;
-  const bool swb = (EPI == EPI_SWIGLU_BF16) || args.swiglu_b;
-
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -485,6 +475,19 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tslot;
+  // everything above overlaps the previous kernel's tail (programmatic launch)
+  pdl_wait();
+  pdl_trigger();
+
+  int M = args.M_cap;
+  if (args.M_dev) M = min(M, __ldg(args.M_dev));
+  if (M < 0) M = 0;
+  const int num_m = (M + BM - 1) / BM;
+  const int num_n = args.N_acc / BN;
+  const int ks = args.ksplit > 1 ? args.ksplit : 1;
+  const int total = num_m * num_n * ks;  // work items: (tile, K range)
+  const int KB = args.K / BK;
+  const bool swb = (EPI == EPI_SWIGLU_BF16) || args.swiglu_b;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -761,16 +764,6 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   const bool leader = (rank == 0);
   int* err = args.err;
 
-  int M = args.M_cap;
-  if (args.M_dev) M = min(M, __ldg(args.M_dev));
-  if (M < 0) M = 0;
-  const int num_m = (M + 2 * BM - 1) / (2 * BM);
-  const int num_n = args.N_acc / BN;
-  const int total = num_m * num_n;
-  const int KB = args.K / BK;
-  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  const Sched sc = make_sched(total, num_m, KB, npairs, pair, args.sk_part != nullptr && args.sk_flags != nullptr);
-
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -791,6 +784,19 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tslot;
+  // everything above overlaps the previous kernel's tail (programmatic launch)
+  pdl_wait();
+  pdl_trigger();
+
+  int M = args.M_cap;
+  if (args.M_dev) M = min(M, __ldg(args.M_dev));
+  if (M < 0) M = 0;
+  const int num_m = (M + 2 * BM - 1) / (2 * BM);
+  const int num_n = args.N_acc / BN;
+  const int total = num_m * num_n;
+  const int KB = args.K / BK;
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const Sched sc = make_sched(total, num_m, KB, npairs, pair, args.sk_part != nullptr && args.sk_flags != nullptr);
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer (both CTAs)
@@ -987,13 +993,15 @@ cudaError_t launch_pair(const CUtensorMap& A, const CUtensorMap& B, const CUtens
   cfg.blockDim = dim3(192, 1, 1);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, gemm_tc2_kernel<BN, EPI>, A, B, O, a);
 }
 
@@ -1017,6 +1025,8 @@ cudaError_t dispatch_pair(const CUtensorMap& A, const CUtensorMap& B, const CUte
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restrict__ part, int ks, int m_pad,
                                                             int M_cap, const int* __restrict__ M_dev, int N_acc,
                                                             int BN, const GemmEpi e, int* err) {
+  pdl_wait();
+  pdl_trigger();
   int M = M_cap;
   if (M_dev) M = min(M, __ldg(M_dev));
   const int row = blockIdx.y;
@@ -1085,7 +1095,8 @@ cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const CUtenso
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  gemm_tc_kernel<BN, EPI><<<grid, 192, C::SMEM, st>>>(A, B, O, a);
+  cudaError_t le = launch_pdl(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(192), C::SMEM, st, A, B, O, a);
+  if (le != cudaSuccess) return le;
   return cudaGetLastError();
 }
 
@@ -1256,7 +1267,9 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
       const int cols = e.kind == EPI_SWIGLU_BF16 ? N_acc / 2 : N_acc;
       dim3 rg((cols + 255) / 256, M_cap);
       prof_begin_launch(st);
-      splitk_reduce_kernel<<<rg, 256, 0, st>>>(sk->splitk, kspl, m_pad, M_cap, M_dev, N_acc, bn, e, err);
+      cudaError_t re = launch_pdl(splitk_reduce_kernel, dim3(rg), dim3(256), 0, st, sk->splitk, kspl, m_pad, M_cap,
+                                  M_dev, N_acc, bn, e, err);
+      if (re != cudaSuccess) return re;
       prof_end_launch(st, SP_K_MISC, 0.0, 4.0 * kspl * (double)m_pad * N_acc);
       return cudaGetLastError();
     }

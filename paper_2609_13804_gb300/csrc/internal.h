@@ -25,6 +25,26 @@ struct GridDesc {
   int grid_w[SP_MAX_BATCH];
 };
 
+// Launch with programmatic stream serialization (the kernel must call
+// pdl_wait before touching memory other kernels use); off when the
+// environment sets SP_PDL=0.
+bool pdl_enabled();
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 bool fill_batch_desc(BatchDesc* d, int B, const int* n_vis, const int* n_txt, int group_size,
                      std::string* msg);
 

@@ -34,6 +34,8 @@ __global__ void __launch_bounds__(NT)
 rmsnorm_kernel(const float* __restrict__ x, const float* __restrict__ gain, void* __restrict__ out,
                int rows_cap, const int* __restrict__ row_count, int d, float eps) {
   __shared__ float red[32];
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x;
   if (row >= rows_from(rows_cap, row_count)) return;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)row * d);
@@ -95,6 +97,8 @@ layernorm_kernel(const float* __restrict__ x, int ldx, const float* __restrict__
 
 __global__ void bf16_to_f32_kernel(const uint2* __restrict__ x, float4* __restrict__ out, int rows_cap,
                                    const int* __restrict__ row_count, int d) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x;
   if (row >= rows_from(rows_cap, row_count)) return;
   const int n4 = d >> 2;
@@ -108,6 +112,8 @@ __global__ void bf16_to_f32_kernel(const uint2* __restrict__ x, float4* __restri
 // Rows [T, T + gridDim.x) of a row-major buffer, T = *row_count, below rows_cap, set to zero.
 __global__ void zero_rows_after_kernel(uint4* __restrict__ buf, int row_u4, const int* __restrict__ row_count,
                                        int rows_cap) {
+  pdl_wait();
+  pdl_trigger();
   const int row = __ldg(row_count) + blockIdx.x;
   if (row < 0 || row >= rows_cap) return;
   for (int i = threadIdx.x; i < row_u4; i += blockDim.x) buf[(size_t)row * row_u4 + i] = make_uint4(0, 0, 0, 0);
@@ -202,18 +208,20 @@ cudaError_t rmsnorm_f32_to_bf16(const float* x, const float* gain, void* out, in
                                 const int* row_count, int d, float eps, cudaStream_t st) {
   if (rows_cap <= 0) return cudaSuccess;
   prof_begin_launch(st);
-  rmsnorm_kernel<true><<<rows_cap, NT, 0, st>>>(x, gain, out, rows_cap, row_count, d, eps);
+  const cudaError_t r = launch_pdl(rmsnorm_kernel<true>, dim3(rows_cap), dim3(NT), 0, st, x, gain, out, rows_cap,
+                                   row_count, d, eps);
   prof_end_launch(st, SP_K_NORM, 0.0, 6.0 * rows_cap * (double)d);
-  return cudaGetLastError();
+  return r;
 }
 
 cudaError_t rmsnorm_f32_to_f32(const float* x, const float* gain, float* out, int rows_cap,
                                const int* row_count, int d, float eps, cudaStream_t st) {
   if (rows_cap <= 0) return cudaSuccess;
   prof_begin_launch(st);
-  rmsnorm_kernel<false><<<rows_cap, NT, 0, st>>>(x, gain, out, rows_cap, row_count, d, eps);
+  const cudaError_t r = launch_pdl(rmsnorm_kernel<false>, dim3(rows_cap), dim3(NT), 0, st, x, gain,
+                                   static_cast<void*>(out), rows_cap, row_count, d, eps);
   prof_end_launch(st, SP_K_NORM, 0.0, 8.0 * rows_cap * (double)d);
-  return cudaGetLastError();
+  return r;
 }
 
 cudaError_t layernorm_f32(const float* x, int ldx, const float* gain, const float* bias, float* out_f32,
@@ -232,20 +240,21 @@ cudaError_t zero_rows_after(void* buf, size_t row_bytes, const int* row_count, i
   if (rows_cap <= 0 || nrows <= 0) return cudaSuccess;
   if (row_bytes % 16 != 0) return cudaErrorInvalidValue;
   prof_begin_launch(st);
-  zero_rows_after_kernel<<<nrows, 256, 0, st>>>(reinterpret_cast<uint4*>(buf), (int)(row_bytes / 16), row_count,
-                                                 rows_cap);
+  const cudaError_t r = launch_pdl(zero_rows_after_kernel, dim3(nrows), dim3(256), 0, st,
+                                   reinterpret_cast<uint4*>(buf), (int)(row_bytes / 16), row_count, rows_cap);
   prof_end_launch(st, SP_K_MISC, 0.0, (double)nrows * row_bytes);
-  return cudaGetLastError();
+  return r;
 }
 
 cudaError_t bf16_to_f32(const void* x, float* out, int rows_cap, const int* row_count, int d,
                         cudaStream_t st) {
   if (rows_cap <= 0) return cudaSuccess;
   prof_begin_launch(st);
-  bf16_to_f32_kernel<<<rows_cap, 256, 0, st>>>(reinterpret_cast<const uint2*>(x),
-                                              reinterpret_cast<float4*>(out), rows_cap, row_count, d);
+  const cudaError_t r = launch_pdl(bf16_to_f32_kernel, dim3(rows_cap), dim3(256), 0, st,
+                                   reinterpret_cast<const uint2*>(x), reinterpret_cast<float4*>(out), rows_cap,
+                                   row_count, d);
   prof_end_launch(st, SP_K_MISC, 0.0, 6.0 * rows_cap * (double)d);
-  return cudaGetLastError();
+  return r;
 }
 
 cudaError_t assemble_encoder_input(const BatchDesc& bd, const void* X, const float* P, int D,

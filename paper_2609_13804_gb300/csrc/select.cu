@@ -80,17 +80,21 @@ __host__ __device__ inline SelSmem sel_layout(int h, int n_loc, int k_max, int C
   L.wsm = o;      o += al16((size_t)NW * 2 * 4);
   L.all_sm = o;   o += al16((size_t)2 * C * 2 * 4);
   L.score = o;    o += al16((size_t)n_loc * 4);
-  // decoders of several layers: the new position's residual / attention /
-  // cross-attention outputs and a normalised input (h each), and the pushed
-  // matrix-vector products (3h q|k|v, 4h FFN hidden, h FFN output)
+  // decoders of several layers: the new position's residual, its running
+  // attention / cross-attention output (updated in place), a normalised input
+  // (h each), and the pushed matrix-vector products.  Aliases: the pushed
+  // q|k|v (3h) and FFN hidden (4h) share one region (q|k|v is consumed before
+  // the self-attention barrier, the hidden written after the cross-attention
+  // one); the pushed FFN output shares the normalised input's region (its last
+  // local reader, the FFN's first mat-vec, is behind a barrier before any push)
   const size_t hm = multi ? (size_t)h : 0;
   L.mx = o;       o += al16(hm * 4);
   L.ma = o;       o += al16(hm * 4);
-  L.mc = o;       o += al16(hm * 4);
+  L.mc = L.ma;
   L.mn = o;       o += al16(hm * 4);
-  L.v3 = o;       o += al16(3 * hm * 4);
+  L.xo = L.mn;
+  L.v3 = o;
   L.hb = o;       o += al16(4 * hm * 4);
-  L.xo = o;       o += al16(hm * 4);
   L.total = o;
   return L;
 }
@@ -516,11 +520,13 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
       out[d] = o * inv;
     }
   };
-  // online-softmax update of a warp's partial with P scored rows
-  auto absorb = [&](const float (&sc)[P], const float4 (&vr)[P][HV], int valid, float& m_w, float& l_w,
+  constexpr int PL = P > 1 ? P / 2 : 1;  // rows per warp batch in the deep-decoder loops
+  // online-softmax update of a warp's partial with PL scored rows (fewer rows per batch than step 1:
+  // these loops share the registers with the step-1 state)
+  auto absorb = [&](const float (&sc)[PL], const float4 (&vr)[PL][HV], int valid, float& m_w, float& l_w,
                     float4 (&o_w)[HV]) {
 #pragma unroll
-    for (int pp = 0; pp < P; ++pp) {
+    for (int pp = 0; pp < PL; ++pp) {
       if (pp < valid) {
         const float sv = sc[pp];
         const float mn2 = fmaxf(m_w, sv);
@@ -547,10 +553,10 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     float4 o_w[HV];
 #pragma unroll
     for (int k = 0; k < HV; ++k) o_w[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k0 = warp * P; k0 < np2; k0 += NW * P) {
-      float4 kr[P][HV], vr[P][HV];
+    for (int k0 = warp * PL; k0 < np2; k0 += NW * PL) {
+      float4 kr[PL][HV], vr[PL][HV];
 #pragma unroll
-      for (int pp = 0; pp < P; ++pp) {
+      for (int pp = 0; pp < PL; ++pp) {
         if (k0 + pp < np2) {
           const int pos = rank + (k0 + pp) * C;
           if (l == 0) {
@@ -572,16 +578,16 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           }
         }
       }
-      float sc[P];
+      float sc[PL];
 #pragma unroll
-      for (int pp = 0; pp < P; ++pp) {
+      for (int pp = 0; pp < PL; ++pp) {
         sc[pp] = 0.f;
         if (k0 + pp < np2) {
 #pragma unroll
           for (int k = 0; k < HV; ++k) sc[pp] += dot4(qv[k], kr[pp][k]);
         }
       }
-      warp_sum_n<P>(sc);
+      warp_sum_n<PL>(sc);
       absorb(sc, vr, np2 - k0, m_w, l_w, o_w);
     }
     push_partial(o_w, m_w, l_w, slot);
@@ -599,10 +605,10 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     float4 o_w[HV];
 #pragma unroll
     for (int k = 0; k < HV; ++k) o_w[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k0 = warp * P; k0 < ncand; k0 += NW * P) {
-      float4 kr[P][HV], vr[P][HV];
+    for (int k0 = warp * PL; k0 < ncand; k0 += NW * PL) {
+      float4 kr[PL][HV], vr[PL][HV];
 #pragma unroll
-      for (int pp = 0; pp < P; ++pp) {
+      for (int pp = 0; pp < PL; ++pp) {
         if (k0 + pp < ncand) {
           const int jj = k0 + pp;
           const int row = jj < nl ? row0 + j0 + jj : a.stop_row;
@@ -614,16 +620,16 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
           }
         }
       }
-      float sc[P];
+      float sc[PL];
 #pragma unroll
-      for (int pp = 0; pp < P; ++pp) {
+      for (int pp = 0; pp < PL; ++pp) {
         sc[pp] = 0.f;
         if (k0 + pp < ncand) {
 #pragma unroll
           for (int k = 0; k < HV; ++k) sc[pp] += dot4(xv[k], kr[pp][k]);
         }
       }
-      warp_sum_n<P>(sc);
+      warp_sum_n<PL>(sc);
       absorb(sc, vr, ncand - k0, m_w, l_w, o_w);
     }
     push_partial(o_w, m_w, l_w, slot);

@@ -4,6 +4,7 @@ launches).  Shapes are those of the 16-image LLaVA-1.5-7B-shaped batch.
 
     python -m paper_2609_13804_gb300.profile_case gemm       # 1 decoder layer, T = 1791 (4 GEMMs)
     python -m paper_2609_13804_gb300.profile_case select     # selection from a given memory H
+    python -m paper_2609_13804_gb300.profile_case select_deep  # 2-layer pointer decoder, 4 images, cap 64
     python -m paper_2609_13804_gb300.profile_case compact    # compaction of the batch
     python -m paper_2609_13804_gb300.profile_case compact_full  # every visual token kept (50 MB)
     python -m paper_2609_13804_gb300.profile_case attention  # 1 decoder layer, like gemm
@@ -68,6 +69,19 @@ def main(case: str):
         ws = None
         for _ in range(2):
             r = B.sp_select(selector, w.n_vis, w.n_txt, H=Hd, stop_bias=bias, k_max=w.k_max, traces=False, ws=ws)
+            ws = r["_ws"]
+        torch.cuda.synchronize()
+    elif case == "select_deep":
+        w.n_vis, w.n_txt = w.n_vis[:4], w.n_txt[:4]
+        s = S.SelectorShape(D=w.selector.D, D_text=w.selector.D_text, h=w.selector.h, n_enc_layers=0,
+                            n_dec_layers=2)
+        w = dataclasses.replace(w, selector=s)
+        selector = B.Selector(s, S.make_selector_weights(w), dev)
+        Hd = B.dev_f32(S.make_memory(w), dev)
+        bias = B.dev_f32(np.full(4, -1e30), dev)
+        ws = None
+        for _ in range(2):
+            r = B.sp_select(selector, w.n_vis, w.n_txt, H=Hd, stop_bias=bias, k_max=64, traces=False, ws=ws)
             ws = r["_ws"]
         torch.cuda.synchronize()
     elif case == "compact_full":
