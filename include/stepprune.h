@@ -490,7 +490,9 @@ SP_API sp_status sp_prefill(const sp_model* m, const sp_prefill_io* io, void* wo
  * RMSNorm of its last residual into hidden[b], and then increments lens[b]
  * (on the device, so steps chain without a host round trip).
  * Errors: a position >= kv_S_cap sets SP_DEVERR_INDEX (nothing is written
- * for that sequence's cache row).
+ * for that sequence's cache row); more than 8 query heads per key / value
+ * head -> SP_ERR_UNSUPPORTED.  max_len_cap sizes the attention's key split
+ * only: a longer sequence is still attended in full (its ranges grow).
  */
 typedef struct {
   int B;                    /* sequences, as in the prefill that wrote kv */

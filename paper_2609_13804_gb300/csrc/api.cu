@@ -942,7 +942,11 @@ struct PrefillParts {
   int* mident = nullptr;    // mRoPE: row r -> r
   float* splitk = nullptr;  // small-M split-K planes (T_cap <= 128)
   size_t splitk_floats = 0;
+  float* dattn = nullptr;   // decode: attention partials of the key ranges
+  int* dcnt = nullptr;      // decode: per layer, per (sequence, kv head) range counters
 };
+
+constexpr int kDecodeSplits = 16;  // key ranges per sequence in a generation step, at most
 
 static size_t model_max_n(const sp_model_cfg& c) {
   return (size_t)std::max(std::max((c.n_heads + 2 * c.n_kv_heads) * c.head_dim, c.d), 2 * c.ffn);
@@ -1093,6 +1097,8 @@ static size_t decode_ws(const sp_model* m, int B, Carve& cv, PrefillParts* p) {
     q.splitk_floats = gemm_splitk_floats((int)model_max_n(c));
     q.splitk = cv.take<float>(q.splitk_floats);
   }
+  q.dattn = cv.take<float>(decode_attention_floats((int)R, c.n_heads, c.head_dim, kDecodeSplits));
+  q.dcnt = cv.take<int>((size_t)c.n_layers * R * c.n_kv_heads);
   if (p) *p = q;
   return cv.off;
 }
@@ -1111,6 +1117,8 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
   if (!io->rope_pos && io->max_len_cap > c.max_pos)  // (explicit rotary positions are checked on the device)
     return fail(SP_ERR_SHAPE, "sp_decode: max_len_cap %d > max_pos %d", io->max_len_cap, c.max_pos);
   if (!io->x || !io->lens || !io->kv || !io->hidden) return fail(SP_ERR_INVALID_ARG, "sp_decode: x, lens, kv, hidden required");
+  if (c.n_heads / c.n_kv_heads > 8)
+    return fail(SP_ERR_UNSUPPORTED, "sp_decode: more than 8 query heads per key / value head");
   if (!al16(io->x) || !al16(io->kv) || !al16(io->hidden)) return fail(SP_ERR_ALIGN, "sp_decode: buffers must be 16-byte aligned");
   Carve cv(ws);
   PrefillParts p;
@@ -1121,13 +1129,15 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
   const int dq = c.n_heads * c.head_dim, qkvw = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim;
   const size_t layer_elems = (size_t)2 * B * io->kv_S_cap * c.n_kv_heads * c.head_dim;
   std::string msg;
-  CUtensorMap tX, tO, tA;
+  CUtensorMap tX, tO, tA, tX16, tO16, tA16;  // box rows 128 / 16 (weight-streaming GEMMs)
   if (!encode_tmap_bf16(&tX, p.xb, B, c.d, 128, &msg) || !encode_tmap_bf16(&tO, p.ob, B, dq, 128, &msg) ||
-      !encode_tmap_bf16(&tA, p.act, B, c.ffn, 128, &msg))
+      !encode_tmap_bf16(&tA, p.act, B, c.ffn, 128, &msg) || !encode_tmap_bf16(&tX16, p.xb, B, c.d, 16, &msg) ||
+      !encode_tmap_bf16(&tO16, p.ob, B, dq, 16, &msg) || !encode_tmap_bf16(&tA16, p.act, B, c.ffn, 16, &msg))
     return fail(SP_ERR_CUDA, "%s", msg.c_str());
   GemmScratch gs;
   gs.splitk = p.splitk;
   gs.splitk_floats = p.splitk_floats;
+  SP_CUDA(cudaMemsetAsync(p.dcnt, 0, sizeof(int) * (size_t)c.n_layers * B * c.n_kv_heads, st), "decode counters");
   SP_CUDA(bf16_to_f32(io->x, p.h32, B, nullptr, c.d, st), "embed");
   for (int l = 0; l < c.n_layers; ++l) {
     void* kv_l = static_cast<uint16_t*>(io->kv) + (size_t)l * layer_elems;
@@ -1141,24 +1151,24 @@ static sp_status decode_impl(const sp_model* m, const sp_decode_io* io, void* ws
     eq.max_pos = c.max_pos;
     eq.head_dim = c.head_dim;
     eq.rope_cols = (c.n_heads + c.n_kv_heads) * c.head_dim;
-    SP_CUDA(gemm_bf16(tX, B, nullptr, m->qkv[l], qkvw, eq, io->err, st, &gs), "qkv");
-    SP_CUDA(kv_append(p.qkv, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim, kv_l, io->kv_S_cap, io->err, st),
-            "kv append");
-    SP_CUDA(decode_attention(p.qkv, kv_l, io->kv_S_cap, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim, p.ob, st),
+    SP_CUDA(gemm_bf16(tX, B, nullptr, m->qkv[l], qkvw, eq, io->err, st, &gs, nullptr, &tX16), "qkv");
+    SP_CUDA(decode_attention(p.qkv, kv_l, io->kv_S_cap, io->lens, B, c.n_heads, c.n_kv_heads, c.head_dim,
+                             io->max_len_cap, p.dattn, kDecodeSplits, p.dcnt + (size_t)l * B * c.n_kv_heads, p.ob,
+                             io->err, st),
             "decode attention");
     GemmEpi er;
     er.kind = EPI_F32_ACC;
     er.out = p.h32;
     er.ldo = c.d;
-    SP_CUDA(gemm_bf16(tO, B, nullptr, m->o[l], c.d, er, io->err, st, &gs), "o");
+    SP_CUDA(gemm_bf16(tO, B, nullptr, m->o[l], c.d, er, io->err, st, &gs, nullptr, &tO16), "o");
     SP_CUDA(rmsnorm_f32_to_bf16(p.h32, m->w.mlp_norm[l], p.xb, B, nullptr, c.d, c.rms_eps, st), "mlp norm");
     GemmEpi eg;
     eg.kind = EPI_SWIGLU_BF16;
     eg.out = p.act;
     eg.ldo = c.ffn;
     eg.up_off = c.ffn;
-    SP_CUDA(gemm_bf16(tX, B, nullptr, m->gu[l], 2 * c.ffn, eg, io->err, st, &gs), "gate/up");
-    SP_CUDA(gemm_bf16(tA, B, nullptr, m->down[l], c.d, er, io->err, st, &gs), "down");
+    SP_CUDA(gemm_bf16(tX, B, nullptr, m->gu[l], 2 * c.ffn, eg, io->err, st, &gs, nullptr, &tX16), "gate/up");
+    SP_CUDA(gemm_bf16(tA, B, nullptr, m->down[l], c.d, er, io->err, st, &gs, nullptr, &tA16), "down");
   }
   SP_CUDA(rmsnorm_f32_to_f32(p.h32, m->w.final_norm, io->hidden, B, nullptr, c.d, c.rms_eps, st), "final norm");
   SP_CUDA(lens_increment(io->lens, io->rope_pos, B, io->kv_S_cap, st), "lens");

@@ -149,6 +149,13 @@ SP_DEVINL void tma_reduce_add_2d(const void* tmap, const void* smem_src, int x, 
                : "memory");
 }
 
+// Untiled bulk copy global -> this CTA's shared memory (addresses 16-byte
+// aligned, bytes a multiple of 16), completing on the CTA's mbarrier `bar`.
+SP_DEVINL void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+
 SP_DEVINL void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 
 // Wait until at most N committed bulk groups of this thread still read shared memory.

@@ -41,7 +41,8 @@ constexpr uint32_t EPI_STAGE_BYTES = 4 * 2 * BOX_BYTES;
 
 template <int BN>
 struct Cfg {
-  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  // BN = 32: the weight-streaming variant (16 KB of weights per stage, deep ring)
+  static constexpr int STAGES = (BN == 256) ? 4 : (BN == 32 ? 9 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
@@ -1084,6 +1085,97 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restr
   }
 }
 
+// Sum of the K-range partials of the weight-streaming GEMM and the epilogue
+// of the unsplit GEMM.  Partials are planes [ks][N_acc][32]: row n = output
+// column n (weight row), column m = activation row m.  Thread (c, q): output
+// column c, activation rows 8q..8q+7 (a warp reads 8 consecutive 128-byte
+// partial rows; its stores cover 8 consecutive columns of 4 rows).
+__global__ void __launch_bounds__(256) splitk_reduce_t_kernel(const float* __restrict__ part, int ks, int N_acc,
+                                                              int M_cap, const int* __restrict__ M_dev,
+                                                              int cols, const GemmEpi e, int* err) {
+  pdl_wait();
+  pdl_trigger();
+  int M = M_cap;
+  if (M_dev) M = min(M, __ldg(M_dev));
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  const int c = t >> 2, m0 = (t & 3) * 8;
+  if (c >= cols || m0 >= M) return;
+  const int mn = min(8, M - m0);
+  const size_t plane = (size_t)N_acc * 32;
+  auto sum8 = [&](int n, float (&v)[8]) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = 0.f;
+    const float* p = part + (size_t)n * 32 + m0;
+    for (int s = 0; s < ks; ++s) {
+      const float4 a = __ldcg(reinterpret_cast<const float4*>(p + s * plane));
+      const float4 b = __ldcg(reinterpret_cast<const float4*>(p + s * plane) + 1);
+      v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
+      v[4] += b.x; v[5] += b.y; v[6] += b.z; v[7] += b.w;
+    }
+  };
+  float v[8];
+  if (e.kind == EPI_SWIGLU_BF16) {
+    float u[8];
+    sum8(c, v);
+    sum8(e.up_off + c, u);
+    __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(e.out) + c;
+    #pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (i < mn) o[(size_t)(m0 + i) * e.ldo] = __float2bfloat16_rn(silu(v[i]) * u[i]);
+    return;
+  }
+  if (e.kind == EPI_BF16_ROPE) {
+    const int dh = e.head_dim, half = dh >> 1;
+    const int hb = (c / dh) * dh, i0 = c - hb;
+    __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(e.out) + c;
+    if (hb < e.rope_cols) {
+      if (i0 >= half) return;  // the pair's first element writes both
+      float u[8];
+      sum8(c, v);
+      sum8(c + half, u);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (i >= mn) break;
+        const int row = m0 + i;
+        const int p = __ldg(e.pos + row);
+        const bool pos_ok = p >= 0 && p < e.max_pos;
+        if (!pos_ok) set_error(err, SP_DEVERR_INDEX);
+        const float2 r = __ldg(e.rope + (size_t)(pos_ok ? p : 0) * half + i0);
+        o[(size_t)row * e.ldo] = __float2bfloat16_rn(v[i] * r.x - u[i] * r.y);
+        o[(size_t)row * e.ldo + half] = __float2bfloat16_rn(u[i] * r.x + v[i] * r.y);
+      }
+    } else {
+      sum8(c, v);
+      #pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (i < mn) o[(size_t)(m0 + i) * e.ldo] = __float2bfloat16_rn(v[i]);
+    }
+    return;
+  }
+  sum8(c, v);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (i >= mn) break;
+    const int row = m0 + i;
+    if (e.kind == EPI_F32) {
+      reinterpret_cast<float*>(e.out)[(size_t)row * e.ldo + c] = v[i];
+    } else if (e.kind == EPI_F32_ACC) {
+      reinterpret_cast<float*>(e.out)[(size_t)row * e.ldo + c] += v[i];
+    } else if (e.kind == EPI_GELU_BF16) {
+      reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)row * e.ldo + c] = __float2bfloat16_rn(gelu_erf(v[i]));
+    } else if (e.kind == EPI_SCATTER_BF16) {
+      const int orow = __ldg(e.row_map + row);
+      if (orow < 0) {
+        set_error(err, SP_DEVERR_INDEX);
+        continue;
+      }
+      reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)orow * e.ldo + c] = __float2bfloat16_rn(v[i]);
+    } else {
+      reinterpret_cast<__nv_bfloat16*>(e.out)[(size_t)row * e.ldo + c] = __float2bfloat16_rn(v[i]);
+    }
+  }
+}
+
 template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& O, const KArgs& a, int grid,
                        cudaStream_t st) {
@@ -1116,6 +1208,51 @@ cudaError_t dispatch(const CUtensorMap& A, const CUtensorMap& B, const CUtensorM
 }
 
 }  // namespace
+
+// K ranges per 128-row weight tile of the weight-streaming GEMM: the split
+// that minimises the busiest CTA's K blocks (units t = blockIdx.x + i * grid,
+// half a K block of hand-over per unit, ~0.36 us per 16 KB block at an SM's
+// share of HBM bandwidth) plus the partial planes' write and read through L2
+// (N_acc x 128 bytes per range).  Cached per shape (host-side cost: O(units)).
+static int swap_split(int tiles, int KB, int sms, size_t cap_floats, int N_acc) {
+  struct Entry { int tiles, KB, sms, N, ks; };
+  static thread_local Entry cache[16];
+  static thread_local int n_cached = 0;
+  for (int i = 0; i < n_cached; ++i)
+    if (cache[i].tiles == tiles && cache[i].KB == KB && cache[i].sms == sms && cache[i].N == N_acc)
+      return cache[i].ks;
+  int best = 1;
+  double best_us = 1e30;
+  for (int ks = 1; ks <= std::min(16, std::max(1, KB / 2)); ++ks) {
+    if ((size_t)ks * N_acc * 32 > cap_floats) break;
+    const int U = tiles * ks, G = std::min(U, sms);
+    double worst = 0.0;
+    for (int c = 0; c < G; ++c) {
+      double kb = 0.0;
+      for (int u = c; u < U; u += G) {
+        const int sp = u % ks;
+        kb += (double)((sp + 1) * KB / ks - sp * KB / ks) + 0.5;
+      }
+      worst = std::max(worst, kb);
+    }
+    const double us = worst * 0.364 + (double)ks * N_acc * 128.0 / 8.0e6;
+    if (us < best_us) {
+      best_us = us;
+      best = ks;
+    }
+  }
+  if (n_cached < 16) cache[n_cached++] = Entry{tiles, KB, sms, N_acc, best};
+  return best;
+}
+
+static bool gemm_swap_enabled() {
+  static int mode = -1;
+  if (mode < 0) {
+    const char* s = getenv("SP_GEMM_SWAP");
+    mode = s ? atoi(s) : 1;
+  }
+  return mode != 0;
+}
 
 // Tile width of the CTA-pair variant for a GEMM, or 0 for the single-CTA one.
 // Pairs with 256-wide tiles wherever M reaches a pair tile: measured on the
@@ -1179,9 +1316,51 @@ bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {
 
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B, int N_acc,
                       const GemmEpi& e, int* err, cudaStream_t st, const GemmScratch* sk,
-                      const GemmASplit* as) {
+                      const GemmASplit* as, const CUtensorMap* A16) {
   if (M_cap <= 0) return cudaSuccess;
   const int sms = device_sm_count();
+  // Weight streaming for M <= 32 rows (generation steps): the weights are the
+  // MMA's 128-row operand and the activations its 32 columns (C^T = B A^T),
+  // each 128-row weight tile's K split into ranges over the SMs; the fp32
+  // partials [range][N_acc][32] are summed, with the fused epilogue, by one
+  // transposed reduce pass.
+  if (A16 && sk && sk->splitk && M_cap <= 32 && N_acc % BM == 0 && B.K % BK == 0 && !(as && as->seg > 0) &&
+      gemm_swap_enabled()) {
+    const int tiles = N_acc / BM, KB = B.K / BK;
+    const int ks = swap_split(tiles, KB, sms, sk->splitk_floats, N_acc);
+    if ((size_t)ks * N_acc * 32 <= sk->splitk_floats) {
+      CUtensorMap tmP;
+      if (!encode_tmap_2d(&tmP, sk->splitk, true, (uint64_t)ks * N_acc, 32, 32, 32, nullptr))
+        return cudaErrorInvalidValue;
+      KArgs a;
+      a.M_cap = N_acc;
+      a.M_dev = nullptr;
+      a.N_acc = 32;
+      a.K = B.K;
+      a.e = GemmEpi();
+      a.e.kind = EPI_F32;
+      a.err = err;
+      a.a_seg = 0;
+      a.a_map = 0;
+      a.ksplit = ks;
+      a.m_pad = N_acc;
+      a.swiglu_b = 0;
+      a.sk_part = nullptr;
+      a.sk_flags = nullptr;
+      const int grid = std::max(1, std::min(tiles * ks, sms));
+      prof_begin_launch(st);
+      cudaError_t r = launch_one<32, EPI_F32>(B.map256, *A16, tmP, a, grid, st);
+      prof_end_launch(st, SP_K_GEMM, 2.0 * (double)M_cap * (double)N_acc * (double)B.K, 0.0);
+      if (r != cudaSuccess) return r;
+      const int cols = e.kind == EPI_SWIGLU_BF16 ? N_acc / 2 : N_acc;
+      prof_begin_launch(st);
+      r = launch_pdl(splitk_reduce_t_kernel, dim3((cols * 4 + 255) / 256), dim3(256), 0, st, sk->splitk, ks, N_acc,
+                     M_cap, M_dev, cols, e, err);
+      prof_end_launch(st, SP_K_MISC, 0.0, 4.0 * ks * (double)N_acc * 32);
+      if (r != cudaSuccess) return r;
+      return cudaGetLastError();
+    }
+  }
   const int mt = (M_cap + BM - 1) / BM;
   // Pick the tile width whose last wave is fullest (RoPE heads and the SwiGLU
   // halves need the 256-wide tile to hold whole heads / 128 output columns).

@@ -128,9 +128,13 @@ struct GemmASplit {
   uint32_t map = 0;
 };
 
+// A16 (optional): A's tensor map with box rows 16.  With it, M_cap <= 32 and
+// split-K scratch, the GEMM streams the weights as the MMA's 128-row operand
+// (generation steps); the result and epilogue are the same.
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B,
                       int N_acc, const GemmEpi& e, int* err, cudaStream_t st,
-                      const GemmScratch* sk = nullptr, const GemmASplit* as = nullptr);
+                      const GemmScratch* sk = nullptr, const GemmASplit* as = nullptr,
+                      const CUtensorMap* A16 = nullptr);
 
 // ------------------------------------------------------------- candidate precompute
 // out [rows, 3K] bf16 = the three bf16 parts of x [rows, K] (fp32, row stride ldx).
@@ -166,10 +170,14 @@ cudaError_t write_enc_cu(const BatchDesc& bd, int* cu, cudaStream_t st);
 // Cache layout: layer block [2][B][S_cap][Hkv * dh] bf16 (K then V).
 cudaError_t kv_store(const void* qkv, const int* cu, const int* pos, int B, int T_cap, int Hq, int Hkv, int dh,
                      void* kv_l, int S_cap, int* err, cudaStream_t st);
-cudaError_t kv_append(const void* qkv, const int* lens, int B, int Hq, int Hkv, int dh, void* kv_l, int S_cap,
-                      int* err, cudaStream_t st);
-cudaError_t decode_attention(const void* qkv, const void* kv_l, int S_cap, const int* lens, int B, int Hq, int Hkv,
-                             int dh, void* out, cudaStream_t st);
+// One generation step's attention, the new key / value appended to the cache
+// at lens[b] on the way: out [B, Hq dh] bf16.  Keys split into at most
+// max_splits ranges per sequence; `part` holds decode_attention_floats() fp32
+// partials, `cnt` B * Hkv ints that must be zero at the launch.
+size_t decode_attention_floats(int B, int Hq, int dh, int max_splits);
+cudaError_t decode_attention(const void* qkv, void* kv_l, int S_cap, const int* lens, int B, int Hq, int Hkv, int dh,
+                             int max_len, float* part, int max_splits, int* cnt, void* out, int* err,
+                             cudaStream_t st);
 cudaError_t lens_increment(int* lens, int* rope_pos, int B, int S_cap, cudaStream_t st);
 
 // ------------------------------------------------------------- attention

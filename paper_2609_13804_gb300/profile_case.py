@@ -8,6 +8,7 @@ launches).  Shapes are those of the 16-image LLaVA-1.5-7B-shaped batch.
     python -m paper_2609_13804_gb300.profile_case compact    # compaction of the batch
     python -m paper_2609_13804_gb300.profile_case compact_full  # every visual token kept (50 MB)
     python -m paper_2609_13804_gb300.profile_case attention  # 1 decoder layer, like gemm
+    python -m paper_2609_13804_gb300.profile_case decode     # 4 decoder layers, 16 sequences, 3 steps
 
 Each case runs its stage twice (the second launch set is the one to capture
 with `-s`).
@@ -27,7 +28,7 @@ def main(case: str):
     dev = torch.device("cuda", 0)
     w = S.llava15_7b_b16()
     counts = S.target_counts(w)
-    if case in ("gemm", "attention"):
+    if case in ("gemm", "attention", "decode"):
         m = dataclasses.replace(w.model, proj_kind="none", proj_in=w.model.d)
         gen = torch.Generator(device=dev)
         gen.manual_seed(1)
@@ -40,8 +41,25 @@ def main(case: str):
              "Wdown": rnd((m.d, m.ffn)), "attn_norm": torch.ones(m.d, device=dev),
              "mlp_norm": torch.ones(m.d, device=dev)}
         head = {"final_norm": torch.ones(m.d, device=dev), "proj_W1": None, "proj_W2": None}
-        model = B.Model(m, None, None, dev, max_pos=512, device_weights={"layers": [L], "head": head})
+        n_layers = 4 if case == "decode" else 1
+        layers = [L] + [{k: (rnd(v.shape) if v.dtype == torch.bfloat16 else v) for k, v in L.items()}
+                        for _ in range(n_layers - 1)]
+        m = dataclasses.replace(m, n_layers=n_layers)
+        model = B.Model(m, None, None, dev, max_pos=512, device_weights={"layers": layers, "head": head})
         lens = [int(k) + 48 for k in counts]
+        if case == "decode":
+            # one generation step per sequence over the pruned prefix (a zeroed
+            # cache with the prefix lengths: the contents do not change the work)
+            S_cap = max(lens) + 8
+            kv = B.kv_cache(model, len(lens), S_cap)
+            x_new = (torch.randn((len(lens), m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+            lens_d = torch.tensor(lens, dtype=torch.int32, device=dev)
+            ws = None
+            for _ in range(3):
+                ws = B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws)["_ws"]
+            torch.cuda.synchronize()
+            print("ok", case)
+            return
         T = sum(lens)
         cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
         pos = torch.tensor(np.concatenate([np.arange(n) for n in lens]), dtype=torch.int32, device=dev)

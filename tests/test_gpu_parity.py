@@ -551,6 +551,25 @@ def test_decode_empty_prefix(B):
     _decode_case(B, w, [0, 7, 1], 2)
 
 
+def test_decode_long_prefix_gqa8(B):
+    # 8 query heads per key / value head (the widest group the decode takes) and
+    # a prefix longer than 16 key ranges of 64: each range then spans several
+    # shared-memory tiles of keys
+    w = S.tiny_workload(66, [1], [1], D=128, d=256, n_heads=8, n_kv_heads=1, head_dim=128, ffn=256, n_layers=1)
+    _decode_case(B, w, [1300, 65, 0, 64], 1)
+
+
 def test_decode_llama7b_dims_1layer(B):
     w = S.llava15_7b_b16()
     _decode_case(B, w, [112, 240, 64, 17], 1)
+
+
+@pytest.mark.parametrize("nb", [16, 32, 33])
+def test_decode_llama7b_dims_batch_edges(B, nb):
+    # 16 and 32 sequences take the weight-streaming GEMMs (activations as the
+    # MMA's 32 columns: one or two 16-row halves), 33 the 128-row-tile path
+    w = S.llava15_7b_b16()
+    rng = np.random.default_rng(900 + nb)
+    lens = [int(v) for v in rng.integers(0, 24, nb)]
+    lens[0] = 0
+    _decode_case(B, w, lens, 1)
