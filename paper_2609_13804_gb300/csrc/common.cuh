@@ -149,6 +149,12 @@ SP_DEVINL void tma_reduce_add_2d(const void* tmap, const void* smem_src, int x, 
                : "memory");
 }
 
+// Hint: one box of a tiled tensor map into L2 (no shared memory, no barrier).
+SP_DEVINL void tma_prefetch_l2_2d(const void* map, int c0, int c1) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1) : "memory");
+}
+
 // Untiled bulk copy global -> this CTA's shared memory (addresses 16-byte
 // aligned, bytes a multiple of 16), completing on the CTA's mbarrier `bar`.
 SP_DEVINL void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {

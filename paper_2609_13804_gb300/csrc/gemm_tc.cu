@@ -32,6 +32,10 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
+// K blocks of the first work item's weights a CTA asks L2 for before it waits
+// on the previous kernel (weights never depend on it): the fetch of the first
+// stages overlaps that kernel's tail.
+constexpr int kPrefetchBlocks = 8;
 
 // Epilogue staging: per epilogue warp two boxes of 32 rows x 128 bytes
 // (128-byte swizzle) that TMA stores (or reduce-adds) to global memory while
@@ -476,6 +480,31 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tslot;
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    // the weight boxes of this CTA's first work item (tile order from the host
+    // cap M_cap; a wrong guess only wastes the hint).  BN = 32 is the
+    // weight-streaming variant, whose weights are A.
+    const int nm0 = (args.M_cap + BM - 1) / BM;
+    const int ks0 = args.ksplit > 1 ? args.ksplit : 1;
+    const int t0 = blockIdx.x;
+    if (t0 < nm0 * (args.N_acc / BN) * ks0) {
+      const int tile = t0 / ks0, sp = t0 - tile * ks0;
+      const int mb = tile % nm0, nb = tile / nm0;
+      const int KB0 = args.K / BK;
+      const int kb0 = sp * KB0 / ks0, kb1 = min((sp + 1) * KB0 / ks0, kb0 + kPrefetchBlocks);
+      const bool sw = (EPI == EPI_SWIGLU_BF16) || args.swiglu_b;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (BN == 32) {
+          tma_prefetch_l2_2d(&tmA, kb * BK, mb * BM);
+        } else {
+          tma_prefetch_l2_2d(&tmB, kb * BK, sw ? nb * (BN / 2) : nb * BN);
+          tma_prefetch_l2_2d(&tmB, kb * BK, sw ? args.e.up_off + nb * (BN / 2) : nb * BN + BN / 2);
+        }
+      }
+    }
+  }
   // everything above overlaps the previous kernel's tail (programmatic launch)
   pdl_wait();
   pdl_trigger();
@@ -493,8 +522,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      tma_prefetch_desc(&tmA);
-      tma_prefetch_desc(&tmB);
       int s = 0;
       uint32_t ph = 0;
       int issued = 0;
@@ -785,6 +812,21 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tslot;
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    // this CTA's half of the B (weight) rows of the pair's first tile (tile
+    // order from the host cap M_cap; a wrong guess only wastes the hint)
+    const int nm0 = (args.M_cap + 2 * BM - 1) / (2 * BM);
+    const int pair0 = blockIdx.x >> 1;
+    if (pair0 < nm0 * (args.N_acc / BN)) {
+      const int nb = pair0 / nm0;
+      const int b_row = (EPI == EPI_SWIGLU_BF16) ? (rank == 0 ? 0 : args.e.up_off) + nb * (BN / 2)
+                                                 : nb * BN + (int)rank * (BN / 2);
+      const int kb1 = min(args.K / BK, kPrefetchBlocks);
+      for (int kb = 0; kb < kb1; ++kb) tma_prefetch_l2_2d(&tmB, kb * BK, b_row);
+    }
+  }
   // everything above overlaps the previous kernel's tail (programmatic launch)
   pdl_wait();
   pdl_trigger();
@@ -802,8 +844,6 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   if (warp == 0) {
     // ------------------------------------------------------------ producer (both CTAs)
     if (lane == 0) {
-      tma_prefetch_desc(&tmA);
-      tma_prefetch_desc(&tmB);
       int s = 0;
       uint32_t ph = 0;
       Cursor cur;
@@ -1314,6 +1354,40 @@ bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {
          encode_tmap_bf16(&b->map256, w, N, K, 128, msg);
 }
 
+cudaError_t gemm_swap_partials(const CUtensorMap& A16, int M_cap, const GemmB& B, int N_acc, int* err,
+                               cudaStream_t st, const GemmScratch& sk, int* ks_out) {
+  const int sms = device_sm_count();
+  if (!sk.splitk || M_cap < 1 || M_cap > 32 || N_acc % BM != 0 || B.K % BK != 0 || !gemm_swap_enabled())
+    return cudaErrorNotSupported;
+  const int tiles = N_acc / BM, KB = B.K / BK;
+  const int ks = swap_split(tiles, KB, sms, sk.splitk_floats, N_acc);
+  if ((size_t)ks * N_acc * 32 > sk.splitk_floats) return cudaErrorNotSupported;
+  CUtensorMap tmP;
+  if (!encode_tmap_2d(&tmP, sk.splitk, true, (uint64_t)ks * N_acc, 32, 32, 32, nullptr)) return cudaErrorInvalidValue;
+  KArgs a;
+  a.M_cap = N_acc;
+  a.M_dev = nullptr;
+  a.N_acc = 32;
+  a.K = B.K;
+  a.e = GemmEpi();
+  a.e.kind = EPI_F32;
+  a.err = err;
+  a.a_seg = 0;
+  a.a_map = 0;
+  a.ksplit = ks;
+  a.m_pad = N_acc;
+  a.swiglu_b = 0;
+  a.sk_part = nullptr;
+  a.sk_flags = nullptr;
+  const int grid = std::max(1, std::min(tiles * ks, sms));
+  prof_begin_launch(st);
+  const cudaError_t r = launch_one<32, EPI_F32>(B.map256, A16, tmP, a, grid, st);
+  prof_end_launch(st, SP_K_GEMM, 2.0 * (double)M_cap * (double)N_acc * (double)B.K, 0.0);
+  if (r != cudaSuccess) return r;
+  *ks_out = ks;
+  return cudaGetLastError();
+}
+
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B, int N_acc,
                       const GemmEpi& e, int* err, cudaStream_t st, const GemmScratch* sk,
                       const GemmASplit* as, const CUtensorMap* A16) {
@@ -1324,42 +1398,19 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
   // each 128-row weight tile's K split into ranges over the SMs; the fp32
   // partials [range][N_acc][32] are summed, with the fused epilogue, by one
   // transposed reduce pass.
-  if (A16 && sk && sk->splitk && M_cap <= 32 && N_acc % BM == 0 && B.K % BK == 0 && !(as && as->seg > 0) &&
-      gemm_swap_enabled()) {
-    const int tiles = N_acc / BM, KB = B.K / BK;
-    const int ks = swap_split(tiles, KB, sms, sk->splitk_floats, N_acc);
-    if ((size_t)ks * N_acc * 32 <= sk->splitk_floats) {
-      CUtensorMap tmP;
-      if (!encode_tmap_2d(&tmP, sk->splitk, true, (uint64_t)ks * N_acc, 32, 32, 32, nullptr))
-        return cudaErrorInvalidValue;
-      KArgs a;
-      a.M_cap = N_acc;
-      a.M_dev = nullptr;
-      a.N_acc = 32;
-      a.K = B.K;
-      a.e = GemmEpi();
-      a.e.kind = EPI_F32;
-      a.err = err;
-      a.a_seg = 0;
-      a.a_map = 0;
-      a.ksplit = ks;
-      a.m_pad = N_acc;
-      a.swiglu_b = 0;
-      a.sk_part = nullptr;
-      a.sk_flags = nullptr;
-      const int grid = std::max(1, std::min(tiles * ks, sms));
-      prof_begin_launch(st);
-      cudaError_t r = launch_one<32, EPI_F32>(B.map256, *A16, tmP, a, grid, st);
-      prof_end_launch(st, SP_K_GEMM, 2.0 * (double)M_cap * (double)N_acc * (double)B.K, 0.0);
-      if (r != cudaSuccess) return r;
+  if (A16 && sk) {
+    int ks = 0;
+    const cudaError_t r = gemm_swap_partials(*A16, M_cap, B, N_acc, err, st, *sk, &ks);
+    if (r == cudaSuccess) {
       const int cols = e.kind == EPI_SWIGLU_BF16 ? N_acc / 2 : N_acc;
       prof_begin_launch(st);
-      r = launch_pdl(splitk_reduce_t_kernel, dim3((cols * 4 + 255) / 256), dim3(256), 0, st, sk->splitk, ks, N_acc,
-                     M_cap, M_dev, cols, e, err);
+      const cudaError_t rr = launch_pdl(splitk_reduce_t_kernel, dim3((cols * 4 + 255) / 256), dim3(256), 0, st,
+                                        sk->splitk, ks, N_acc, M_cap, M_dev, cols, e, err);
       prof_end_launch(st, SP_K_MISC, 0.0, 4.0 * ks * (double)N_acc * 32);
-      if (r != cudaSuccess) return r;
+      if (rr != cudaSuccess) return rr;
       return cudaGetLastError();
     }
+    if (r != cudaErrorNotSupported) return r;
   }
   const int mt = (M_cap + BM - 1) / BM;
   // Pick the tile width whose last wave is fullest (RoPE heads and the SwiGLU

@@ -128,6 +128,13 @@ struct GemmASplit {
   uint32_t map = 0;
 };
 
+// The weight-streaming GEMM without an epilogue (M_cap <= 32 rows): fp32
+// partial planes [ks][N_acc][32] (plane row n = output column n, column m =
+// row m of A) in sk.splitk, *ks_out ranges, to be summed in range order by the
+// consumer.  cudaErrorNotSupported when the shape or scratch does not allow it.
+cudaError_t gemm_swap_partials(const CUtensorMap& A16, int M_cap, const GemmB& B, int N_acc, int* err,
+                               cudaStream_t st, const GemmScratch& sk, int* ks_out);
+
 // A16 (optional): A's tensor map with box rows 16.  With it, M_cap <= 32 and
 // split-K scratch, the GEMM streams the weights as the MMA's 128-row operand
 // (generation steps); the result and epilogue are the same.
