@@ -423,7 +423,26 @@ def run_ours(args):
         torch.cuda.synchronize()
         return a.elapsed_time(b_) / reps
 
-    compact_ms = kernel_ms(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap, reuse=True))
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # twice the L2
+
+    def kernel_ms_cold(fn, reps=10):
+        # device time of a one-launch call with L2 flushed before each call (its
+        # inputs are smaller than L2): flush, then a spin kernel so the host has
+        # enqueued the events and the call before the GPU reaches them
+        fn()
+        total = 0.0
+        for _ in range(reps):
+            flush_buf.zero_()
+            a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(1_000_000)
+            a.record()
+            fn()
+            b_.record()
+            torch.cuda.synchronize()
+            total += a.elapsed_time(b_)
+        return total / reps
+
+    compact_ms = kernel_ms_cold(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap, reuse=True))
     comp_bytes = 2.0 * (K_sum * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
 
     def prefill_stage(idx, count, kc):
@@ -440,7 +459,7 @@ def run_ours(args):
     full_cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
     full_ms = timed(lambda: prefill_stage(full_idx, full_cnt, 576), reps=3)
     # compaction at a bandwidth-sized case: every visual token kept (the full prefix)
-    full_compact_ms = kernel_ms(lambda: do_compact(full_idx, full_cnt, 576, reuse=True))
+    full_compact_ms = kernel_ms_cold(lambda: do_compact(full_idx, full_cnt, 576, reuse=True))
     full_T = sum(w.n_vis) + sum(w.n_txt)
     full_comp_bytes = 2.0 * (sum(w.n_vis) * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + full_T)
 

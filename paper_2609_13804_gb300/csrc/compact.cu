@@ -1,7 +1,8 @@
 // Compaction (Algorithm 1 step 5, X_S = Gather(X, S)): the kept visual rows of
 // every image, in native order, followed by its text rows, written as one packed
 // variable-length buffer with cu_seqlens and per-sequence positions.  Pure data
-// movement, HBM-bound: one warp per output row, 16-byte vector copies.
+// movement, HBM-bound: rows are cut into 2 KB pieces and a warp moves three
+// pieces per pass with 16-byte vector copies.
 //
 // Every block recomputes the (small) prefix sums of the per-image counts from
 // the device counts, so the kernel needs no host round trip and no second
@@ -15,27 +16,7 @@ namespace {
 
 constexpr int NT = 256;
 
-// One row, 16-byte chunks per lane; eight loads are issued before their stores
-// so a warp keeps up to 4 KB in flight instead of one chunk per round trip.
-SP_DEVINL void copy_row(const uint4* __restrict__ src, uint4* __restrict__ dst, int n16, int lane) {
-  int i = lane;
-  for (; i + 7 * 32 < n16; i += 8 * 32) {
-    uint4 v[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) v[u] = __ldg(src + i + u * 32);
-#pragma unroll
-    for (int u = 0; u < 8; ++u) dst[i + u * 32] = v[u];
-  }
-  uint4 v[8];
-#pragma unroll
-  for (int u = 0; u < 8; ++u)
-    if (i + u * 32 < n16) v[u] = __ldg(src + i + u * 32);
-#pragma unroll
-  for (int u = 0; u < 8; ++u)
-    if (i + u * 32 < n16) dst[i + u * 32] = v[u];
-}
-
-__global__ void __launch_bounds__(NT, 4)
+__global__ void __launch_bounds__(NT, 2)
 compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vis,
                const __nv_bfloat16* __restrict__ text, int W_txt, const int* __restrict__ idx, int k_cap,
                const int* __restrict__ count, __nv_bfloat16* __restrict__ packed, int* __restrict__ cu,
@@ -85,41 +66,92 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
   }
   const int T = min(s_cu[B], T_cap);
   const int nv16 = W_vis / 8, nt16 = W_txt / 8;
-
-  for (int r = blockIdx.x * (NT / 32) + w; r < T; r += gridDim.x * (NT / 32)) {
-    int lo = 0, hi = B - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (s_cu[mid] <= r) lo = mid; else hi = mid - 1;
+  const int gw = blockIdx.x * (NT / 32) + w, nw = gridDim.x * (NT / 32);
+  // The copy is cut into pieces of at most PIECE16 16-byte chunks (2 KB): a
+  // visual row of 1,024 bf16 is one piece, a text row of 4,096 bf16 four.
+  // Visual pieces come first, then text pieces.  A warp takes PPW pieces per
+  // pass: it locates their rows (the visual rows' index loads go out
+  // together), then loads every chunk of the PPW pieces before storing any
+  // (12 loads per lane, 6 KB per warp in flight).
+  constexpr int PPW = 3, PIECE16 = 128;
+  const int V = s_vcu[B], Lt = bd.txt_off[B];
+  const int ppv = (nv16 + PIECE16 - 1) / PIECE16, ppt = (nt16 + PIECE16 - 1) / PIECE16;
+  const int NPv = V * ppv, NP = NPv + Lt * ppt;
+  for (int p0 = gw * PPW; p0 < NP; p0 += nw * PPW) {
+    const uint4* src[PPW];
+    uint4* dst[PPW];
+    int nc[PPW], jv[PPW], vb[PPW], c0v[PPW];
+#pragma unroll
+    for (int u = 0; u < PPW; ++u) {
+      const int pc = p0 + u;
+      nc[u] = 0;
+      jv[u] = -1;
+      vb[u] = -1;
+      c0v[u] = 0;
+      src[u] = nullptr;
+      dst[u] = nullptr;
+      if (pc >= NP) continue;
+      if (pc < NPv) {  // a piece of kept visual row vr
+        const int vr = pc / ppv, sub = pc - vr * ppv;
+        int lo = 0, hi = B - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (s_vcu[mid] <= vr) lo = mid; else hi = mid - 1;
+        }
+        const int local = vr - s_vcu[lo];
+        const int r = s_cu[lo] + local;
+        if (r >= T) continue;
+        jv[u] = __ldg(idx + (size_t)lo * k_cap + local);  // resolved below, with every index load out
+        vb[u] = lo;
+        const int c0 = sub * PIECE16;
+        c0v[u] = c0;
+        nc[u] = min(PIECE16, nv16 - c0);
+        dst[u] = (vis_packed ? reinterpret_cast<uint4*>(vis_packed + (size_t)vr * W_vis)
+                             : reinterpret_cast<uint4*>(packed + (size_t)r * W_txt)) + c0;
+        if (sub == 0 && lane == 0) {
+          pos[r] = local;
+          if (vis_packed) vis_row_map[vr] = r;
+        }
+      } else {  // a piece of text row tr
+        const int tp = pc - NPv;
+        const int tr = tp / ppt, sub = tp - tr * ppt;
+        int lo = 0, hi = B - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (bd.txt_off[mid] <= tr) lo = mid; else hi = mid - 1;
+        }
+        const int local = s_cnt[lo] + (tr - bd.txt_off[lo]);
+        const int r = s_cu[lo] + local;
+        if (r >= T) continue;
+        const int c0 = sub * PIECE16;
+        nc[u] = min(PIECE16, nt16 - c0);
+        src[u] = reinterpret_cast<const uint4*>(text + (size_t)tr * W_txt) + c0;
+        dst[u] = reinterpret_cast<uint4*>(packed + (size_t)r * W_txt) + c0;
+        if (sub == 0 && lane == 0) pos[r] = local;
+      }
     }
-    const int b = lo;
-    const int local = r - s_cu[b];
-    if (lane == 0) pos[r] = local;
-    const uint4* src;
-    uint4* dst;
-    int n16;
-    if (local < s_cnt[b]) {
-      const int j = __ldg(idx + (size_t)b * k_cap + local);
-      const int n_img = bd.vis_off[b + 1] - bd.vis_off[b];
-      if (j < 0 || j >= n_img) {
+#pragma unroll
+    for (int u = 0; u < PPW; ++u) {
+      if (vb[u] < 0) continue;
+      const int n_img = bd.vis_off[vb[u] + 1] - bd.vis_off[vb[u]];
+      if (jv[u] < 0 || jv[u] >= n_img) {
         if (lane == 0) set_error(err, SP_DEVERR_INDEX);
+        nc[u] = 0;
         continue;
       }
-      src = reinterpret_cast<const uint4*>(X + (size_t)(bd.vis_off[b] + j) * W_vis);
-      n16 = nv16;
-      if (vis_packed) {
-        const int vr = s_vcu[b] + local;
-        if (lane == 0) vis_row_map[vr] = r;
-        dst = reinterpret_cast<uint4*>(vis_packed + (size_t)vr * W_vis);
-      } else {
-        dst = reinterpret_cast<uint4*>(packed + (size_t)r * W_txt);
-      }
-    } else {
-      src = reinterpret_cast<const uint4*>(text + (size_t)(bd.txt_off[b] + local - s_cnt[b]) * W_txt);
-      dst = reinterpret_cast<uint4*>(packed + (size_t)r * W_txt);
-      n16 = nt16;
+      src[u] = reinterpret_cast<const uint4*>(X + (size_t)(bd.vis_off[vb[u]] + jv[u]) * W_vis) + c0v[u];
     }
-    copy_row(src, dst, n16, lane);
+    uint4 x[PPW][PIECE16 / 32];
+#pragma unroll
+    for (int u = 0; u < PPW; ++u)
+#pragma unroll
+      for (int q = 0; q < PIECE16 / 32; ++q)
+        if (lane + q * 32 < nc[u]) x[u][q] = __ldg(src[u] + lane + q * 32);
+#pragma unroll
+    for (int u = 0; u < PPW; ++u)
+#pragma unroll
+      for (int q = 0; q < PIECE16 / 32; ++q)
+        if (lane + q * 32 < nc[u]) dst[u][lane + q * 32] = x[u][q];
   }
 }
 
@@ -129,9 +161,11 @@ cudaError_t compact_launch(const BatchDesc& bd, const void* X, int W_vis, const 
                            const int* idx, int k_cap, const int* count, void* packed, int* cu,
                            int* pos, void* vis_packed, int* vis_row_map, int* vis_cu, int T_cap,
                            int* err, cudaStream_t st) {
-  const int rows_per_block = NT / 32;
-  int grid = (T_cap + rows_per_block - 1) / rows_per_block;
-  grid = std::max(1, std::min(grid, device_sm_count() * 8));
+  // pieces of at most 2 KB (one per visual row of 1,024 bf16, more for wider
+  // rows), three per warp and pass
+  const long long pieces = (long long)T_cap * ((std::max(W_vis, W_txt) / 8 + 127) / 128);
+  int grid = (int)std::min<long long>((pieces + NT / 32 * 3 - 1) / (NT / 32 * 3), 1 << 20);
+  grid = std::max(1, std::min(grid, device_sm_count() * 2));  // resident: two CTAs per SM
   prof_begin_launch(st);
   compact_kernel<<<grid, NT, 0, st>>>(bd, reinterpret_cast<const __nv_bfloat16*>(X), W_vis,
                                       reinterpret_cast<const __nv_bfloat16*>(text), W_txt, idx, k_cap,
