@@ -458,10 +458,34 @@ def run_ours(args):
     full_idx = torch.arange(576, dtype=torch.int32, device=dev).repeat(w.B, 1).contiguous()
     full_cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
     full_ms = timed(lambda: prefill_stage(full_idx, full_cnt, 576), reps=3)
+    # per-kind split of one full-prefix pass (events around every launch): the
+    # attention at 624-token sequences, where it has enough work to be bound by
+    # the tensor pipe rather than by launch latency
+    B.sp_profile_begin(4000)
+    prefill_stage(full_idx, full_cnt, 576)
+    torch.cuda.synchronize()
+    full_prof = B.sp_profile_end()
+    full_lens = [n + t for n, t in zip(w.n_vis, w.n_txt)]
+    attn_full_flops = 4.0 * m.n_heads * m.head_dim * sum(L * (L + 1) / 2 for L in full_lens) * m.n_layers
+    attn_full_ms = full_prof["attention"]["ms"]
     # compaction at a bandwidth-sized case: every visual token kept (the full prefix)
     full_compact_ms = kernel_ms_cold(lambda: do_compact(full_idx, full_cnt, 576, reuse=True))
     full_T = sum(w.n_vis) + sum(w.n_txt)
     full_comp_bytes = 2.0 * (sum(w.n_vis) * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + full_T)
+    # bandwidth-sized compaction: 128 images, every visual token kept (201 MB
+    # read + 201 MB written, above the L2's 126 MB), timed back to back
+    nbig = 128
+    Xbig = torch.randn((nbig * 576, s.D), device=dev, generator=gen).to(torch.bfloat16)
+    Ebig = (torch.randn((nbig * 48, m.d), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+    big_idx = torch.arange(576, dtype=torch.int32, device=dev).repeat(nbig, 1).contiguous()
+    big_cnt = torch.full((nbig,), 576, dtype=torch.int32, device=dev)
+    big_nv, big_nt = [576] * nbig, [48] * nbig
+    big_out = B.sp_compact(big_nv, big_nt, X=Xbig, text=Ebig, idx=big_idx, count=big_cnt, k_cap=576,
+                           projector_mode=True)
+    big_ms = kernel_ms(lambda: B.sp_compact(big_nv, big_nt, X=Xbig, text=Ebig, idx=big_idx, count=big_cnt,
+                                            k_cap=576, projector_mode=True, out=big_out), reps=10)
+    big_bytes = 2.0 * (nbig * 576 * s.D + nbig * 48 * m.d) * 2 + 4.0 * (nbig + 1 + nbig * 624)
+    del Xbig, Ebig, big_out
 
     # ---- generation over the pruned prefix vs the full prefix (one token per
     #      sequence per step, 32 layers; the cache contents do not change the
@@ -595,6 +619,15 @@ def run_ours(args):
             "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,
             "compaction_full_prefix_gbs": full_comp_bytes / (full_compact_ms * 1e-3) / 1e9,
             "compaction_full_prefix_hbm_frac": full_comp_bytes / (full_compact_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
+            "compaction_128_images_gbs": big_bytes / (big_ms * 1e-3) / 1e9,
+            "compaction_128_images_hbm_frac": big_bytes / (big_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
+            "compaction_note": ("16-image figures: one call after an L2 flush, events around it (launch latency "
+                                "included); 128 images: 402 MB moved per call, back to back"),
+            "attention_full_prefix": {
+                "ms": attn_full_ms, "layers": m.n_layers, "sequences": w.B, "seq_len": full_lens[0],
+                "algorithmic_tflops": attn_full_flops / (attn_full_ms * 1e-3) / 1e12,
+                "frac_of_bf16_burst": attn_full_flops / (attn_full_ms * 1e-3) / 1e12 / pk["bf16"],
+                "note": "causal flops 4 H d_h sum L(L+1)/2 per layer; events around each launch"},
             "pruned_prefill_ms": pruned_ms,
             "full_prefix_prefill_ms": full_ms,
             "speedup_prefill": full_ms / pruned_ms,
