@@ -241,22 +241,20 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         plo[e] = __uint_as_float(pack_bf16x2(p0 - h0, p1 - h1));
       }
       l = l * corr + ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
-      if (i > 0 && __any_sync(0xffffffffu, moved)) {
-        // O is rescaled once P V of the previous block has finished with it.
-        // Without a rescale nothing here waits on that P V: P(i) goes to the
-        // S buffer of block i, released by P V(i - 2) before S(i) was issued.
-        // (o_done has then completed i - 1 or i phases, never i + 1, so its
-        // parity wait stays unambiguous when it is skipped.)
+      if (i > 0) {
+        // P V of the previous block has finished with O
         if (!mbar_wait_warp(o_done, (i - 1) & 1, err)) { ok = false; break; }
         tc_fence_after();
-        float o[32];
+        if (__any_sync(0xffffffffu, moved)) {
+          float o[32];
 #pragma unroll 1
-        for (int c = 0; c < DH; c += 32) {
-          tmem_ld_32x32b_x32(trow + C::T_O + c, o);
-          tmem_ld_wait();
+          for (int c = 0; c < DH; c += 32) {
+            tmem_ld_32x32b_x32(trow + C::T_O + c, o);
+            tmem_ld_wait();
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] *= corr;
-          tmem_st_32x32b_x32(trow + C::T_O + c, o);
+            for (int e = 0; e < 32; ++e) o[e] *= corr;
+            tmem_st_32x32b_x32(trow + C::T_O + c, o);
+          }
         }
       }
       tmem_st_32x32b_x32(trow + st * BKV, phi);

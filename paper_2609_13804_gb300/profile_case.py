@@ -8,6 +8,7 @@ launches).  Shapes are those of the 16-image LLaVA-1.5-7B-shaped batch.
     python -m paper_2609_13804_gb300.profile_case compact    # compaction of the batch
     python -m paper_2609_13804_gb300.profile_case compact_full  # every visual token kept (50 MB)
     python -m paper_2609_13804_gb300.profile_case attention  # 1 decoder layer, like gemm
+    python -m paper_2609_13804_gb300.profile_case attention_full  # 1 layer over the full prefix (16 x 624)
     python -m paper_2609_13804_gb300.profile_case decode     # 4 decoder layers, 16 sequences, 3 steps
 
 Each case runs its stage twice (the second launch set is the one to capture
@@ -28,7 +29,7 @@ def main(case: str):
     dev = torch.device("cuda", 0)
     w = S.llava15_7b_b16()
     counts = S.target_counts(w)
-    if case in ("gemm", "attention", "decode"):
+    if case in ("gemm", "attention", "attention_full", "decode"):
         m = dataclasses.replace(w.model, proj_kind="none", proj_in=w.model.d)
         gen = torch.Generator(device=dev)
         gen.manual_seed(1)
@@ -45,8 +46,10 @@ def main(case: str):
         layers = [L] + [{k: (rnd(v.shape) if v.dtype == torch.bfloat16 else v) for k, v in L.items()}
                         for _ in range(n_layers - 1)]
         m = dataclasses.replace(m, n_layers=n_layers)
-        model = B.Model(m, None, None, dev, max_pos=512, device_weights={"layers": layers, "head": head})
+        model = B.Model(m, None, None, dev, max_pos=1024, device_weights={"layers": layers, "head": head})
         lens = [int(k) + 48 for k in counts]
+        if case == "attention_full":
+            lens = [n + t for n, t in zip(w.n_vis, w.n_txt)]  # every visual token kept: 624 per sequence
         if case == "decode":
             # one generation step per sequence over the pruned prefix (a zeroed
             # cache with the prefix lengths: the contents do not change the work)
@@ -65,8 +68,9 @@ def main(case: str):
         pos = torch.tensor(np.concatenate([np.arange(n) for n in lens]), dtype=torch.int32, device=dev)
         x = (torch.randn((T, m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
         # the caps of the pipeline (k_cap 192 per image) so tile widths match the benchmark's launches
-        T_cap = sum(min(n, w.k_max) + t for n, t in zip(w.n_vis, w.n_txt))
-        len_cap = max(min(n, w.k_max) + t for n, t in zip(w.n_vis, w.n_txt))
+        kc = max(w.n_vis) if case == "attention_full" else w.k_max
+        T_cap = sum(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
+        len_cap = max(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
         xc = torch.zeros((T_cap, m.d), dtype=torch.bfloat16, device=dev)
         xc[:T] = x
         pc = torch.zeros(T_cap, dtype=torch.int32, device=dev)
