@@ -49,12 +49,18 @@ Parity status of each function:
   decode_step, cache_from_prefill       pinned (equals the prefill over the extended
                                         sequences at the new positions, with and
                                         without bf16 storage)
-  projector, prefill_layer, prefill     pinned through their parts plus special cases
-                                        (acc='fp32' variant: pinned against acc='fp64'
-                                        to fp32 precision)
-                                        (zero output weights -> identity; uniform attention);
-                                        the composition of a whole random-weight LM is
-                                        parity unpinned beyond those checks.
+  projector                             pinned (torch nn.Sequential Linear-GELU-Linear)
+  prefill_layer, prefill                pinned (a Llama decoder layer composed from
+                                        torch.nn.functional in fp64: rms_norm, linear,
+                                        complex-rotation RoPE, sdpa with repeated kv
+                                        heads, silu -- GQA, ragged, both halves with
+                                        residuals, with and without bf16 storage; zero
+                                        output weights -> identity; uniform attention;
+                                        varlen isolation and causality; acc='fp32'
+                                        variant against acc='fp64' to fp32 precision)
+  prefill_layer_rows                    pinned (equals prefill_layer at the chosen rows,
+                                        1-D and 3-D positions, with and without storage
+                                        rounding)
 """
 from __future__ import annotations
 
@@ -136,20 +142,23 @@ def softmax(x, axis: int = -1) -> np.ndarray:
     return e / e.sum(axis=axis, keepdims=True)
 
 
-def attention(q, k, v, n_heads: int, n_kv_heads: int, causal: bool) -> np.ndarray:
+def attention(q, k, v, n_heads: int, n_kv_heads: int, causal: bool, q_pos=None) -> np.ndarray:
     """Scaled dot-product attention of one sequence.
 
-    q [L, Hq*dh], k/v [L, Hkv*dh].  Query head i reads key/value head
+    q [Lq, Hq*dh], k/v [L, Hkv*dh].  Query head i reads key/value head
     floor(i * Hkv / Hq) (grouped-query attention; Hkv == Hq is plain MHA).
-    Causal: position p attends to positions 0..p.
+    Causal: the query at position p attends to key positions 0..p.  The query
+    rows are the positions 0..L-1 of the sequence unless q_pos gives their
+    positions (a subset of the sequence's rows).
     """
     q, k, v = _f(q), _f(k), _f(v)
-    L = q.shape[0]
+    Lq, L = q.shape[0], k.shape[0]
     dh = q.shape[1] // n_heads
-    out = np.zeros((L, n_heads * dh), dtype=F64)
-    mask = np.zeros((L, L), dtype=F64)
+    out = np.zeros((Lq, n_heads * dh), dtype=F64)
+    mask = np.zeros((Lq, L), dtype=F64)
     if causal:
-        mask[np.triu_indices(L, 1)] = NEG_INF
+        qp = np.arange(Lq) if q_pos is None else np.asarray(q_pos, dtype=np.int64)
+        mask[np.arange(L)[None, :] > qp[:, None]] = NEG_INF
     for i in range(n_heads):
         j = (i * n_kv_heads) // n_heads
         qi = q[:, i * dh:(i + 1) * dh]
@@ -331,7 +340,8 @@ class _IncrementalDecoder:
 
 
 def select_episode(H, dec: Dict, *, k_max: int, g: int = 1, stop_bias: float = 0.0,
-                   eps: float = 1e-5, mode: str = "incremental") -> Dict:
+                   eps: float = 1e-5, mode: str = "incremental",
+                   force: Optional[Sequence[int]] = None) -> Dict:
     """Algorithm 1, steps 2-3, over one candidate memory.
 
     H: [N, D] encoded visual candidates; M = [H; s_stop] (STOP is row N).
@@ -351,6 +361,18 @@ def select_episode(H, dec: Dict, *, k_max: int, g: int = 1, stop_bias: float = 0
     available visual logits and STOP: the sensitivity of the round's decision)
     and 'gap' (best available visual logit minus the raw STOP logit, before
     stop_bias).
+
+    force: teacher forcing along another implementation's step-order list.
+    Each round takes the next min(g, k_max - |S|, #available) forced indices in
+    the forced order instead of its own TopG, and STOP once the list is used up
+    (with candidates left and |S| < k_max); the logits are those of the forced
+    history.  'slack' then holds, per evaluated round, how far the forced
+    decision is from one this oracle could take: the largest of (the take-th
+    best available logit minus the lowest forced logit), (the STOP logit minus
+    the best available logit: STOP is checked once per round, against the
+    round's best), the largest rise between consecutive forced logits, and for
+    a forced STOP (the best available logit minus the STOP logit); 0 when the
+    forced decision is an exact optimum.
     """
     H = _f(H)
     N = H.shape[0]
@@ -369,6 +391,7 @@ def select_episode(H, dec: Dict, *, k_max: int, g: int = 1, stop_bias: float = 0
     elif mode != "scratch":
         raise ValueError(mode)
 
+    slacks: List[float] = []
     while len(S) < k_max:
         if inc is not None:
             raw = inc.logits()
@@ -381,6 +404,7 @@ def select_episode(H, dec: Dict, *, k_max: int, g: int = 1, stop_bias: float = 0
         if avail.size == 0:
             gaps.append(NEG_INF)
             margins.append(np.inf)
+            slacks.append(0.0)
             stopped = True
             break
         vis = logits[avail]
@@ -391,19 +415,36 @@ def select_episode(H, dec: Dict, *, k_max: int, g: int = 1, stop_bias: float = 0
         top = sorted([float(v) for v in vis[rank[:g + 1]]] + [float(logits[stop])], reverse=True)
         top = top[:g + 1]
         margins.append(min((top[i] - top[i + 1] for i in range(len(top) - 1)), default=np.inf))
-        if logits[stop] > best:
-            stopped = True
-            break
         take = min(g, k_max - len(S), avail.size)
-        U = [int(avail[i]) for i in rank[:take]]
+        if force is not None:
+            if len(S) == len(force):
+                slacks.append(max(0.0, float(best - logits[stop])))
+                stopped = True
+                break
+            U = [int(a) for a in force[len(S):len(S) + take]]
+            if len(U) < take or len(set(U)) < take or any(taken[u] for u in U):
+                raise ValueError("forced actions: too few, repeated or already taken")
+            lu = logits[U]
+            slacks.append(max(0.0, float(vis[rank[take - 1]] - lu.min()), float(logits[stop] - best),
+                              max((float(lu[i + 1] - lu[i]) for i in range(take - 1)), default=0.0)))
+        else:
+            if logits[stop] > best:
+                stopped = True
+                break
+            U = [int(avail[i]) for i in rank[:take]]
         S.extend(U)
         taken[U] = True
         if inc is not None:
             inc.append(M[U])
         else:
             history.extend(M[U])
-    return {"order": S, "count": len(S), "margin": margins, "gap": gaps,
-            "rounds": len(margins), "stopped": stopped}
+    out = {"order": S, "count": len(S), "margin": margins, "gap": gaps,
+           "rounds": len(margins), "stopped": stopped}
+    if force is not None:
+        if len(S) != len(force):
+            raise ValueError("forced list longer than the cap allows")
+        out["slack"] = slacks
+    return out
 
 
 def restore(S: Sequence[int]) -> np.ndarray:
@@ -778,6 +819,41 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
     gu = _mm(x2, _f(L["Wgu"]).T, acc)
     h = h + _mm(_store(silu(gu[:, :F]) * gu[:, F:], store), _f(L["Wdown"]).T, acc)
     return h
+
+
+def prefill_layer_rows(h, L: Dict, m, cu: Sequence[int], pos, rows, store: Optional[str] = None) -> np.ndarray:
+    """prefill_layer's output at the packed rows `rows` only (for sequences of
+    thousands of tokens, where the whole layer is too slow for this oracle).
+
+    Every step of the layer is row-local except the attention, whose query at
+    position p reads the keys and values 0..p of its own sequence.  So the keys
+    and values are projected (and rotated) for every row of the sequences the
+    chosen rows lie in, while the queries, the attention, the output projection,
+    the residuals and the MLP are evaluated for the chosen rows alone, in the
+    same order, with the same storage rounding as prefill_layer.  Returns
+    [len(rows), d] in the order of `rows`."""
+    h = _f(h)
+    rows = np.asarray(rows, dtype=np.int64)
+    cu = np.asarray(cu, dtype=np.int64)
+    Hq, Hkv, dh, F = m.n_heads, m.n_kv_heads, m.head_dim, m.ffn
+    Wqkv = _f(L["Wqkv"])
+    Wq, Wk, Wv = Wqkv[:Hq * dh], Wqkv[Hq * dh:(Hq + Hkv) * dh], Wqkv[(Hq + Hkv) * dh:]
+    seq = np.searchsorted(cu, rows, side="right") - 1
+    out = np.zeros((len(rows), h.shape[1]), dtype=F64)
+    for b in np.unique(seq):
+        s, e = int(cu[b]), int(cu[b + 1])
+        sel = np.flatnonzero(seq == b)
+        r = rows[sel]
+        x = _store(rms_norm(h[s:e], m.rms_eps, L.get("attn_norm")), store)
+        k = _store(_rotary(x @ Wk.T, pos[s:e], Hkv, m), store)
+        v = _store(x @ Wv.T, store)
+        q = _store(_rotary(x[r - s] @ Wq.T, pos[r], Hq, m), store)
+        o = attention(q, k, v, Hq, Hkv, causal=True, q_pos=r - s)
+        hr = h[r] + _store(o, store) @ _f(L["Wo"]).T
+        x2 = _store(rms_norm(hr, m.rms_eps, L.get("mlp_norm")), store)
+        gu = x2 @ _f(L["Wgu"]).T
+        out[sel] = hr + _store(silu(gu[:, :F]) * gu[:, F:], store) @ _f(L["Wdown"]).T
+    return out
 
 
 def final_norm(h, m, gain=None) -> np.ndarray:

@@ -61,8 +61,9 @@ def _deep_case(B, w, *, scale=1.0, targets=None, mean_target=None):
     assert int(out["err"].item()) == 0
     gpu = {k: np_(out[k]) for k in ("order", "ep_count", "rounds", "margin", "gap", "idx", "count")}
     images = PT.oracle_select(H, w.n_vis, sel, k_max=w.k_max, g=1, group_size=w.group_size, biases=biases)
+    replay, eps_list = PT.replayer(H, w.n_vis, sel, k_max=w.k_max, g=1, group_size=w.group_size, biases=biases)
     report = []
-    near = PT.compare_selection(gpu, images, g=1, report=report)
+    near = PT.compare_selection(gpu, images, g=1, report=report, replay=replay, episodes=eps_list)
     for r in report:
         print("near-tie:", r)
     selector.close()

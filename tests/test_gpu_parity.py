@@ -53,8 +53,9 @@ def _run_select_case(B, w, *, scale=1.0, ln_affine=True, targets=None, seed_bias
     gpu = {k: np_(out[k]) for k in ("order", "ep_count", "rounds", "margin", "gap", "idx", "count")}
     np.testing.assert_array_equal(np_(out["memory"]), H)
     images = PT.oracle_select(H, w.n_vis, sel, k_max=w.k_max, g=w.g, group_size=w.group_size, biases=biases)
+    replay, eps_list = PT.replayer(H, w.n_vis, sel, k_max=w.k_max, g=w.g, group_size=w.group_size, biases=biases)
     report = []
-    near = PT.compare_selection(gpu, images, g=w.g, report=report)
+    near = PT.compare_selection(gpu, images, g=w.g, report=report, replay=replay, episodes=eps_list)
     for r in report:
         print("near-tie:", r)
     # invariants that hold whatever the ties did

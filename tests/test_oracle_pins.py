@@ -350,6 +350,58 @@ def test_candidate_groups_are_independent_episodes():
     assert list(img["idx"]) == sorted(want)
 
 
+@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("g", [1, 3])
+def test_forcing_the_own_order_changes_nothing(seed, g):
+    sel, H = _scaled_selector(400 + seed, N=17)
+    for bias in (-0.3, 0.1, -1e9):
+        for k_max in (5, 40):
+            r = O.select_episode(H, sel, k_max=k_max, g=g, stop_bias=bias)
+            f = O.select_episode(H, sel, k_max=k_max, g=g, stop_bias=bias, force=r["order"])
+            assert f["order"] == r["order"] and f["rounds"] == r["rounds"] and f["stopped"] == r["stopped"]
+            assert f["gap"] == r["gap"] and f["margin"] == r["margin"]
+            assert all(x == 0.0 for x in f["slack"])
+
+
+@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("g", [1, 2])
+def test_forced_slack_equals_brute_force_rescoring(seed, g):
+    """Along an arbitrary forced trajectory the slack of every round is the
+    distance of the forced decision from an optimal one, rescoring all
+    candidates from scratch over the forced history (written from Alg. 1 and
+    Eq. 11, without the oracle's episode loop)."""
+    sel, H = _scaled_selector(500 + seed, N=12)
+    N = H.shape[0]
+    rng = np.random.default_rng(seed)
+    k_max, bias = 9, -0.2
+    force = [int(x) for x in rng.permutation(N)[:int(rng.integers(0, k_max + 1))]]
+    f = O.select_episode(H, sel, k_max=k_max, g=g, stop_bias=bias, force=force)
+    M = np.concatenate([H, sel["s_stop"][None].astype(np.float64)])
+    hist, done, want = [sel["s_start"].astype(np.float64)], [], []
+    while len(done) < k_max:
+        l = O.pointer_logits_from_scratch(np.stack(hist), M, sel, 1e-5)
+        l[N] += bias
+        av = sorted((l[j] for j in range(N) if j not in done), reverse=True)
+        if not av:
+            want.append(0.0)
+            break
+        if len(done) == len(force):
+            want.append(max(0.0, av[0] - l[N]))
+            break
+        take = min(g, k_max - len(done), len(av))
+        U = force[len(done):len(done) + take]
+        lu = [l[u] for u in U]
+        rise = max([lu[i + 1] - lu[i] for i in range(take - 1)] + [0.0])
+        want.append(max(0.0, av[take - 1] - min(lu), l[N] - av[0], rise))
+        done += U
+        hist += [M[u] for u in U]
+    assert f["order"] == force
+    np.testing.assert_allclose(f["slack"], want, atol=1e-12)
+    assert max(want) > 0.0  # a random trajectory is not the greedy one
+    with pytest.raises(ValueError):
+        O.select_episode(H, sel, k_max=k_max, g=1, stop_bias=bias, force=[0, 0])
+
+
 # ---------------------------------------------------------------- compaction (Alg. 1 step 5)
 
 def test_compaction_golden_fixture():
@@ -498,6 +550,91 @@ def test_prefill_layer_uniform_attention_closed_form():
         for p in range(s, e):
             want[p] = v[s:p + 1].mean(axis=0)
     np.testing.assert_allclose(out - x, want, atol=1e-12)
+
+
+def _torch_llama_layer(h, L, m, lens, store=None):
+    """A Llama decoder layer over packed sequences assembled from
+    torch.nn.functional in fp64: rms_norm, linear, rotary as a complex rotation
+    of the (i, i + dh/2) pairs (torch.polar), scaled_dot_product_attention with
+    the key / value heads repeated for their query groups, silu.  With
+    store='bf16' the same tensors the oracle stores as bf16 are rounded."""
+    F = torch.nn.functional
+    rnd = (lambda t: t.float().to(torch.bfloat16).double()) if store == "bf16" else (lambda t: t)
+    dq, dkv, half = m.n_heads * m.head_dim, m.n_kv_heads * m.head_dim, m.head_dim // 2
+    Wq, Wk, Wv = t64(L["Wqkv"]).split([dq, dkv, dkv])
+    Wg, Wu = t64(L["Wgu"]).split([m.ffn, m.ffn])
+    inv = m.rope_theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / m.head_dim)
+    H, out, s0 = t64(h), [], 0
+    for n in lens:
+        hs = H[s0:s0 + n]
+        s0 += n
+        rot = torch.polar(torch.ones(n, half), torch.arange(n, dtype=torch.float64)[:, None] * inv[None, :])
+
+        def rope(t):
+            z = torch.complex(t[..., :half], t[..., half:]) * rot[:, None, :]
+            return torch.cat([z.real, z.imag], dim=-1)
+
+        x = rnd(F.rms_norm(hs, (m.d,), t64(L["attn_norm"]), m.rms_eps))
+        q = rnd(rope(F.linear(x, Wq).view(n, m.n_heads, m.head_dim)))
+        k = rnd(rope(F.linear(x, Wk).view(n, m.n_kv_heads, m.head_dim)))
+        v = rnd(F.linear(x, Wv).view(n, m.n_kv_heads, m.head_dim))
+        rep = m.n_heads // m.n_kv_heads
+        o = F.scaled_dot_product_attention(q.transpose(0, 1), k.transpose(0, 1).repeat_interleave(rep, 0),
+                                           v.transpose(0, 1).repeat_interleave(rep, 0), is_causal=True)
+        hs = hs + F.linear(rnd(o.transpose(0, 1).reshape(n, dq)), t64(L["Wo"]))
+        x2 = rnd(F.rms_norm(hs, (m.d,), t64(L["mlp_norm"]), m.rms_eps))
+        hs = hs + F.linear(rnd(F.silu(F.linear(x2, Wg)) * F.linear(x2, Wu)), t64(L["Wdown"]))
+        out.append(hs)
+    return torch.cat(out).numpy()
+
+
+@pytest.mark.parametrize("hq,hkv,store", [(4, 2, None), (4, 4, None), (6, 1, None), (4, 2, "bf16")])
+def test_prefill_layer_matches_torch_llama_layer(hq, hkv, store):
+    """The whole LM layer, attention and SwiGLU halves with their residuals,
+    against the torch composition: GQA, ragged sequences (one of length 1),
+    non-trivial norm gains, weights large enough that the MLP moves the
+    residual as much as the attention does."""
+    w = S.tiny_workload(19, [5], [2], d=48, n_heads=hq, n_kv_heads=hkv, head_dim=8, ffn=56)
+    m = w.model
+    L = S.make_layer_weights(w, 0, norm_affine=True)
+    for k in ("Wqkv", "Wo", "Wgu", "Wdown"):
+        L[k] = L[k] / 0.02 * 0.2
+    lens = [5, 1, 9, 4]
+    x = S.normal(19, "x", (sum(lens), m.d)).astype(np.float64)
+    cu = np.r_[0, np.cumsum(lens)]
+    pos = np.concatenate([np.arange(n) for n in lens])
+    got = O.prefill_layer(x, L, m, cu, pos, store=store)
+    want = _torch_llama_layer(x, L, m, lens, store=store)
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-10)
+    # both halves move the residual: the pin sees the MLP, not only the attention
+    L0 = dict(L, Wdown=np.zeros_like(L["Wdown"]))
+    assert np.abs(O.prefill_layer(x, L0, m, cu, pos) - got).max() > 0.1
+
+
+@pytest.mark.parametrize("store,mrope", [(None, False), ("bf16", False), (None, True)])
+def test_prefill_layer_rows_equals_the_whole_layer(store, mrope):
+    """The row-sampled layer (keys / values of the whole sequence, the rest at
+    the chosen rows) equals the whole layer at those rows."""
+    w = S.tiny_workload(20, [5], [2], d=32, n_heads=4, n_kv_heads=2, head_dim=8, ffn=40)
+    m = w.model
+    if mrope:
+        m = dataclasses.replace(m, mrope_section=(2, 1, 1))
+    L = S.make_layer_weights(w, 0, norm_affine=True)
+    for k in ("Wqkv", "Wo", "Wgu", "Wdown"):
+        L[k] = L[k] / 0.02 * 0.2
+    lens = [7, 1, 12, 5]
+    T = sum(lens)
+    x = S.normal(20, "x", (T, m.d)).astype(np.float64)
+    cu = np.r_[0, np.cumsum(lens)]
+    pos = np.concatenate([np.arange(n) for n in lens])
+    if mrope:
+        pos = np.stack([pos, pos // 3, pos % 3], axis=1).astype(np.float64)
+    full = O.prefill_layer(x, L, m, cu, pos, store=store)
+    rows = np.array([0, 3, 6, 7, 8, 9, 15, 19, 20, 24])
+    got = O.prefill_layer_rows(x, L, m, cu, pos, rows, store=store)
+    np.testing.assert_allclose(got, full[rows], rtol=0, atol=1e-10 if store is None else 1e-2)
+    if store == "bf16":  # a rounding boundary may flip between the two matmul shapes, rarely
+        assert np.mean(np.abs(got - full[rows]) < 1e-10) > 0.95
 
 
 def test_prefill_varlen_isolation_and_causality():
