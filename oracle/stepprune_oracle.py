@@ -25,7 +25,9 @@ Readings of points the paper leaves open are stated at each function (see the
 Parity status of each function:
   layer_norm, rms_norm, gelu, silu      pinned (torch.nn.functional, closed forms)
   attention                             pinned (torch scaled_dot_product_attention, brute force)
-  text_projection, encoder              pinned (torch.nn.TransformerEncoderLayer, fp64)
+  text_projection, encoder              pinned (torch.nn.TransformerEncoderLayer, fp64; the
+                                        bf16-storage variant against a torch.nn.functional
+                                        composition rounding the same tensors)
   pointer logits / select_episode       pinned (brute-force from-scratch decoder; torch
                                         nn.MultiheadAttention decoder; deeper decoders against
                                         torch nn.TransformerDecoderLayer; history-free top-K
@@ -182,24 +184,27 @@ def text_projection(E_text, sel: Dict, eps: float, g_text: float = 1.0) -> np.nd
     return g_text * layer_norm(P, eps, sel.get("ln_text_g"), sel.get("ln_text_b"))
 
 
-def encoder_block(x, L: Dict, n_heads: int, eps: float) -> np.ndarray:
+def encoder_block(x, L: Dict, n_heads: int, eps: float, store: Optional[str] = None) -> np.ndarray:
     """One pre-norm ViT block with bidirectional self-attention (Sec. 3.2; the
     bidirectional mask is the default of Table 7(a)).
 
-    Reading: no linear biases; MLP is W2 GELU(W1 x) with exact GELU.
+    Reading: no linear biases; MLP is W2 GELU(W1 x) with exact GELU.  The
+    residual stream stays fp64; with store='bf16' the activations a bf16 model
+    keeps between ops (normalised inputs, q / k / v, attention output, GELU
+    output) are rounded to bf16 where they are stored.
     """
     x = _f(x)
     D = x.shape[1]
-    a = layer_norm(x, eps, L.get("ln1_g"), L.get("ln1_b"))
-    qkv = a @ _f(L["Wqkv"]).T
+    a = _store(layer_norm(x, eps, L.get("ln1_g"), L.get("ln1_b")), store)
+    qkv = _store(a @ _f(L["Wqkv"]).T, store)
     o = attention(qkv[:, :D], qkv[:, D:2 * D], qkv[:, 2 * D:], n_heads, n_heads, causal=False)
-    x = x + o @ _f(L["Wo"]).T
-    m = layer_norm(x, eps, L.get("ln2_g"), L.get("ln2_b"))
-    x = x + gelu(m @ _f(L["W1"]).T) @ _f(L["W2"]).T
+    x = x + _store(o, store) @ _f(L["Wo"]).T
+    m = _store(layer_norm(x, eps, L.get("ln2_g"), L.get("ln2_b")), store)
+    x = x + _store(gelu(m @ _f(L["W1"]).T), store) @ _f(L["W2"]).T
     return x
 
 
-def encoder(X, E_tilde, sel: Dict, n_heads: int, eps: float) -> np.ndarray:
+def encoder(X, E_tilde, sel: Dict, n_heads: int, eps: float, store: Optional[str] = None) -> np.ndarray:
     """H = Enc([X; E~_text])_[1:N] (Eq. 3): joint encoding, visual rows kept.
 
     Reading: the blocks are followed by no final norm.
@@ -207,7 +212,7 @@ def encoder(X, E_tilde, sel: Dict, n_heads: int, eps: float) -> np.ndarray:
     X = _f(X)
     x = np.concatenate([X, _f(E_tilde)], axis=0)
     for L in sel["enc"]:
-        x = encoder_block(x, L, n_heads, eps)
+        x = encoder_block(x, L, n_heads, eps, store)
     return x[:X.shape[0]]
 
 

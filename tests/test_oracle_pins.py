@@ -108,6 +108,38 @@ def test_encoder_matches_torch_transformer_encoder_layer():
     assert H.shape == (10, s.D)
 
 
+@pytest.mark.parametrize("store", [None, "bf16"])
+def test_encoder_storage_variant_matches_torch_functional(store):
+    """The encoder block assembled from torch.nn.functional (layer_norm, linear,
+    sdpa over heads, gelu) in fp64, rounding to bf16 the same tensors as the
+    oracle's store='bf16' (the normalised inputs, q / k / v, the attention
+    output, the GELU output); residuals unrounded."""
+    F = torch.nn.functional
+    w = S.tiny_workload(5, [9], [4], D=32, D_text=48, enc_head_dim=8)
+    sel = S.make_selector_weights(w, ln_affine=True)
+    for L in sel["enc"]:
+        for k in ("Wqkv", "Wo", "W1", "W2"):
+            L[k] = L[k] / 0.02 * 0.2
+    s = w.selector
+    X = S.normal(5, "X", (9, s.D)).astype(np.float64)
+    Et = S.normal(5, "Et", (4, s.D)).astype(np.float64)
+    got = O.encoder(X, Et, sel, s.enc_heads, s.ln_eps, store=store)
+    rnd = (lambda t: t.float().to(torch.bfloat16).double()) if store == "bf16" else (lambda t: t)
+    x = t64(np.concatenate([X, Et]))
+    n, D, nh = x.shape[0], s.D, s.enc_heads
+    for L in sel["enc"]:
+        a = rnd(F.layer_norm(x, (D,), t64(L["ln1_g"]), t64(L["ln1_b"]), s.ln_eps))
+        q, k, v = rnd(F.linear(a, t64(L["Wqkv"]))).split(D, dim=1)
+        heads = [t.view(n, nh, D // nh).transpose(0, 1) for t in (q, k, v)]
+        o = F.scaled_dot_product_attention(*heads).transpose(0, 1).reshape(n, D)
+        x = x + F.linear(rnd(o), t64(L["Wo"]))
+        m = rnd(F.layer_norm(x, (D,), t64(L["ln2_g"]), t64(L["ln2_b"]), s.ln_eps))
+        x = x + F.linear(rnd(F.gelu(F.linear(m, t64(L["W1"])))), t64(L["W2"]))
+    np.testing.assert_allclose(got, x[:9].numpy(), rtol=0, atol=1e-10)
+    if store == "bf16":
+        assert np.abs(got - O.encoder(X, Et, sel, s.enc_heads, s.ln_eps)).max() > 1e-4
+
+
 # ---------------------------------------------------------------- pointer decoder (Eq. 4)
 
 def _scaled_selector(seed, N=14, D=24, h=16, scale=0.3, ln_affine=True):
