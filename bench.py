@@ -53,6 +53,53 @@ def gemm_traffic():
     return GEMM_TRAFFIC["bytes_per_launch"] if h.hexdigest()[:16] == GEMM_TRAFFIC["sources_sha256_16"] else None
 
 
+PROBES_SRC = os.path.join(ROOT, "bench_probes.cu")
+PROBES_LIB = os.path.join(ROOT, "bench_probes.so")
+
+
+def build_probes() -> str:
+    """Compiles bench_probes.cu (the on-chip peak and synchronisation-floor
+    probes this script reports against) for sm_103a, next to this file."""
+    if os.path.exists(PROBES_LIB) and os.path.getmtime(PROBES_LIB) >= os.path.getmtime(PROBES_SRC):
+        return PROBES_LIB
+    from paper_2609_13804_gb300.build import _nvcc, ARCH
+    tmp = PROBES_LIB + ".tmp"
+    subprocess.run([_nvcc(), *ARCH, "-O3", "-std=c++17", "-shared", "-Xcompiler", "-fPIC", PROBES_SRC, "-o", tmp],
+                   check=True, capture_output=True, text=True)
+    os.replace(tmp, PROBES_LIB)
+    return PROBES_LIB
+
+
+class Probes:
+    """ctypes view of bench_probes.so."""
+
+    def __init__(self):
+        import ctypes as C
+        self.C = C
+        self.lib = C.CDLL(build_probes())
+        for n in ("bench_probe_smem_gbs", "bench_probe_l2_gbs"):
+            getattr(self.lib, n).argtypes = [C.POINTER(C.c_double)]
+            getattr(self.lib, n).restype = C.c_int
+        self.lib.bench_probe_select_floor.argtypes = [C.c_int, C.c_int, C.c_int, C.c_int, C.POINTER(C.c_double)]
+        self.lib.bench_probe_select_floor.restype = C.c_int
+
+    def _call(self, fn, *args):
+        v = self.C.c_double()
+        rc = fn(*args, self.C.byref(v))
+        if rc != 0:
+            raise RuntimeError(f"{fn.__name__}: CUDA error {rc}")
+        return v.value
+
+    def smem_gbs(self):
+        return self._call(self.lib.bench_probe_smem_gbs)
+
+    def l2_gbs(self):
+        return self._call(self.lib.bench_probe_l2_gbs)
+
+    def select_floor(self, cluster_size, h, rounds, episodes):
+        return self._call(self.lib.bench_probe_select_floor, cluster_size, h, rounds, episodes)
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -159,42 +206,50 @@ def gemm_flops(w, T, K_sum, T_enc, n_txt_sum):
 _SAMPLE_CACHE = {}
 
 
-def cpu_oracle_sample(w, n_images=1, n_layers=1):
-    """Times the oracle on a bounded sample of the workload and scales it to one
-    batch: per image the encoder + selection, the projector on its kept rows and
-    n_layers of the 32 decoder layers (weights are drawn once, outside the timing)."""
+def cpu_oracle_sample(w, b=0, n_layers=1):
+    """Times the oracle on a bounded sample of the workload: image b through
+    the text projection, the encoder and the selection with that image's
+    calibrated STOP bias (the GPU's kept-count target for it), the projector on
+    its kept rows, and n_layers of the 32 decoder layers over its packed
+    sequence.  Weights are drawn and the bias calibrated once, outside the
+    timing.  Returns (the batch time extrapolated from the sample in ms, the
+    measured parts in seconds)."""
     from oracle import core as O
     s, m = w.selector, w.model
     key = (w.name, n_layers)
     if key not in _SAMPLE_CACHE:
         _SAMPLE_CACHE[key] = (S.make_selector_weights(w), S.make_model_head(w), S.make_inputs(w),
-                              [S.make_layer_weights(w, l) for l in range(n_layers)])
-    sel, head, inp, layers = _SAMPLE_CACHE[key]
+                              [S.make_layer_weights(w, l) for l in range(n_layers)], {})
+    sel, head, inp, layers, biases = _SAMPLE_CACHE[key]
     n_heads = s.D // s.enc_head_dim
-    t_sel = t_proj = t_lm = 0.0
-    for b in range(n_images):
-        v0, t0 = b * w.n_vis[0], b * w.n_txt[0]
-        X = inp["X"][v0:v0 + w.n_vis[b]]
-        E = inp["E_text"][t0:t0 + w.n_txt[b]]
-        t = time.perf_counter()
+    v0, t0 = sum(w.n_vis[:b]), sum(w.n_txt[:b])
+    X = inp["X"][v0:v0 + w.n_vis[b]]
+    E = inp["E_text"][t0:t0 + w.n_txt[b]]
+    if b not in biases:
         Et = O.text_projection(E, sel, s.ln_eps, s.g_text)
         H = O.encoder(X, Et, sel, n_heads, s.ln_eps)
-        r = O.select_episode(H, sel, k_max=w.k_max, g=w.g, stop_bias=0.0, eps=s.ln_eps)
-        idx = O.restore(r["order"])
-        if len(idx) < int(w.target_mean_k):  # time a mean-sized prefix whatever this bias kept
-            idx = np.arange(int(w.target_mean_k))
-        t_sel += time.perf_counter() - t
-        t = time.perf_counter()
-        vis = O.projector(X[idx], head)
-        t_proj += time.perf_counter() - t
-        x = np.concatenate([vis, E])
-        cu, pos = np.array([0, len(x)]), np.arange(len(x))
-        t = time.perf_counter()
-        for L in layers:
-            x = O.prefill_layer(x, L, m, cu, pos)
-        t_lm += time.perf_counter() - t
-    per_image_ms = 1e3 * (t_sel + t_proj + t_lm * m.n_layers / n_layers) / n_images
-    return per_image_ms * w.B, t_sel + t_proj + t_lm
+        free = O.select_episode(H, sel, k_max=w.k_max, g=w.g, stop_bias=-1e30, eps=s.ln_eps)
+        bias, _ = S.stop_biases([free["gap"]], [int(S.target_counts(w)[b])], g=w.g, k_max=w.k_max,
+                                n_cand=[w.n_vis[b]])
+        biases[b] = float(bias[0])
+    t = time.perf_counter()
+    Et = O.text_projection(E, sel, s.ln_eps, s.g_text)
+    H = O.encoder(X, Et, sel, n_heads, s.ln_eps)
+    r = O.select_episode(H, sel, k_max=w.k_max, g=w.g, stop_bias=biases[b], eps=s.ln_eps)
+    idx = O.restore(r["order"])
+    t_sel = time.perf_counter() - t
+    t = time.perf_counter()
+    vis = O.projector(X[idx], head)
+    t_proj = time.perf_counter() - t
+    x = np.concatenate([vis, E])
+    cu, pos = np.array([0, len(x)]), np.arange(len(x))
+    t = time.perf_counter()
+    for L in layers:
+        x = O.prefill_layer(x, L, m, cu, pos)
+    t_lm = (time.perf_counter() - t) / n_layers
+    per_image_ms = 1e3 * (t_sel + t_proj + t_lm * m.n_layers)
+    return per_image_ms * w.B, {"select_s": t_sel, "projector_s": t_proj, "layer_s": t_lm, "kept": int(len(idx)),
+                                "image": b}
 
 
 def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
@@ -205,7 +260,7 @@ def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
     enter the round (the last position's query and residual rows, the key and
     value rows of the positions appended); the kernel's time is the longest
     episode's rounds.  Peaks and the synchronisation floor come from the
-    library's probes."""
+    probes of bench_probes.cu."""
     r = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bias, group_size=w.group_size, g=w.g,
                     k_max=w.k_max)
     import torch
@@ -226,10 +281,11 @@ def selection_report(B, w, selector, X, E, bias, kernel_ms, dev):
             tmem_b += 2.0 * in_tmem * h * 4.0
             l2_b += 2.0 * (t - in_tmem) * h * 4.0 + 2.0 * h * 4.0
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    smem_peak = B.probe_smem_gbs()
-    l2_peak = B.probe_l2_gbs()
+    probes = Probes()
+    smem_peak = probes.smem_gbs()
+    l2_peak = probes.l2_gbs()
     r_max = int(rounds.max())
-    floor_us = B.probe_select_floor(C, h, max(r_max, 1), len(eps))
+    floor_us = probes.select_floor(C, h, max(r_max, 1), len(eps))
     ks = kernel_ms * 1e-3
     used = min(len(eps) * C, sms) / sms
     onchip = smem_b + tmem_b + l2_b
@@ -256,22 +312,30 @@ def run_reference(args):
     if rank != 0:
         return
     w = S.llava15_7b_b16()
-    samples = []
-    wall = 0.0
+    samples, parts = [], []
     for i in range(args.warmup + args.steps):
-        v, secs = cpu_oracle_sample(w)
-        wall += secs
+        v, part = cpu_oracle_sample(w, b=i % w.B)
         if i >= args.warmup:
             samples.append(v)
+            parts.append(part)
     value = statistics.median(samples)
-    sample = ("per step: 1 of 16 images through text projection + 2-block encoder + selection, projector on "
-              "its kept rows, 1 of 32 decoder layers; scaled to 16 images x 32 layers")
+    sample = ("per step: one of the 16 images (in turn) through text projection + 2-block encoder + selection with "
+              "its calibrated STOP bias, the projector on its kept rows and 1 of the 32 decoder layers over its "
+              "packed sequence; extrapolated to 16 images x 32 layers")
+    measured = {"select_s_median": statistics.median(p["select_s"] for p in parts),
+                "projector_s_median": statistics.median(p["projector_s"] for p in parts),
+                "layer_s_median": statistics.median(p["layer_s"] for p in parts),
+                "kept": [p["kept"] for p in parts]}
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": value, "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "images": w.B, "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
                        "layers": w.model.n_layers},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle", "sample": sample},
+            "extrapolated": True, "samples_timed": len(samples), "measured": measured,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle", "sample": sample,
+                             "extrapolated": True,
+                             "threads": "numpy's BLAS may spread a matmul over the cores; the selection and "
+                                        "attention loops run on one"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -307,7 +371,7 @@ def run_ours(args):
     head = {"final_norm": torch.ones(m.d, device=dev),
             "proj_W1": (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16),
             "proj_W2": (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)}
-    model = B.Model(m, layers, head, dev, max_pos=1024)
+    model = B.Model(m, layers, head, dev, max_pos=4096)
     inp = S.make_inputs(w)
     X = B.dev_bf16(inp["X"], dev)
     E = B.dev_bf16(inp["E_text"], dev)
@@ -588,13 +652,25 @@ def run_ours(args):
     h2d = Xh.numel() * 2 + Eh.numel() * 2 + bh.numel() * 4
     d2h = oi.numel() * 4 + oc.numel() * 4 + ocu.numel() * 4 + oh.numel() * 4
 
+    # ---- the other workloads (their own weights and inputs, drawn on the
+    #      device) and the scaling table, outside the timed region
+    workloads = scaling = None
+    if not args.no_configs:
+        workloads = measure_workloads(B, torch, dev, gen, peaks(), model)
+        scaling = {"sweep": "visual-prefix length at 10% retention, one image, llava15-7b dims, 32 layers",
+                   "steps": 3, "warmup": 1, "paper_gpu": "RTX PRO 6000 Blackwell (the paper's; context only)",
+                   "rows": scaling_rows(B, torch, dev, gen, selector, model, 3, 1)}
+
     if rank == 0:
         cpu_line = None
         if world == 1 and not args.no_cpu:
-            v, secs = cpu_oracle_sample(w)
-            cpu_line = {"value": v, "unit": UNIT, "cores": cores(), "kind": "oracle",
-                        "sample": "1 of 16 images (encoder + selection, projector, 1 of 32 layers), scaled to "
-                                  f"16 images x 32 layers; {secs:.1f} s of CPU work"}
+            v, part = cpu_oracle_sample(w)
+            cpu_line = {"value": v, "unit": UNIT, "cores": cores(), "kind": "oracle", "extrapolated": True,
+                        "measured": part,
+                        "threads": "numpy's BLAS may spread a matmul over the cores; the selection and attention "
+                                   "loops run on one",
+                        "sample": "image 0 (encoder + selection with its calibrated STOP bias, projector on its "
+                                  "kept rows, 1 of 32 layers), extrapolated to 16 images x 32 layers"}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": False, "scaling": "weak",
@@ -652,10 +728,260 @@ def run_ours(args):
                 "select_1_layer_ms": deep[1], "select_2_layers_ms": deep[2], "rounds": w.k_max,
                 "us_per_round_1_layer": 1e3 * deep[1] / w.k_max, "us_per_round_2_layers": 1e3 * deep[2] / w.k_max,
                 "note": "16 episodes x 192 rounds from a given memory H (precompute GEMMs included)"},
+            "workloads": workloads,
+            "scaling_table": scaling,
         }
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
+
+
+# ----------------------------------------------------------------------------- per-workload measurements
+
+def device_selector_weights(s, dev, gen, torch):
+    """Selector weights drawn on the device (timing only), with the
+    distributions of synth.make_selector_weights: N(0, 0.02) matrices (bf16 for
+    the encoder and the text projection, fp32 for the pointer decoder), unit
+    LayerNorm gains and zero biases."""
+    def bf(shape):
+        return (torch.randn(shape, device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+
+    def f32(shape):
+        return torch.randn(shape, device=dev, generator=gen) * 0.02
+
+    def ones(n):
+        return torch.ones(n, device=dev)
+
+    def zeros(n):
+        return torch.zeros(n, device=dev)
+
+    D, Dt, h, F = s.D, s.D_text, s.h, s.enc_ffn
+    out = {"W_p": bf((D, Dt)), "ln_text_g": ones(D), "ln_text_b": zeros(D), "enc": [],
+           "s_stop": f32((D,)), "s_start": f32((D,)), "W_in": f32((h, D)), "ln1_g": ones(h), "ln1_b": zeros(h),
+           "ln2_g": ones(h), "ln2_b": zeros(h), "Wk_p": f32((h, D))}
+    for n in ("Wq_s", "Wk_s", "Wv_s", "Wo_s", "Wq_p"):
+        out[n] = f32((h, h))
+    for _ in range(s.n_enc_layers):
+        out["enc"].append({"ln1_g": ones(D), "ln1_b": zeros(D), "Wqkv": bf((3 * D, D)), "Wo": bf((D, D)),
+                           "ln2_g": ones(D), "ln2_b": zeros(D), "W1": bf((F, D)), "W2": bf((D, F))})
+    return out
+
+
+def device_model(B, m, dev, gen, torch, max_pos):
+    layers = [device_layer_weights(m, l, dev, gen, torch) for l in range(m.n_layers)]
+    head = {"final_norm": torch.ones(m.d, device=dev), "proj_W1": None, "proj_W2": None}
+    if m.proj_kind == "linear":
+        head["proj_W1"] = (torch.randn((m.d, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+    elif m.proj_kind == "mlp2":
+        head["proj_W1"] = (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+        head["proj_W2"] = (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+    return B.Model(m, layers, head, dev, max_pos=max_pos)
+
+
+def attn_flops(m, lens, causal=True):
+    """Algorithmic attention flops of one layer: 4 H d_h sum L(L+1)/2 causal,
+    4 H d_h sum L^2 bidirectional."""
+    if causal:
+        return 4.0 * m.n_heads * m.head_dim * sum(L * (L + 1) / 2 for L in lens)
+    return 4.0 * m.n_heads * m.head_dim * sum(L * L for L in lens)
+
+
+class Timing:
+    """CUDA-event timers on the current stream (warmed, synchronised on both sides)."""
+
+    def __init__(self, torch, dev):
+        self.torch = torch
+        self.flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # twice the L2
+
+    def timed(self, fn, reps=3, warm=1):
+        torch = self.torch
+        for _ in range(warm):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    def cold(self, fn, reps=5):
+        """One call after an L2 flush, a spin kernel ahead so the host has
+        enqueued the events and the call before the GPU reaches them."""
+        torch = self.torch
+        fn()
+        total = 0.0
+        for _ in range(reps):
+            self.flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(1_000_000)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            total += a.elapsed_time(b)
+        return total / reps
+
+    def profiled(self, B, fn):
+        """Per-kernel-kind event time of one call (events around every launch)."""
+        B.sp_profile_begin(20000)
+        fn()
+        self.torch.cuda.synchronize()
+        return B.sp_profile_end()
+
+
+def measure_config(B, torch, tm, w, model, dev, gen, pk, *, targets, mean_target, reps=2):
+    """One workload end to end on device-drawn weights and inputs: STOP biases
+    calibrated for the targets; the whole pipeline; selection alone (us per
+    image); compaction (GB/s, HBM fraction, one call after an L2 flush); the
+    pruned prefill (compaction + projector + prefill) against the full-prefix
+    prefill on the same kernels; GEMM and attention flop rates from per-launch
+    events against the measured bf16 peak."""
+    s, m = w.selector, w.model
+    sel = B.Selector(s, device_selector_weights(s, dev, gen, torch), dev)
+    X = torch.randn((sum(w.n_vis), s.D), device=dev, generator=gen).to(torch.bfloat16)
+    E = (torch.randn((sum(w.n_txt), s.D_text), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+    eps = w.episodes()
+    n_ep = len(eps)
+    cal = B.sp_select(sel, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=B.dev_f32(np.full(n_ep, -1e30), dev),
+                      group_size=w.group_size, g=w.g, k_max=w.k_max)
+    torch.cuda.synchronize()
+    gaps, rounds = cal["gap"].cpu().numpy(), cal["rounds"].cpu().numpy()
+    biases, _ = S.stop_biases([gaps[e, :rounds[e]] for e in range(n_ep)], targets, g=w.g, k_max=w.k_max,
+                              n_cand=[n for (_, _, n) in eps], mean_target=mean_target)
+    bias = B.dev_f32(biases, dev)
+    pipe = B.Pipeline(sel, model, w.n_vis, w.n_txt, group_size=w.group_size, g=w.g, k_max=w.k_max)
+    pipe_ms = tm.timed(lambda: pipe(X, E, bias), reps=reps, warm=2)
+    assert int(pipe.err.item()) == 0
+    counts = pipe.count.cpu().numpy().astype(int)
+    T = int(pipe.cu[-1].item())
+    K_sum = int(counts.sum())
+    lens = [int(k) + t for k, t in zip(counts, w.n_txt)]
+    sws = {}
+
+    def select():
+        r = B.sp_select(sel, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bias, group_size=w.group_size, g=w.g,
+                        k_max=w.k_max, traces=False, ws=sws.get("ws"))
+        sws["ws"], sws["r"] = r["_ws"], r
+    select_ms = tm.timed(select, reps=reps)
+    proj = m.proj_kind != "none"
+    comp = {}
+
+    def compact(idx, count, kc, key):
+        comp[key] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
+                                 projector_mode=proj, out=comp.get(key))
+        return comp[key]
+
+    r = sws["r"]
+    compact_ms = tm.cold(lambda: compact(r["idx"], r["count"], pipe.k_cap, "p"))
+    vis_w = s.D
+    comp_bytes = 2.0 * (K_sum * vis_w + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
+    st = {}
+
+    def prefill_stage(idx, count, kc, key):
+        o = compact(idx, count, kc, key)
+        if proj:
+            B.sp_project(model, vis_packed=o["vis_packed"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
+                         packed=o["packed"], rows_cap=o["rows_cap"], B=w.B, ws=st.get(key + "pw"))
+        lens_cap = max(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
+        res = B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=w.B, T_cap=o["T_cap"],
+                           max_seqlen_cap=lens_cap, ws=st.get(key + "ws"), hidden=st.get(key + "h"))
+        st[key + "ws"], st[key + "h"] = res["_ws"], res["hidden"]
+
+    pruned_ms = tm.timed(lambda: prefill_stage(r["idx"], r["count"], pipe.k_cap, "p"), reps=reps)
+    nmax = max(w.n_vis)
+    full_idx = torch.full((w.B, nmax), -1, dtype=torch.int32, device=dev)
+    for b, n in enumerate(w.n_vis):
+        full_idx[b, :n] = torch.arange(n, dtype=torch.int32, device=dev)
+    full_cnt = torch.tensor(w.n_vis, dtype=torch.int32, device=dev)
+    full_ms = tm.timed(lambda: prefill_stage(full_idx, full_cnt, nmax, "f"), reps=reps)
+    full_lens = [n + t for n, t in zip(w.n_vis, w.n_txt)]
+    pf = tm.profiled(B, lambda: prefill_stage(full_idx, full_cnt, nmax, "f"))
+    pp = tm.profiled(B, lambda: prefill_stage(r["idx"], r["count"], pipe.k_cap, "p"))
+    pl = tm.profiled(B, lambda: pipe(X, E, bias))
+    qkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
+    p_lin = m.d * qkv + m.n_heads * m.head_dim * m.d + 3 * m.d * m.ffn
+    proj_f = {"mlp2": m.proj_in * m.proj_hidden + m.proj_hidden * m.d, "linear": m.proj_in * m.d}.get(m.proj_kind, 0)
+
+    def rates(prof, T_, K_, lens_):
+        g_fl = 2.0 * (m.n_layers * p_lin * T_ + proj_f * K_)
+        a_fl = m.n_layers * attn_flops(m, lens_)
+        g_ms, a_ms = prof["gemm"]["ms"], prof["attention"]["ms"]
+        return {"gemm_ms": g_ms, "gemm_tflops": g_fl / (g_ms * 1e-3) / 1e12 if g_ms else None,
+                "gemm_frac_of_bf16_burst": g_fl / (g_ms * 1e-3) / 1e12 / pk["bf16"] if g_ms else None,
+                "attention_ms": a_ms, "attention_tflops": a_fl / (a_ms * 1e-3) / 1e12 if a_ms else None,
+                "attention_frac_of_bf16_burst": a_fl / (a_ms * 1e-3) / 1e12 / pk["bf16"] if a_ms else None}
+
+    out = {"workload": w.name, "images": w.B, "visual_tokens": list(w.n_vis), "text_tokens": list(w.n_txt),
+           "group_size": w.group_size, "g": w.g, "k_max": w.k_max, "layers": m.n_layers, "d": m.d,
+           "heads": [m.n_heads, m.n_kv_heads], "kept": counts.tolist(), "mean_kept": float(counts.mean()),
+           "packed_tokens": T, "full_tokens": sum(full_lens),
+           "pipeline_ms": pipe_ms, "select_ms": select_ms, "select_us_per_image": 1e3 * select_ms / w.B,
+           "compaction_ms": compact_ms, "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,
+           "compaction_hbm_frac": comp_bytes / (compact_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
+           "pruned_prefill_ms": pruned_ms, "full_prefix_prefill_ms": full_ms,
+           "speedup_prefill": full_ms / pruned_ms, "speedup_with_selection": full_ms / (pruned_ms + select_ms),
+           "token_ratio": sum(full_lens) / T, "full_prefix": rates(pf, sum(full_lens), sum(w.n_vis), full_lens),
+           "pruned": rates(pp, T, K_sum, lens),
+           "pipeline_stages_ms": {k: v["ms"] for k, v in pl.items() if v["launches"]}}
+    if m.n_layers == 1:
+        wbytes = 2.0 * (p_lin + proj_f)
+        out["weight_bytes"] = wbytes
+        out["pruned_prefill_weight_gbs"] = wbytes / (pruned_ms * 1e-3) / 1e9
+        out["pruned_prefill_hbm_frac"] = wbytes / (pruned_ms * 1e-3) / 1e9 / pk["hbm_gbs"]
+    sel.close()
+    return out
+
+
+def episode_targets(w):
+    """Kept-count targets per selection episode: the workload's statements
+    (mean 64 for one 576-token image; AnyRes: 16..128 per tile group, mean 64,
+    so 80..640 per image; Qwen: 11% of every group; InternVL: the mean kept)."""
+    eps = w.episodes()
+    if w.name.startswith("llavanext"):
+        z = S.normal(w.seed, "group_targets", (len(eps),))
+        t = np.clip(np.round(64 * np.exp(0.6 * z) / np.exp(0.6 * z).mean()), 16, 128).astype(int)
+        return t, 64.0
+    if w.name.startswith("qwen"):
+        return np.array([max(1, int(round(0.11 * n))) for (_, _, n) in eps]), None
+    return np.full(len(eps), int(w.target_mean_k)), float(w.target_mean_k)
+
+
+def measure_workloads(B, torch, dev, gen, pk, c2_model, reps=2):
+    """Every workload other than the headline one, and the InternVL STOP sweep."""
+    tm = Timing(torch, dev)
+    out = {}
+    w1 = S.llava15_1layer()
+    m1 = device_model(B, w1.model, dev, gen, torch, max_pos=1024)
+    t, mt = episode_targets(w1)
+    out["llava15-576-1layer"] = measure_config(B, torch, tm, w1, m1, dev, gen, pk, targets=t, mean_target=mt,
+                                               reps=reps)
+    m1.close()
+    w3 = S.llavanext_anyres_b8()
+    t, mt = episode_targets(w3)
+    out["llavanext-anyres-b8"] = measure_config(B, torch, tm, w3, c2_model, dev, gen, pk, targets=t,
+                                                mean_target=mt, reps=reps)
+    w4 = S.qwen25vl_varres_b8()
+    mq = device_model(B, w4.model, dev, gen, torch, max_pos=4096 + 256)
+    t, mt = episode_targets(w4)
+    out["qwen25vl-varres-b8"] = measure_config(B, torch, tm, w4, mq, dev, gen, pk, targets=t, mean_target=mt,
+                                               reps=reps)
+    sweep = []
+    for k in (32, 64, 128, 256, 512):
+        w5 = S.internvl3_tiles_b4(mean_k=k)
+        t, mt = episode_targets(w5)
+        r = measure_config(B, torch, tm, w5, mq, dev, gen, pk, targets=t, mean_target=mt, reps=reps)
+        if k == 64:
+            out["internvl3-tiles-b4"] = r
+        sweep.append({"target_mean_kept": k, "mean_kept": r["mean_kept"], "select_us_per_image":
+                      r["select_us_per_image"], "compaction_gbs": r["compaction_gbs"],
+                      "pruned_prefill_ms": r["pruned_prefill_ms"], "full_prefix_prefill_ms": r["full_prefix_prefill_ms"],
+                      "speedup_prefill": r["speedup_prefill"], "speedup_with_selection": r["speedup_with_selection"],
+                      "pipeline_ms": r["pipeline_ms"]})
+    out["internvl3_stop_sweep"] = sweep
+    mq.close()
+    return out
 
 
 # Sec. 4 scaling table (LLaVA-1.5-7B rows): input tokens, retained tokens,
@@ -666,57 +992,30 @@ PAPER_SCALING = {
     2240: (224, 236.55, 57.73, 39.14)}
 
 
-def run_sweep(args):
+def scaling_rows(B, torch, dev, gen, selector, model, steps, warmup):
     """Scaling with the visual-prefix length at 10% retention: one image of N
     visual + 48 text tokens on the LLaVA-1.5-7B-shaped model, N = 320..2240.
     Per N: the full-prefix prefill (projector on N rows + 32 layers over N + 48),
     the pruned path (selector incl. its encoder, compaction, projector on the
     kept rows, 32 layers over K + 48) and the selector alone, each the mean of
-    `--steps` calls after `--warmup`."""
-    import torch
-    from paper_2609_13804_gb300 import binding as B
-
-    dev = torch.device("cuda", 0)
-    torch.cuda.set_device(dev)
-    w = S.llava15_7b_b16()
-    s, m = w.selector, w.model
-    selector = B.Selector(s, S.make_selector_weights(w), dev)
-    gen = torch.Generator(device=dev)
-    gen.manual_seed(w.seed)
-    layers = [device_layer_weights(m, l, dev, gen, torch) for l in range(m.n_layers)]
-    head = {"final_norm": torch.ones(m.d, device=dev),
-            "proj_W1": (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16),
-            "proj_W2": (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)}
-    model = B.Model(m, layers, head, dev, max_pos=4096)
+    `steps` calls after `warmup`."""
     L = 48
-
-    def timed(fn):
-        for _ in range(args.warmup):
-            fn()
-        torch.cuda.synchronize()
-        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
-        for _ in range(args.steps):
-            fn()
-        b_.record()
-        torch.cuda.synchronize()
-        return a.elapsed_time(b_) / args.steps
-
+    tm = Timing(torch, dev)
     rows = []
     for N in sorted(PAPER_SCALING):
         K = N // 10
-        X = (torch.randn((N, s.D), device=dev, generator=gen)).to(torch.bfloat16)
-        E = (torch.randn((L, m.d), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+        X = (torch.randn((N, selector.shape.D), device=dev, generator=gen)).to(torch.bfloat16)
+        E = (torch.randn((L, model.shape.d), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
         bias = torch.full((1,), -1e30, dtype=torch.float32, device=dev)  # STOP never wins: exactly K kept
         pipe = B.Pipeline(selector, model, [N], [L], group_size=0, g=1, k_max=K)
-        pruned_ms = timed(lambda: pipe(X, E, bias))
+        pruned_ms = tm.timed(lambda: pipe(X, E, bias), reps=steps, warm=warmup)
         sel_ws = {}
 
         def select():
             r = B.sp_select(selector, [N], [L], X=X, E_text=E, stop_bias=bias, group_size=0, g=1, k_max=K,
                             traces=False, ws=sel_ws.get("ws"))
             sel_ws["ws"] = r["_ws"]
-        selector_ms = timed(select)
+        selector_ms = tm.timed(select, reps=steps, warm=warmup)
         full_idx = torch.arange(N, dtype=torch.int32, device=dev).reshape(1, N)
         full_cnt = torch.full((1,), N, dtype=torch.int32, device=dev)
         st = {}
@@ -730,7 +1029,7 @@ def run_sweep(args):
             r = B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=1, T_cap=o["T_cap"],
                              max_seqlen_cap=N + L, ws=st.get("ws"), hidden=st.get("h"))
             st["ws"], st["h"] = r["_ws"], r["hidden"]
-        full_ms = timed(full_prefill)
+        full_ms = tm.timed(full_prefill, reps=steps, warm=warmup)
         kept = int(pipe.count[0].item())
         pk, pf, pp, ps = PAPER_SCALING[N]
         rows.append({"input_tokens": N, "retained": kept, "full_prefill_ms": full_ms, "stepprune_prefill_ms": pruned_ms,
@@ -739,10 +1038,154 @@ def run_sweep(args):
                      "paper": {"retained": pk, "full_prefill_ms": pf, "stepprune_prefill_ms": pp, "selector_ms": ps,
                                "speedup": pf / pp, "selector_share": ps / pp}})
         del pipe
+    return rows
+
+
+def run_sweep(args):
+    """The scaling table alone (one JSON line, no headline)."""
+    import torch
+    from paper_2609_13804_gb300 import binding as B
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = S.llava15_7b_b16()
+    s, m = w.selector, w.model
+    selector = B.Selector(s, S.make_selector_weights(w), dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(w.seed)
+    model = device_model(B, m, dev, gen, torch, max_pos=4096)
+    rows = scaling_rows(B, torch, dev, gen, selector, model, args.steps, args.warmup)
     line = {"sweep": "visual-prefix length at 10% retention", "config": {"workload": "llava15-7b dims, 1 image",
-            "text_tokens": L, "layers": m.n_layers}, "steps": args.steps, "warmup": args.warmup,
+            "text_tokens": 48, "layers": m.n_layers}, "steps": args.steps, "warmup": args.warmup,
             "paper_gpu": "RTX PRO 6000 Blackwell (the paper's; context only)", "rows": rows}
     print(json.dumps(line), flush=True)
+
+
+def run_profile_case(case: str):
+    """Small, self-contained invocations of one stage of the path, sized for
+    `ncu --set full` captures (a few GB on the device at most, a handful of
+    launches).  Shapes are those of the 16-image LLaVA-1.5-7B-shaped batch
+    unless the case names another workload:
+
+      gemm            1 decoder layer, T = 1791 (4 GEMMs)
+      attention       1 decoder layer, like gemm
+      attention_full  1 layer over the full prefix (16 x 624)
+      attention_gqa   1 Qwen2.5-VL-dims layer (GQA 28/4) over 4 sequences of 3,424
+      select          selection from a given memory H
+      select_deep     2-layer pointer decoder, 4 images, cap 64
+      compact         compaction of the batch
+      compact_full    every visual token kept (50 MB)
+      decode          4 decoder layers, 16 sequences, 3 steps
+
+    Each case runs its stage twice (the second launch set is the one to capture
+    with `-s`)."""
+    import torch
+
+    from paper_2609_13804_gb300 import binding as B
+
+    dev = torch.device("cuda", 0)
+    w = S.internvl3_tiles_b4() if case == "attention_gqa" else S.llava15_7b_b16()
+    counts = S.target_counts(w)
+    if case in ("gemm", "attention", "attention_full", "attention_gqa", "decode"):
+        m = dataclasses.replace(w.model, proj_kind="none", proj_in=w.model.d)
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(1)
+
+        def rnd(shape):
+            return (torch.randn(shape, device=dev, generator=gen) * 0.02).to(torch.bfloat16)
+
+        qkv = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
+        L = {"Wqkv": rnd((qkv, m.d)), "Wo": rnd((m.d, m.n_heads * m.head_dim)), "Wgu": rnd((2 * m.ffn, m.d)),
+             "Wdown": rnd((m.d, m.ffn)), "attn_norm": torch.ones(m.d, device=dev),
+             "mlp_norm": torch.ones(m.d, device=dev)}
+        head = {"final_norm": torch.ones(m.d, device=dev), "proj_W1": None, "proj_W2": None}
+        n_layers = 4 if case == "decode" else 1
+        layers = [L] + [{k: (rnd(v.shape) if v.dtype == torch.bfloat16 else v) for k, v in L.items()}
+                        for _ in range(n_layers - 1)]
+        m = dataclasses.replace(m, n_layers=n_layers)
+        model = B.Model(m, None, None, dev, max_pos=4096, device_weights={"layers": layers, "head": head})
+        lens = [int(k) + 48 for k in counts]
+        if case in ("attention_full", "attention_gqa"):
+            lens = [n + t for n, t in zip(w.n_vis, w.n_txt)]  # every visual token kept: 624 per sequence
+        if case == "decode":
+            # one generation step per sequence over the pruned prefix (a zeroed
+            # cache with the prefix lengths: the contents do not change the work)
+            S_cap = max(lens) + 8
+            kv = B.kv_cache(model, len(lens), S_cap)
+            x_new = (torch.randn((len(lens), m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+            lens_d = torch.tensor(lens, dtype=torch.int32, device=dev)
+            ws = None
+            for _ in range(3):
+                ws = B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws)["_ws"]
+            torch.cuda.synchronize()
+            print("ok", case)
+            return
+        T = sum(lens)
+        cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
+        pos = torch.tensor(np.concatenate([np.arange(n) for n in lens]), dtype=torch.int32, device=dev)
+        x = (torch.randn((T, m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+        # the caps of the pipeline (k_cap 192 per image) so tile widths match the benchmark's launches
+        kc = max(w.n_vis) if case in ("attention_full", "attention_gqa") else w.k_max
+        T_cap = sum(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
+        len_cap = max(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
+        xc = torch.zeros((T_cap, m.d), dtype=torch.bfloat16, device=dev)
+        xc[:T] = x
+        pc = torch.zeros(T_cap, dtype=torch.int32, device=dev)
+        pc[:T] = pos
+        ws = None
+        for _ in range(2):
+            out = B.sp_prefill(model, x=xc, cu_seqlens=cu, pos=pc, B=len(lens), T_cap=T_cap, max_seqlen_cap=len_cap,
+                               ws=ws)
+            ws = out["_ws"]
+        torch.cuda.synchronize()
+    elif case == "select":
+        s = S.SelectorShape(D=w.selector.D, D_text=w.selector.D_text, h=w.selector.h, n_enc_layers=0)
+        sel = S.make_selector_weights(w)
+        H = S.make_memory(w)
+        selector = B.Selector(s, sel, dev)
+        Hd = B.dev_f32(H, dev)
+        bias = B.dev_f32(np.full(w.B, -1e30), dev)   # every episode runs to its cap of 192
+        ws = None
+        for _ in range(2):
+            r = B.sp_select(selector, w.n_vis, w.n_txt, H=Hd, stop_bias=bias, k_max=w.k_max, traces=False, ws=ws)
+            ws = r["_ws"]
+        torch.cuda.synchronize()
+    elif case == "select_deep":
+        w.n_vis, w.n_txt = w.n_vis[:4], w.n_txt[:4]
+        s = S.SelectorShape(D=w.selector.D, D_text=w.selector.D_text, h=w.selector.h, n_enc_layers=0,
+                            n_dec_layers=2)
+        w = dataclasses.replace(w, selector=s)
+        selector = B.Selector(s, S.make_selector_weights(w), dev)
+        Hd = B.dev_f32(S.make_memory(w), dev)
+        bias = B.dev_f32(np.full(4, -1e30), dev)
+        ws = None
+        for _ in range(2):
+            r = B.sp_select(selector, w.n_vis, w.n_txt, H=Hd, stop_bias=bias, k_max=64, traces=False, ws=ws)
+            ws = r["_ws"]
+        torch.cuda.synchronize()
+    elif case == "compact_full":
+        # every visual token kept: the bandwidth-sized compaction (50 MB moved)
+        X = B.dev_bf16(S.bf16_round(S.normal(w.seed, "X", (sum(w.n_vis), 1024))), dev)
+        E = B.dev_bf16(S.bf16_round(S.normal(w.seed, "E", (sum(w.n_txt), 4096), 0.02)), dev)
+        idx = torch.arange(576, dtype=torch.int32, device=dev).repeat(w.B, 1).contiguous()
+        cnt = torch.full((w.B,), 576, dtype=torch.int32, device=dev)
+        for _ in range(2):
+            B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=cnt, k_cap=576, projector_mode=True)
+        torch.cuda.synchronize()
+    elif case == "compact":
+        X = B.dev_bf16(S.bf16_round(S.normal(w.seed, "X", (sum(w.n_vis), 1024))), dev)
+        E = B.dev_bf16(S.bf16_round(S.normal(w.seed, "E", (sum(w.n_txt), 4096), 0.02)), dev)
+        k_cap = 192
+        idx = torch.full((w.B, k_cap), -1, dtype=torch.int32, device=dev)
+        for b, k in enumerate(counts):
+            idx[b, :k] = torch.arange(0, 576, 576 // max(int(k), 1), device=dev)[:k].to(torch.int32)
+        cnt = torch.tensor(counts, dtype=torch.int32, device=dev)
+        for _ in range(2):
+            B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=cnt, k_cap=k_cap, projector_mode=True)
+        torch.cuda.synchronize()
+    else:
+        raise SystemExit(f"unknown case {case}")
+    print("ok", case)
 
 
 def main():
@@ -754,12 +1197,18 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--launch-list", action="store_true",
                     help="set up, warm up and run one more step only (for an ncu launch list)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads, the InternVL STOP sweep and the scaling table")
+    ap.add_argument("--profile-case", default=None,
+                    help="run one small stage invocation for an ncu capture (see run_profile_case)")
     ap.add_argument("--sweep", action="store_true",
                     help="scaling with the visual-prefix length at 10%% retention (one JSON line, no headline)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.sweep:
+    if args.profile_case:
+        run_profile_case(args.profile_case)
+    elif args.sweep:
         run_sweep(args)
     elif args.impl == "reference":
         run_reference(args)

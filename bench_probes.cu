@@ -1,23 +1,46 @@
-// Measurement probes, not on the path: the on-chip peaks the selection
-// kernel's traffic is reported against (aggregate shared-memory and L2 read
-// bandwidth), and the per-round floor of its cluster synchronisation (the
-// round skeleton of select.cu -- two DSMEM push exchanges, two cluster
-// barriers, the block reductions -- with no candidate or history work).
-// Each call allocates what it needs, runs on the current device, synchronises
-// and returns the figure; none is meant for a hot path.
+// Measurement probes of bench.py (not part of libstepprune): the on-chip peaks
+// the selection kernel's traffic is reported against (aggregate shared-memory
+// and L2 read bandwidth), and the per-round floor of its cluster
+// synchronisation (the round skeleton of the selection kernel -- two DSMEM push
+// exchanges, two cluster barriers, the block reductions -- with no candidate or
+// history work).  Each call allocates what it needs, runs on the current
+// device, synchronises and returns the figure; the return value is the CUDA
+// error code (0 = success).
+//
+//   nvcc -gencode arch=compute_103a,code=sm_103a -O3 -shared -Xcompiler -fPIC \
+//        bench_probes.cu -o bench_probes.so       (bench.py's build_probes())
 #include <cooperative_groups.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
 
 #include <algorithm>
 
-#include "common.cuh"
-#include "internal.h"
-#include "stepprune.h"
-
 namespace cg = cooperative_groups;
 
-namespace sp {
-
 namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n;
+}
 
 constexpr int PNT = 512;
 constexpr int SMEM_F4 = 4096;  // 64 KB per CTA
@@ -112,15 +135,11 @@ struct Timer {
 
 }  // namespace
 
-}  // namespace sp
-
-using namespace sp;
-
 extern "C" {
 
-sp_status sp_probe_smem_gbs(double* gbs) {
-  if (!gbs) return report(SP_ERR_INVALID_ARG, "sp_probe_smem_gbs: NULL output");
-  const int grid = device_sm_count() * 2, iters = 4096;
+int bench_probe_smem_gbs(double* gbs) {
+  if (!gbs) return (int)cudaErrorInvalidValue;
+  const int grid = sm_count() * 2, iters = 4096;
   float* sink = nullptr;
   cudaError_t e = cudaMalloc(&sink, (size_t)grid * PNT * sizeof(float));
   Timer t;
@@ -136,16 +155,16 @@ sp_status sp_probe_smem_gbs(double* gbs) {
   float ms = 0.f;
   if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, t.a, t.b);
   if (sink) cudaFree(sink);
-  if (e != cudaSuccess) return report(SP_ERR_CUDA, "sp_probe_smem_gbs: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) return (int)e;
   *gbs = (double)grid * PNT * iters * sizeof(float4) / (ms * 1e-3) / 1e9;
-  return SP_OK;
+  return 0;
 }
 
-sp_status sp_probe_l2_gbs(double* gbs) {
-  if (!gbs) return report(SP_ERR_INVALID_ARG, "sp_probe_l2_gbs: NULL output");
+int bench_probe_l2_gbs(double* gbs) {
+  if (!gbs) return (int)cudaErrorInvalidValue;
   const size_t bytes = (size_t)48 << 20;  // well inside the L2
   const size_t n4 = bytes / sizeof(float4);
-  const int grid = device_sm_count() * 4, passes = 20;
+  const int grid = sm_count() * 4, passes = 20;
   float4* src = nullptr;
   float* sink = nullptr;
   cudaError_t e = cudaMalloc(&src, bytes);
@@ -163,16 +182,16 @@ sp_status sp_probe_l2_gbs(double* gbs) {
   if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, t.a, t.b);
   if (src) cudaFree(src);
   if (sink) cudaFree(sink);
-  if (e != cudaSuccess) return report(SP_ERR_CUDA, "sp_probe_l2_gbs: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) return (int)e;
   *gbs = (double)bytes * passes / (ms * 1e-3) / 1e9;
-  return SP_OK;
+  return 0;
 }
 
-sp_status sp_probe_select_floor(int cluster_size, int h, int rounds, int episodes, double* us_per_round) {
-  if (!us_per_round) return report(SP_ERR_INVALID_ARG, "sp_probe_select_floor: NULL output");
+int bench_probe_select_floor(int cluster_size, int h, int rounds, int episodes, double* us_per_round) {
+  if (!us_per_round) return (int)cudaErrorInvalidValue;
   if ((cluster_size != 8 && cluster_size != 16) || h < 128 || h > 1024 || rounds < 1 || episodes < 1 ||
       episodes * cluster_size > 4096)
-    return report(SP_ERR_SHAPE, "sp_probe_select_floor: bad cluster size / h / rounds / episodes");
+    return (int)cudaErrorInvalidValue;
   const int C = cluster_size;
   const size_t smem = (size_t)(2 * C * h + 2 * C * 4 + FNT / 32) * sizeof(float);
   float* sink = nullptr;
@@ -201,9 +220,9 @@ sp_status sp_probe_select_floor(int cluster_size, int h, int rounds, int episode
   float ms = 0.f;
   if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, t.a, t.b);
   if (sink) cudaFree(sink);
-  if (e != cudaSuccess) return report(SP_ERR_CUDA, "sp_probe_select_floor: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) return (int)e;
   *us_per_round = (double)ms * 1e3 / rounds;
-  return SP_OK;
+  return 0;
 }
 
 }  // extern "C"

@@ -429,10 +429,14 @@ SP_API sp_status sp_project(const sp_model* m, const sp_project_io* io, void* wo
                      size_t workspace_bytes, sp_stream stream);
 
 /*
- * Prefill of the packed sequences: causal attention within each sequence
- * (cu_seqlens), rotary positions pos, pre-RMSNorm Llama-style layers, and the
- * final RMSNorm.  hidden rows t < T = cu_seqlens[B] are written; rows >= T are
- * untouched.  residual (optional) receives the last residual stream (fp32,
+ * Prefill of the packed sequences: the frozen LM run over the pruned prefix
+ * that Algorithm 1 hands it (Sec. 3.3, last paragraph: the kept tokens,
+ * restored to native order and projected, precede the text; Sec. 1: the
+ * prefill cost the selection removes is that of the dropped visual tokens).
+ * The layers are those of the evaluated backbones (Sec. 4.1): causal attention
+ * within each sequence (cu_seqlens), grouped-query heads, rotary positions
+ * pos, pre-RMSNorm Llama-style layers with SwiGLU, and the final RMSNorm.
+ * hidden rows t < T = cu_seqlens[B] are written; rows >= T are untouched.  residual (optional) receives the last residual stream (fp32,
  * before the final norm).  kv (optional) receives the key / value cache the
  * generation that follows reads (sp_decode): per layer l, sequence b and
  * position p = pos[row] the rotated key at
@@ -517,6 +521,18 @@ SP_API sp_status sp_decode(const sp_model* m, const sp_decode_io* io, void* work
 /* The whole path: select -> compact -> project -> prefill.                  */
 /* ------------------------------------------------------------------------ */
 
+/*
+ * Algorithm 1 (Sec. 3.5) end to end on the device, followed by the prefill
+ * over its result: the text projection and the encoder (Eq. 3), the pointer
+ * rounds of Eq. 4 / Eq. 11 with the STOP action per episode, the restore to
+ * native order, the gather into packed sequences [kept visual rows; text
+ * rows] (Sec. 3.3, last paragraph), the projector on the kept rows, and the
+ * LM prefill of sp_prefill.  One stream, no host synchronisation: sizes that
+ * depend on the selection stay on the device (grids are sized from caps).
+ * Outputs: idx / count as sp_select's, cu_seqlens as sp_compact's, hidden as
+ * sp_prefill's.  Errors: the union of those of the four calls; the
+ * workspace must hold sp_pipeline_workspace() bytes (SP_ERR_WORKSPACE).
+ */
 typedef struct {
   sp_select_in sel;          /* X and E_text required (H ignored); E_text is also the
                                 text rows of the LM input, so D_text must equal d */
@@ -567,29 +583,6 @@ SP_API sp_status sp_profile_begin(int capacity);
 /* Synchronises on the recorded events and returns, per sp_kernel_kind, the
  * summed milliseconds, launch counts and algorithmic flops / bytes. */
 SP_API sp_status sp_profile_end(double* ms, long long* launches, double* flops, double* bytes);
-
-/* ------------------------------------------------------------------ measurement probes
- * Not part of the method (the paper has no counterpart): the on-chip peaks the
- * selection kernel's traffic is measured against, and the per-round floor of
- * its cluster synchronisation.  Each call allocates its own buffers on the
- * current device, runs, synchronises the device and returns the figure; use
- * them outside timed regions.  Errors: SP_ERR_INVALID_ARG (NULL output),
- * SP_ERR_SHAPE (sizes out of range), SP_ERR_CUDA. */
-
-/* Aggregate shared-memory read bandwidth of the device (GB/s): two CTAs per
- * SM stream 16-byte reads over a 64 KB buffer each. */
-SP_API sp_status sp_probe_smem_gbs(double* gbs);
-
-/* Read bandwidth from an L2-resident 48 MB buffer (GB/s, all SMs, 16-byte
- * cache-global loads). */
-SP_API sp_status sp_probe_l2_gbs(double* gbs);
-
-/* Microseconds per round of the selection loop's synchronisation alone:
- * `episodes` clusters of `cluster_size` (8 or 16) CTAs of 256 threads, each
- * round two DSMEM push exchanges (h floats, then a short list, into every CTA
- * of the cluster), two cluster barriers and the block reductions, no
- * candidate or history work.  h in 128..1024, rounds >= 1. */
-SP_API sp_status sp_probe_select_floor(int cluster_size, int h, int rounds, int episodes, double* us_per_round);
 
 #ifdef __cplusplus
 }

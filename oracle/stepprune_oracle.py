@@ -144,14 +144,17 @@ def softmax(x, axis: int = -1) -> np.ndarray:
     return e / e.sum(axis=axis, keepdims=True)
 
 
-def attention(q, k, v, n_heads: int, n_kv_heads: int, causal: bool, q_pos=None) -> np.ndarray:
+def attention(q, k, v, n_heads: int, n_kv_heads: int, causal: bool, q_pos=None,
+              p_store: Optional[str] = None) -> np.ndarray:
     """Scaled dot-product attention of one sequence.
 
     q [Lq, Hq*dh], k/v [L, Hkv*dh].  Query head i reads key/value head
     floor(i * Hkv / Hq) (grouped-query attention; Hkv == Hq is plain MHA).
     Causal: the query at position p attends to key positions 0..p.  The query
     rows are the positions 0..L-1 of the sequence unless q_pos gives their
-    positions (a subset of the sequence's rows).
+    positions (a subset of the sequence's rows).  p_store='bf16' rounds the
+    attention probabilities to bf16 before they weight the values (the operand
+    precision of a bf16 tensor-core P V product).
     """
     q, k, v = _f(q), _f(k), _f(v)
     Lq, L = q.shape[0], k.shape[0]
@@ -167,7 +170,7 @@ def attention(q, k, v, n_heads: int, n_kv_heads: int, causal: bool, q_pos=None) 
         kj = k[:, j * dh:(j + 1) * dh]
         vj = v[:, j * dh:(j + 1) * dh]
         s = qi @ kj.T / math.sqrt(dh) + mask
-        out[:, i * dh:(i + 1) * dh] = softmax(s, axis=-1) @ vj
+        out[:, i * dh:(i + 1) * dh] = _store(softmax(s, axis=-1), p_store) @ vj
     return out
 
 
@@ -793,7 +796,7 @@ def _mm(a, b, acc: str) -> np.ndarray:
 
 
 def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = None,
-                  acc: str = "fp64", kv_out: Optional[list] = None) -> np.ndarray:
+                  acc: str = "fp64", kv_out: Optional[list] = None, p_store: Optional[str] = None) -> np.ndarray:
     """One pre-norm decoder layer of the frozen LM over the packed sequences:
     h += Wo Attn(RoPE(Wq x), RoPE(Wk x), Wv x), x = RMSNorm(h);
     h += Wdown (SiLU(Wg x') * Wu x'), x' = RMSNorm(h).  Attention is causal and
@@ -802,7 +805,8 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
     inputs, rotated q / k, v, attention output, SwiGLU output) are rounded to
     bf16 where they are stored.  acc='fp32' computes the four projections in
     fp32 instead of fp64 (used only to size how far two exact bf16 prefills
-    drift apart through rounding decisions alone).  kv_out, if given, receives
+    drift apart through rounding decisions alone; p_store='bf16' likewise
+    rounds the attention probabilities).  kv_out, if given, receives
     this layer's (rotated keys, values) of every packed row: the cache a
     generation step reads."""
     h = _f(h).copy()
@@ -818,7 +822,7 @@ def prefill_layer(h, L: Dict, m, cu: Sequence[int], pos, store: Optional[str] = 
     for b in range(len(cu) - 1):
         s, e = int(cu[b]), int(cu[b + 1])
         if e > s:
-            o[s:e] = attention(q[s:e], k[s:e], v[s:e], Hq, Hkv, causal=True)
+            o[s:e] = attention(q[s:e], k[s:e], v[s:e], Hq, Hkv, causal=True, p_store=p_store)
     h = h + _mm(_store(o, store), _f(L["Wo"]).T, acc)
     x2 = _store(rms_norm(h, m.rms_eps, L.get("mlp_norm")), store)
     gu = _mm(x2, _f(L["Wgu"]).T, acc)
@@ -868,10 +872,10 @@ def final_norm(h, m, gain=None) -> np.ndarray:
 
 
 def prefill(x, layers: Sequence[Dict], m, cu, pos, final_gain=None, store: Optional[str] = None,
-            acc: str = "fp64", kv_out: Optional[list] = None) -> np.ndarray:
+            acc: str = "fp64", kv_out: Optional[list] = None, p_store: Optional[str] = None) -> np.ndarray:
     h = _f(x)
     for L in layers:
-        h = prefill_layer(h, L, m, cu, pos, store, acc, kv_out)
+        h = prefill_layer(h, L, m, cu, pos, store, acc, kv_out, p_store)
     return final_norm(h, m, final_gain)
 
 

@@ -32,8 +32,8 @@ EXPORTS = [
     "sp_num_episodes", "sp_select_workspace", "sp_select", "sp_packed_cap", "sp_compact", "sp_model_create",
     "sp_model_destroy", "sp_project_workspace", "sp_project", "sp_prefill_workspace", "sp_prefill",
     "sp_pipeline_workspace", "sp_pipeline", "sp_pipeline_host_workspace", "sp_pipeline_host",
-    "sp_profile_begin", "sp_profile_end", "sp_select_noalloc", "sp_probe_smem_gbs", "sp_probe_l2_gbs",
-    "sp_probe_select_floor", "sp_decode_workspace", "sp_decode", "sp_select_train", "sp_soft_topk", "sp_vp_gate",
+    "sp_profile_begin", "sp_profile_end", "sp_select_noalloc",
+    "sp_decode_workspace", "sp_decode", "sp_select_train", "sp_soft_topk", "sp_vp_gate",
     "sp_mrope_positions",
 ]
 SP_SELECT_NOALLOC_SCRATCH_BYTES = 64 << 20
@@ -172,9 +172,6 @@ def lib():
         "sp_profile_begin": (C.c_int, [C.c_int]),
         "sp_profile_end": (C.c_int, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]),
-        "sp_probe_smem_gbs": (C.c_int, [C.POINTER(C.c_double)]),
-        "sp_probe_l2_gbs": (C.c_int, [C.POINTER(C.c_double)]),
-        "sp_probe_select_floor": (C.c_int, [C.c_int, C.c_int, C.c_int, C.c_int, C.POINTER(C.c_double)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -628,24 +625,3 @@ def sp_profile_end() -> Dict[str, Dict[str, float]]:
     _check(lib().sp_profile_end(ms, la, fl, by), "sp_profile_end")
     return {k: {"ms": ms[i], "launches": int(la[i]), "flops": fl[i], "bytes": by[i]}
             for i, k in enumerate(KERNEL_KINDS)}
-
-
-def probe_smem_gbs() -> float:
-    """Aggregate shared-memory read bandwidth of the current device (GB/s)."""
-    v = C.c_double()
-    _check(lib().sp_probe_smem_gbs(C.byref(v)), "sp_probe_smem_gbs")
-    return v.value
-
-
-def probe_l2_gbs() -> float:
-    """Read bandwidth from an L2-resident buffer (GB/s)."""
-    v = C.c_double()
-    _check(lib().sp_probe_l2_gbs(C.byref(v)), "sp_probe_l2_gbs")
-    return v.value
-
-
-def probe_select_floor(cluster_size: int, h: int, rounds: int, episodes: int) -> float:
-    """Microseconds per round of the selection loop's synchronisation alone."""
-    v = C.c_double()
-    _check(lib().sp_probe_select_floor(cluster_size, h, rounds, episodes, C.byref(v)), "sp_probe_select_floor")
-    return v.value

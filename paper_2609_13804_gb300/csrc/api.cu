@@ -1015,9 +1015,9 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
   gs.splitk_floats = p.splitk_floats;
   SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   SP_CUDA(bf16_to_f32(io->x, h32, T_cap, T_dev, c.d, st), "embed");
-  // the attention's last key tile reads up to 63 rows past the packed length
+  // the attention's last key block reads up to 127 rows past the packed length
   // (weighted by zero); keep them finite: the QKV GEMMs leave them untouched
-  SP_CUDA(zero_rows_after(p.qkv, (size_t)qkvw * 2, T_dev, T_cap, 64, st), "qkv tail");
+  SP_CUDA(zero_rows_after(p.qkv, (size_t)qkvw * 2, T_dev, T_cap, 128, st), "qkv tail");
   if (mrope)
     SP_CUDA(mrope_rows_launch(m->rope, c.max_pos, c.head_dim / 2, io->pos3, c.mrope_section[0],
                               c.mrope_section[0] + c.mrope_section[1], T_dev, T_cap, p.mrows, p.mident, io->err, st),

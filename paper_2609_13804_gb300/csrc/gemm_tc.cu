@@ -1285,40 +1285,14 @@ static int swap_split(int tiles, int KB, int sms, size_t cap_floats, int N_acc) 
   return best;
 }
 
-static bool gemm_swap_enabled() {
-  static int mode = -1;
-  if (mode < 0) {
-    const char* s = getenv("SP_GEMM_SWAP");
-    mode = s ? atoi(s) : 1;
-  }
-  return mode != 0;
-}
-
 // Tile width of the CTA-pair variant for a GEMM, or 0 for the single-CTA one.
 // Pairs with 256-wide tiles wherever M reaches a pair tile: measured on the
 // 7B-dims prefill they beat the single-CTA kernel on every GEMM, while 128-wide
 // pair tiles lose (the MMA issue per stage no longer hides behind the MMA).
-// SP_GEMM_PAIRS=0 in the environment selects the single-CTA kernel (A/B runs);
-// SP_GEMM_PAIRS=1 allows 128-wide pair tiles where the column-tile count is small.
-// SP_GEMM_STREAMK=0 in the environment turns the stream-K tail off (A/B runs).
-static bool gemm_stream_k_enabled() {
-  static int mode = -1;
-  if (mode < 0) {
-    const char* s = getenv("SP_GEMM_STREAMK");
-    mode = s ? atoi(s) : 1;
-  }
-  return mode != 0;
-}
-
 int gemm_pair_policy(int M_cap, int N_acc, int kind) {
-  static int mode = -1;
-  if (mode < 0) {
-    const char* s = getenv("SP_GEMM_PAIRS");
-    mode = s ? atoi(s) : 2;
-  }
-  if (mode == 0 || M_cap < 2 * BM) return 0;
-  if (N_acc % 256 == 0 && (mode == 2 || N_acc / 256 >= 20 || kind == EPI_SWIGLU_BF16)) return 256;
-  return (N_acc % 128 == 0 && mode == 1) ? 128 : 0;
+  (void)kind;
+  if (M_cap < 2 * BM) return 0;
+  return N_acc % 256 == 0 ? 256 : 0;
 }
 
 size_t gemm_scratch_bytes() {
@@ -1357,7 +1331,7 @@ bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {
 cudaError_t gemm_swap_partials(const CUtensorMap& A16, int M_cap, const GemmB& B, int N_acc, int* err,
                                cudaStream_t st, const GemmScratch& sk, int* ks_out) {
   const int sms = device_sm_count();
-  if (!sk.splitk || M_cap < 1 || M_cap > 32 || N_acc % BM != 0 || B.K % BK != 0 || !gemm_swap_enabled())
+  if (!sk.splitk || M_cap < 1 || M_cap > 32 || N_acc % BM != 0 || B.K % BK != 0)
     return cudaErrorNotSupported;
   const int tiles = N_acc / BM, KB = B.K / BK;
   const int ks = swap_split(tiles, KB, sms, sk.splitk_floats, N_acc);
@@ -1457,7 +1431,7 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
     const int mp = (M_cap + 2 * BM - 1) / (2 * BM);
     const int tiles = mp * (N_acc / pair_bn);
     int slots = 0;
-    if (sk && sk->part && sk->flags && gemm_stream_k_enabled()) {
+    if (sk && sk->part && sk->flags) {
       a.sk_part = sk->part;
       a.sk_flags = sk->flags;
       slots = sk->slots;

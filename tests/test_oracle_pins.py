@@ -56,6 +56,26 @@ def test_attention_matches_torch_sdpa(hq, hkv, causal):
     np.testing.assert_allclose(out, ref.transpose(0, 1).reshape(L, hq * dh).numpy(), atol=1e-12)
 
 
+def test_attention_probability_rounding_matches_torch():
+    """p_store='bf16': the softmax probabilities rounded to bf16 before they
+    weight the values, as torch computes it; the rounding moves each output by
+    at most 2^-8 of the largest |value| (probabilities sum to 1)."""
+    L, dh, hq, hkv = 11, 8, 4, 2
+    q = S.normal(6, "q", (L, hq * dh)).astype(np.float64)
+    k = S.normal(6, "k", (L, hkv * dh)).astype(np.float64)
+    v = S.normal(6, "v", (L, hkv * dh)).astype(np.float64)
+    got = O.attention(q, k, v, hq, hkv, True, p_store="bf16")
+    Q = t64(q).view(L, hq, dh).transpose(0, 1)
+    K = t64(k).view(L, hkv, dh).transpose(0, 1).repeat_interleave(hq // hkv, dim=0)
+    V = t64(v).view(L, hkv, dh).transpose(0, 1).repeat_interleave(hq // hkv, dim=0)
+    mask = torch.triu(torch.full((L, L), float("-inf")), 1)
+    P = torch.softmax(Q @ K.transpose(1, 2) / math.sqrt(dh) + mask, dim=-1)
+    ref = (P.float().to(torch.bfloat16).double() @ V).transpose(0, 1).reshape(L, hq * dh).numpy()
+    np.testing.assert_allclose(got, ref, atol=1e-12)
+    exact = O.attention(q, k, v, hq, hkv, True)
+    assert 0 < np.abs(got - exact).max() <= 2.0 ** -8 * np.abs(v).max()
+
+
 def test_attention_single_token_returns_value_and_is_causal():
     dh = 4
     q = S.normal(3, "q", (5, 2 * dh)).astype(np.float64)
