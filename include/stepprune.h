@@ -570,6 +570,28 @@ SP_API sp_status sp_pipeline_host(const sp_selector* s, const sp_model* m, const
                            void* workspace, size_t workspace_bytes, sp_stream stream);
 
 /* ------------------------------------------------------------------------ */
+/* Failure-detection self-test (the paper has no counterpart).               */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Every wait in this library's kernels is bounded (2 s): one that runs out
+ * sets SP_DEVERR_TIMEOUT in the call's error word and the kernel returns, so a
+ * lost arrival never hangs the GPU.  This call runs the two wait helpers the
+ * kernels use, with limit_us microseconds (1 .. 2,000,000) in place of 2 s:
+ *   out[0] = 1 if a wait on an mbarrier completed, 0 if it timed out,
+ *   out[1] = 1 if a wait for *flag == 1 completed, 0 if it timed out.
+ * The mbarrier gets no arrival (so the wait runs out) unless `complete` is
+ * non-zero; the flag wait completes iff the caller's DEVICE int *flag is 1.
+ * A timeout ORs SP_DEVERR_TIMEOUT into *err (DEVICE, may be NULL);
+ * sp_device_error_status() maps it to SP_ERR_TIMEOUT.  The stream and the
+ * context stay usable.  flag, out: DEVICE.  Asynchronous on `stream`.
+ * Errors: SP_ERR_INVALID_ARG (NULL flag / out), SP_ERR_SHAPE (limit out of
+ * range), SP_ERR_CUDA.
+ */
+SP_API sp_status sp_wait_probe(const int* flag, unsigned int limit_us, int complete, int* out, int* err,
+                               sp_stream stream);
+
+/* ------------------------------------------------------------------------ */
 /* Per-kernel timing (CUDA events recorded around every launch).             */
 /* ------------------------------------------------------------------------ */
 

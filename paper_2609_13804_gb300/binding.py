@@ -34,7 +34,7 @@ EXPORTS = [
     "sp_pipeline_workspace", "sp_pipeline", "sp_pipeline_host_workspace", "sp_pipeline_host",
     "sp_profile_begin", "sp_profile_end", "sp_select_noalloc",
     "sp_decode_workspace", "sp_decode", "sp_select_train", "sp_soft_topk", "sp_vp_gate",
-    "sp_mrope_positions",
+    "sp_mrope_positions", "sp_wait_probe",
 ]
 SP_SELECT_NOALLOC_SCRATCH_BYTES = 64 << 20
 
@@ -169,6 +169,7 @@ def lib():
         "sp_soft_topk": (C.c_int, [C.c_int, IP, C.c_int, P, P, C.c_float, P, P, P]),
         "sp_vp_gate": (C.c_int, [C.c_int, C.c_int, P, P, P, P, P]),
         "sp_mrope_positions": (C.c_int, [C.c_int, IP, IP, IP, P, C.c_int, P, P, C.c_int, P, P]),
+        "sp_wait_probe": (C.c_int, [P, C.c_uint, C.c_int, P, P, P]),
         "sp_profile_begin": (C.c_int, [C.c_int]),
         "sp_profile_end": (C.c_int, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), C.POINTER(C.c_double),
                                      C.POINTER(C.c_double)]),
@@ -625,3 +626,14 @@ def sp_profile_end() -> Dict[str, Dict[str, float]]:
     _check(lib().sp_profile_end(ms, la, fl, by), "sp_profile_end")
     return {k: {"ms": ms[i], "launches": int(la[i]), "flops": fl[i], "bytes": by[i]}
             for i, k in enumerate(KERNEL_KINDS)}
+
+
+def sp_wait_probe(*, flag, limit_us: int, complete: bool, out, err=None, stream=None):
+    """The bounded-wait self-test: out[0] / out[1] = 1 if the mbarrier / flag
+    wait completed, 0 if it ran out after limit_us (SP_DEVERR_TIMEOUT in err)."""
+    _check(lib().sp_wait_probe(ptr(flag), int(limit_us), 1 if complete else 0, ptr(out), ptr(err), _stream(stream)),
+           "sp_wait_probe")
+
+
+def sp_device_error_status(word: int) -> int:
+    return lib().sp_device_error_status(int(word))

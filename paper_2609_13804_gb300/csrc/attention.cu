@@ -12,56 +12,64 @@ namespace {
 // ===========================================================================
 // Persistent tcgen05 flash attention.  One CTA per SM walks a static list of
 // work items; an item is 128 query rows (one tile) of one sequence for a PAIR
-// of query heads (2p, 2p + 1).  The two heads see the same keys positions and
-// the same mask, so their pipelines advance in lockstep and the tensor pipe
-// alternates between them: while one head's softmax runs, the other head's
-// S = Q K^T or O += P V keeps the tensor cores busy.
+// of query heads (2p, 2p + 1).  Each head of the pair has its own pipeline in
+// the CTA (its TMA thread, its MMA-issuing thread, its softmax warpgroup, its
+// TMEM columns); the two share the SM's tensor pipe, which interleaves them,
+// and the issue work of two threads.
 //
-//   warp 0      TMA: per head its Q tile once per item, then per 128-key block
-//               its K and V blocks (one buffer each per head; the next block's
-//               load starts as soon as the MMA that read the buffer is done)
-//   warp 1      TMEM allocation (all 512 columns); one thread issues, per key
-//               block: S_0 = Q_0 K_0^T, S_1 = Q_1 K_1^T (M 128, N 128, both
-//               K-major from shared memory), then O_0 += P_0 V_0 and
-//               O_1 += P_1 V_1 with P read from Tensor Memory (where the
-//               softmax wrote it over its S) and V an MN-major operand straight
-//               from its TMA block.  Before S_t overwrites P_t, the previous
-//               O_t += P_t V_t must have completed (its commit is waited on).
-//   warps 2-3   idle
+//   warps 0 / 3  TMA of head 0 / 1: the Q tile once per item, then per 64-key
+//                block the K and V blocks into two-stage rings
+//   warps 1 / 2  MMA issue of head 0 / 1 (warp 1 also allocates the 512 TMEM
+//                columns), software-pipelined by one key block: the scores of
+//                block j + 1 (S = Q K^T, M 128, N 64, both K-major from shared
+//                memory) go to the tensor pipe before O += P V of block j (P
+//                read from Tensor Memory where the softmax wrote it over its S,
+//                V an MN-major operand straight from its TMA block).  Two S / P
+//                buffers per head let the softmax of block j overlap the scores
+//                of block j + 1; S of block j + 2 reuses block j's buffer only
+//                once O += P V of block j has completed (its commit).
 //   warps 4-7   softmax of head 0, warps 8-11 of head 1: one thread per query
 //               row (= TMEM lane): S row from TMEM, mask (causal diagonal
-//               block, sequence tail), running max / sum in the exp2 domain, P
+//               blocks, sequence tail), running max / sum in the exp2 domain, P
 //               as bf16 back over S, O rescaled in TMEM only when the running
 //               max grows by more than 2^8 (lazy rescale: O and the sum l share
 //               the stale max, so the result is exact), final O / l to global.
-// TMEM columns: S / P of head t at [128 t, 128 t + 128) (P: 64 columns of
-// bf16 pairs over the first half of S), O of head t at [256 + DH t, + DH).
+// TMEM columns: S / P buffer b of head t at [128 t + 64 b, + 64) (P: 32
+// columns of bf16 pairs over the first half of S), O of head t at
+// [256 + DH t, + DH).
 // Keys past the sequence get P = 0; their V rows must be finite (the caller
 // keeps the rows past the packed length zero, or the tensor map ends there).
 namespace fa {
 
-constexpr int BQ = 128, BKV = 128, NTHR = 384;
+constexpr int BQ = 128, BKV = 64, NTHR = 384;
 constexpr float kRescaleLog2 = 8.f;  // rescale O once the max moved by more than this (log2 units)
 
 template <int DH>
 struct Cfg {
-  static constexpr uint32_t BOX_BYTES = 128 * 128;      // 128 rows x 64 bf16 (one 128-byte swizzle box)
-  static constexpr uint32_t TILE_BYTES = DH / 64 * BOX_BYTES;  // a Q tile or a K / V block of one head
-  static constexpr uint32_t OFF_Q = 0;                   // [2 heads]
-  static constexpr uint32_t OFF_K = 2 * TILE_BYTES;      // [2 heads]
-  static constexpr uint32_t OFF_V = 4 * TILE_BYTES;      // [2 heads]
-  static constexpr uint32_t OFF_BAR = 6 * TILE_BYTES;
-  static constexpr size_t SMEM_USED = 1024 + OFF_BAR + 256;
+  static constexpr uint32_t BOX_Q = BQ * 128;              // 128 rows x 64 bf16 (one 128-byte swizzle box)
+  static constexpr uint32_t BOX_KV = BKV * 128;            // 64 rows x 64 bf16
+  static constexpr uint32_t Q_BYTES = DH / 64 * BOX_Q;     // a Q tile of one head
+  static constexpr uint32_t KV_BYTES = DH / 64 * BOX_KV;   // a K or V block of one head
+  static constexpr uint32_t OFF_Q = 0;                     // [2 heads]
+  static constexpr uint32_t OFF_K = 2 * Q_BYTES;           // [2 heads][2 stages]
+  static constexpr uint32_t OFF_V = OFF_K + 4 * KV_BYTES;  // [2 heads][2 stages]
+  static constexpr uint32_t OFF_BAR = OFF_V + 4 * KV_BYTES;
+  static constexpr size_t SMEM_USED = 1024 + OFF_BAR + 512;
   // a CTA holds all 512 TMEM columns: ask for more than half of the shared
   // memory so that a second CTA is never co-resident (it would only wait)
   static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
   static constexpr uint32_t T_O = 256;
 };
 
-// Barriers, per head t: index base + t.
+// Barriers.  Per head t: Q_FULL + t, Q_EMPTY + t, O_FULL + t, O_EMPTY + t,
+// MMA_DONE + t; per head t and stage / buffer b (= block index & 1): X + 2 t + b.
+// A slot's K is free once the scores that read it are complete (S_FULL), its
+// V once O += P V is (PV_DONE): no "empty" barriers.  The V block's bytes
+// complete on the P-ready barrier of its block (four softmax warps plus the
+// TMA thread's expect-tx arrive), so O += P V waits once for both.
 enum Bar {
-  Q_FULL = 0, Q_EMPTY = 2, K_FULL = 4, K_EMPTY = 6, V_FULL = 8, V_EMPTY = 10,
-  S_FULL = 12, P_FULL = 14, PV_DONE = 16, O_FULL = 18, O_EMPTY = 20, MMA_DONE = 22, N_BARS = 23
+  Q_FULL = 0, Q_EMPTY = 2, K_FULL = 4, S_FULL = 8, P_FULL = 12, PV_DONE = 16, O_FULL = 20, O_EMPTY = 22,
+  MMA_DONE = 24, N_BARS = 26
 };
 
 SP_DEVINL float ex2(float x) {
@@ -99,8 +107,9 @@ SP_DEVINL bool item_at(int it, const int* __restrict__ cu, int B, int HP, int n_
 
 template <int DH>
 __global__ void __launch_bounds__(NTHR, 1)
-attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict__ out, const int* __restrict__ cu,
-               int B, int Hq, int Hkv, int n_tiles, int ld_out, int causal_i, float scale_log2, int* err) {
+attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
+               __nv_bfloat16* __restrict__ out, const int* __restrict__ cu, int B, int Hq, int Hkv, int n_tiles,
+               int ld_out, int causal_i, float scale_log2, int* err) {
   using C = Cfg<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -112,7 +121,8 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < N_BARS; ++i) mbar_init(&bar[i], (i == P_FULL || i == P_FULL + 1 || i == O_EMPTY || i == O_EMPTY + 1) ? 4 : 1);
+    for (int i = 0; i < N_BARS; ++i)
+      mbar_init(&bar[i], (i >= P_FULL && i < P_FULL + 4) ? 5 : (i == O_EMPTY || i == O_EMPTY + 1) ? 4 : 1);
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -126,112 +136,115 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict
   pdl_wait();  // programmatic launch: the previous kernel's outputs are visible from here
   pdl_trigger();
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA
+  if (warp == 0 || warp == 3) {
+    // ------------------------------------------------------------ TMA of head t
     if (lane == 0) {
-      tma_prefetch_desc(&tm);
+      const int t = warp == 3;
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmKV);
       uint32_t g = 0, nitem = 0;
       bool ok = true;
+      uint8_t* sQ = sm + C::OFF_Q + t * C::Q_BYTES;
       for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
         Item I;
         if (!item_at(it, cu, B, HP, n_tiles, Hq, Hkv, causal, I)) continue;
+        if (!mbar_wait(&bar[Q_EMPTY + t], (nitem & 1) ^ 1u, err)) break;
+        mbar_arrive_expect_tx(&bar[Q_FULL + t], C::Q_BYTES);
+        const int qcol = (t ? I.h1 : I.h0) * DH;
+        const int kvh = t ? I.kvh1 : I.kvh0;
+        const int kcol = (Hq + kvh) * DH, vcol = (Hq + Hkv + kvh) * DH;
 #pragma unroll
-        for (int t = 0; t < 2; ++t) {
-          if (!mbar_wait(&bar[Q_EMPTY + t], (nitem & 1) ^ 1u, err)) { ok = false; break; }
-          mbar_arrive_expect_tx(&bar[Q_FULL + t], C::TILE_BYTES);
-          uint8_t* dst = sm + C::OFF_Q + t * C::TILE_BYTES;
-          const int col = (t ? I.h1 : I.h0) * DH;
+        for (int bx = 0; bx < DH / 64; ++bx)
+          tma_load_2d(sQ + bx * C::BOX_Q, &tmQ, &bar[Q_FULL + t], qcol + bx * 64, I.s0 + I.q0);
+        for (int j = 0; j < I.nkv; ++j, ++g) {
+          // slot st last held block g - 2: its K is free once that block's
+          // scores are complete, its V once its O += P V is
+          const uint32_t st = g & 1, pe = ((g >> 1) & 1) ^ 1u;
+          uint8_t* sK = sm + C::OFF_K + (2 * t + st) * C::KV_BYTES;
+          uint8_t* sV = sm + C::OFF_V + (2 * t + st) * C::KV_BYTES;
+          uint64_t* kfull = &bar[K_FULL + 2 * t + st];
+          uint64_t* vfull = &bar[P_FULL + 2 * t + st];
+          if (g >= 2 && !mbar_wait(&bar[S_FULL + 2 * t + st], pe, err)) { ok = false; break; }
+          mbar_arrive_expect_tx(kfull, C::KV_BYTES);
 #pragma unroll
           for (int bx = 0; bx < DH / 64; ++bx)
-            tma_load_2d(dst + bx * C::BOX_BYTES, &tm, &bar[Q_FULL + t], col + bx * 64, I.s0 + I.q0);
-        }
-        for (int j = 0; ok && j < I.nkv; ++j, ++g) {
-          const uint32_t pe = (g & 1) ^ 1u;
+            tma_load_2d(sK + bx * C::BOX_KV, &tmKV, kfull, kcol + bx * 64, I.s0 + j * BKV);
+          if (g >= 2 && !mbar_wait(&bar[PV_DONE + 2 * t + st], pe, err)) { ok = false; ++g; break; }
+          mbar_arrive_expect_tx(vfull, C::KV_BYTES);
 #pragma unroll
-          for (int kv = 0; kv < 2; ++kv) {  // K of both heads, then V of both heads
-#pragma unroll
-            for (int t = 0; t < 2; ++t) {
-              const int e_bar = (kv ? V_EMPTY : K_EMPTY) + t, f_bar = (kv ? V_FULL : K_FULL) + t;
-              if (!mbar_wait(&bar[e_bar], pe, err)) { ok = false; break; }
-              mbar_arrive_expect_tx(&bar[f_bar], C::TILE_BYTES);
-              uint8_t* dst = sm + (kv ? C::OFF_V : C::OFF_K) + t * C::TILE_BYTES;
-              const int kvh = t ? I.kvh1 : I.kvh0;
-              const int col = (kv ? Hq + Hkv + kvh : Hq + kvh) * DH;
-#pragma unroll
-              for (int bx = 0; bx < DH / 64; ++bx)
-                tma_load_2d(dst + bx * C::BOX_BYTES, &tm, &bar[f_bar], col + bx * 64, I.s0 + j * BKV);
-            }
-            if (!ok) break;
-          }
+          for (int bx = 0; bx < DH / 64; ++bx)
+            tma_load_2d(sV + bx * C::BOX_KV, &tmKV, vfull, vcol + bx * 64, I.s0 + j * BKV);
         }
         ++nitem;
       }
       // every copy lands before the CTA may exit (bounded waits; normally
       // the consumers have waited for all of them already)
-      if (nitem > 0)
-        for (int t = 0; t < 2; ++t) mbar_wait(&bar[Q_FULL + t], (nitem - 1) & 1, err);
-      if (g > 0)
-        for (int t = 0; t < 2; ++t) {
-          mbar_wait(&bar[K_FULL + t], (g - 1) & 1, err);
-          mbar_wait(&bar[V_FULL + t], (g - 1) & 1, err);
-        }
+      if (nitem > 0) mbar_wait(&bar[Q_FULL + t], (nitem - 1) & 1, err);
+      for (uint32_t gg = g >= 2 ? g - 2 : 0; gg < g; ++gg) {
+        mbar_wait(&bar[K_FULL + 2 * t + (gg & 1)], (gg >> 1) & 1, err);
+        mbar_wait(&bar[P_FULL + 2 * t + (gg & 1)], (gg >> 1) & 1, err);  // (V, and the block's P)
+      }
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 || warp == 2) {
+    // ------------------------------------------------------------ MMA issuer of head t
     if (lane == 0) {
+      const int t = warp - 1;
       constexpr uint32_t IDESC_S = umma_idesc_bf16_f32(BQ, BKV);
       constexpr uint32_t IDESC_O = umma_idesc_bf16_f32(BQ, DH) | (1u << 16);  // B (V) MN-major
+      // shared-memory descriptors of the stage bases; a K step adds its byte
+      // offset / 16 to the address field (it stays below the field's 14 bits)
+      const uint64_t dQ = umma_desc_sw128(smem_u32(sm + C::OFF_Q + t * C::Q_BYTES));
+      const uint64_t dK0 = umma_desc_sw128(smem_u32(sm + C::OFF_K + 2 * t * C::KV_BYTES));
+      const uint64_t dK1 = umma_desc_sw128(smem_u32(sm + C::OFF_K + (2 * t + 1) * C::KV_BYTES));
+      const uint64_t dV0 = umma_desc_sw128_mn(smem_u32(sm + C::OFF_V + 2 * t * C::KV_BYTES), C::BOX_KV);
+      const uint64_t dV1 = umma_desc_sw128_mn(smem_u32(sm + C::OFF_V + (2 * t + 1) * C::KV_BYTES), C::BOX_KV);
+      const uint32_t tS = tmem + t * 128, tO = tmem + C::T_O + t * DH;
       uint32_t g = 0, nitem = 0;
       bool ok = true;
+      // scores of global block gg (= block j of the current item)
+      auto issue_s = [&](uint32_t gg, bool last) -> bool {
+        const uint32_t b = gg & 1, ph = (gg >> 1) & 1;
+        // buffer b held P of block gg - 2: its O += P V must be complete
+        if (!mbar_wait(&bar[K_FULL + 2 * t + b], ph, err) ||
+            (gg >= 2 && !mbar_wait(&bar[PV_DONE + 2 * t + b], ph ^ 1u, err)))
+          return false;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk)
+          umma_bf16(tS + b * BKV, dQ + (((kk >> 2) * C::BOX_Q + (kk & 3) * 32) >> 4),
+                    (b ? dK1 : dK0) + (((kk >> 2) * C::BOX_KV + (kk & 3) * 32) >> 4), IDESC_S, kk ? 1u : 0u);
+        umma_commit(&bar[S_FULL + 2 * t + b]);
+        if (last) umma_commit(&bar[Q_EMPTY + t]);
+        return true;
+      };
+      // O += P V of global block gg (block j of the current item)
+      auto issue_pv = [&](uint32_t gg, int j, bool last) -> bool {
+        const uint32_t b = gg & 1, ph = (gg >> 1) & 1;
+        // (P_FULL completes once the softmax wrote P and this block's V landed)
+        if (!mbar_wait(&bar[P_FULL + 2 * t + b], ph, err) ||
+            (j == 0 && !mbar_wait(&bar[O_EMPTY + t], (nitem & 1) ^ 1u, err)))
+          return false;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < BKV / 16; ++kk)
+          umma_bf16_ta(tO, tS + b * BKV + kk * 8, (b ? dV1 : dV0) + ((kk * 2048) >> 4), IDESC_O, (j | kk) ? 1u : 0u);
+        umma_commit(&bar[PV_DONE + 2 * t + b]);
+        if (last) umma_commit(&bar[O_FULL + t]);
+        return true;
+      };
       for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
         Item I;
         if (!item_at(it, cu, B, HP, n_tiles, Hq, Hkv, causal, I)) continue;
-        for (int t = 0; t < 2 && ok; ++t) ok = mbar_wait(&bar[Q_FULL + t], nitem & 1, err);
-        for (int j = 0; ok && j < I.nkv; ++j, ++g) {
-          const uint32_t ph = g & 1;
-          const bool last = j == I.nkv - 1;
-#pragma unroll
-          for (int t = 0; t < 2; ++t) {
-            // S_t overwrites P_t: the previous O_t += P_t V_t must be complete
-            if (!mbar_wait(&bar[K_FULL + t], ph, err) || (g > 0 && !mbar_wait(&bar[PV_DONE + t], (g - 1) & 1, err))) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            const uint32_t a0 = smem_u32(sm + C::OFF_Q + t * C::TILE_BYTES);
-            const uint32_t b0 = smem_u32(sm + C::OFF_K + t * C::TILE_BYTES);
-#pragma unroll
-            for (int kk = 0; kk < DH / 16; ++kk) {
-              const uint32_t o = (kk >> 2) * C::BOX_BYTES + (kk & 3) * 32;
-              umma_bf16(tmem + t * BKV, umma_desc_sw128(a0 + o), umma_desc_sw128(b0 + o), IDESC_S, kk ? 1u : 0u);
-            }
-            umma_commit(&bar[S_FULL + t]);
-            umma_commit(&bar[K_EMPTY + t]);
-            if (last) umma_commit(&bar[Q_EMPTY + t]);
-          }
-          if (!ok) break;
-#pragma unroll
-          for (int t = 0; t < 2; ++t) {
-            if (!mbar_wait(&bar[V_FULL + t], ph, err) || !mbar_wait(&bar[P_FULL + t], ph, err) ||
-                (j == 0 && !mbar_wait(&bar[O_EMPTY + t], (nitem & 1) ^ 1u, err))) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            const uint32_t bv = smem_u32(sm + C::OFF_V + t * C::TILE_BYTES);
-#pragma unroll
-            for (int kk = 0; kk < BKV / 16; ++kk)
-              umma_bf16_ta(tmem + C::T_O + t * DH, tmem + t * BKV + kk * 8,
-                           umma_desc_sw128_mn(bv + kk * 2048, C::BOX_BYTES), IDESC_O, (j | kk) ? 1u : 0u);
-            umma_commit(&bar[PV_DONE + t]);
-            umma_commit(&bar[V_EMPTY + t]);
-            if (last) umma_commit(&bar[O_FULL + t]);
-          }
+        ok = mbar_wait(&bar[Q_FULL + t], nitem & 1, err) && issue_s(g, I.nkv == 1);
+        for (int j = 0; ok && j < I.nkv; ++j) {
+          if (j + 1 < I.nkv) ok = issue_s(g + j + 1, j + 2 == I.nkv);
+          ok = ok && issue_pv(g + j, j, j + 1 == I.nkv);
         }
+        g += I.nkv;
         ++nitem;
       }
-      umma_commit(&bar[MMA_DONE]);  // TMEM stays allocated until every issued MMA is done
-      mbar_wait(&bar[MMA_DONE], 0, err);
+      umma_commit(&bar[MMA_DONE + t]);  // TMEM stays allocated until every issued MMA is done
+      mbar_wait(&bar[MMA_DONE + t], 0, err);
     }
     __syncwarp();
   } else if (warp >= 4) {
@@ -240,7 +253,7 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    const uint32_t tS = trow + t * BKV, tO = trow + C::T_O + t * DH;
+    const uint32_t tS = trow + t * 128, tO = trow + C::T_O + t * DH;
     uint32_t g = 0, nitem = 0;
     bool ok = true;
     for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
@@ -250,11 +263,12 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict
       const int row_lim = qpos >= I.len ? 0 : (causal ? qpos + 1 : I.len);  // keys [0, row_lim) are visible
       float m = -INFINITY, l = 0.f;  // m: running max in log2 units
       for (int j = 0; j < I.nkv; ++j, ++g) {
-        if (!mbar_wait_warp(&bar[S_FULL + t], g & 1, err)) { ok = false; break; }
+        const uint32_t b = g & 1;
+        if (!mbar_wait_warp(&bar[S_FULL + 2 * t + b], (g >> 1) & 1, err)) { ok = false; break; }
         tc_fence_after();
         float v[BKV];
-#pragma unroll
-        for (int c = 0; c < BKV; c += 32) tmem_ld_32x32b_x32(tS + c, *reinterpret_cast<float(*)[32]>(v + c));
+        tmem_ld_32x32b_x32(tS + b * BKV, *reinterpret_cast<float(*)[32]>(v));
+        tmem_ld_32x32b_x32(tS + b * BKV + 32, *reinterpret_cast<float(*)[32]>(v + 32));
         tmem_ld_wait();
         const int lim = row_lim - j * BKV;
         if (lim < BKV) {
@@ -291,9 +305,8 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict
         }
         l = l * corr + ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
         if (__any_sync(0xffffffffu, moved)) {
-          // O += P V of the previous block has finished with O (it completed
-          // before this block's S was issued; the wait makes it explicit)
-          if (!mbar_wait_warp(&bar[PV_DONE + t], (g - 1) & 1, err)) { ok = false; break; }
+          // O += P V of the previous block must be done with O before it is rescaled
+          if (!mbar_wait_warp(&bar[PV_DONE + 2 * t + ((g - 1) & 1)], ((g - 1) >> 1) & 1, err)) { ok = false; break; }
           tc_fence_after();
           float o[32];
 #pragma unroll 1
@@ -305,12 +318,11 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tm, __nv_bfloat16* __restrict
             tmem_st_32x32b_x32(tO + c, o);
           }
         }
-        tmem_st_32x32b_x32(tS, *reinterpret_cast<float(*)[32]>(pk));
-        tmem_st_32x32b_x32(tS + 32, *reinterpret_cast<float(*)[32]>(pk + 32));
+        tmem_st_32x32b_x32(tS + b * BKV, pk);
         tmem_st_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bar[P_FULL + t]);
+        if (lane == 0) mbar_arrive(&bar[P_FULL + 2 * t + b]);
       }
       if (!ok) break;
       // ---- O / l to global
@@ -369,13 +381,14 @@ cudaError_t launch_attn_fa(const void* qkv, void* out, const int* cu, int B, int
   }
   if (Hkv <= 0 || Hq % Hkv != 0) return cudaErrorInvalidValue;
   const int ld_qkv = (Hq + 2 * Hkv) * DH;
-  CUtensorMap tm;
-  if (!encode_tmap_2d(&tm, qkv, false, (uint64_t)rows_cap, (uint64_t)ld_qkv, 64, fa::BQ, nullptr))
+  CUtensorMap tq, tkv;
+  if (!encode_tmap_2d(&tq, qkv, false, (uint64_t)rows_cap, (uint64_t)ld_qkv, 64, fa::BQ, nullptr) ||
+      !encode_tmap_2d(&tkv, qkv, false, (uint64_t)rows_cap, (uint64_t)ld_qkv, 64, fa::BKV, nullptr))
     return cudaErrorInvalidValue;
   const int n_tiles = (max_len + fa::BQ - 1) / fa::BQ;
   const long n_items = (long)n_tiles * B * ((Hq + 1) / 2);
   const int grid = (int)std::min<long>(n_items, (long)device_sm_count());
-  return launch_pdl(fa::attn_fa_kernel<DH>, dim3(grid), dim3(fa::NTHR), C::SMEM, st, tm,
+  return launch_pdl(fa::attn_fa_kernel<DH>, dim3(grid), dim3(fa::NTHR), C::SMEM, st, tq, tkv,
                     reinterpret_cast<__nv_bfloat16*>(out), cu, B, Hq, Hkv, n_tiles, Hq * DH, causal ? 1 : 0,
                     scale_log2, err);
 }

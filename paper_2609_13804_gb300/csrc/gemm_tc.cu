@@ -726,29 +726,6 @@ SP_DEVINL int sched_contributors(const Sched& s, int t) {
   return n;
 }
 
-SP_DEVINL int ld_acquire_gpu(const int* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
-SP_DEVINL void st_release_gpu(int* p, int v) {
-  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-// The calling thread waits until *flag == 1 (bounded).
-SP_DEVINL bool wait_flag(const int* flag, int* err) {
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t i = 0;; ++i) {
-    if (ld_acquire_gpu(flag) == 1) return true;
-    if ((i & 63u) == 0 && globaltimer_ns() - t0 > kWaitLimitNs) {
-      set_error(err, SP_DEVERR_TIMEOUT);
-      return false;
-    }
-    __nanosleep(32);
-  }
-}
-
 // ---------------------------------------------------------------------------
 // CTA-pair variant (cta_group::2): a cluster of two CTAs on two SMs computes a
 // 256 x BN tile with M = 256 MMAs issued by the even CTA.  Each CTA stages its

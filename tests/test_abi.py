@@ -124,3 +124,11 @@ def test_mrope_argument_checks(L):
     assert L.sp_mrope_positions(*args(b._int_array([4, 10]), 8, ok)) == 2  # grid wider than the image
     assert L.sp_mrope_positions(*args(gw, 8, None)) == 1
     assert L.sp_mrope_positions(*args(gw, 8, C.c_void_p(260))) == 3         # pos3 misaligned
+
+
+def test_wait_probe_argument_checks_fail_before_any_launch(L):
+    one = C.c_int(0)
+    assert L.sp_wait_probe(None, 1000, 0, C.byref(one), None, None) == 1      # SP_ERR_INVALID_ARG: no flag
+    assert L.sp_wait_probe(C.byref(one), 0, 0, C.byref(one), None, None) == 2  # SP_ERR_SHAPE: limit 0
+    assert L.sp_wait_probe(C.byref(one), 2000001, 0, C.byref(one), None, None) == 2
+    assert L.sp_device_error_status(0x1) == 6   # SP_DEVERR_TIMEOUT -> SP_ERR_TIMEOUT
