@@ -509,10 +509,13 @@ def run_ours(args):
     compact_ms = kernel_ms_cold(lambda: do_compact(sel_out["idx"], sel_out["count"], k_cap, reuse=True))
     comp_bytes = 2.0 * (K_sum * s.D + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
 
+    icomp = {}
+
     def prefill_stage(idx, count, kc):
-        do_compact(idx, count, kc)
-        o = comp["o"]
-        B.sp_project(model, vis_packed=o["vis_packed"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
+        # the pipeline's form: index-mode compaction, the projector gathering the kept rows of X
+        o = icomp[kc] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
+                                     index_mode=True, out=icomp.get(kc))
+        B.sp_project(model, X=X, vis_src=o["vis_src"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
                      packed=o["packed"], rows_cap=o["rows_cap"], B=w.B)
         lens_cap = max(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
         B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=w.B, T_cap=o["T_cap"],
@@ -868,21 +871,23 @@ def measure_config(B, torch, tm, w, model, dev, gen, pk, *, targets, mean_target
     proj = m.proj_kind != "none"
     comp = {}
 
-    def compact(idx, count, kc, key):
+    def compact(idx, count, kc, key, index_mode=False):
         comp[key] = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=idx, count=count, k_cap=kc,
-                                 projector_mode=proj, out=comp.get(key))
+                                 projector_mode=proj and not index_mode, index_mode=proj and index_mode,
+                                 out=comp.get(key))
         return comp[key]
 
     r = sws["r"]
-    compact_ms = tm.cold(lambda: compact(r["idx"], r["count"], pipe.k_cap, "p"))
+    # the gather as its own kernel (the copy the pipeline folds into the projector's operand loads)
+    compact_ms = tm.cold(lambda: compact(r["idx"], r["count"], pipe.k_cap, "c"))
     vis_w = s.D
     comp_bytes = 2.0 * (K_sum * vis_w + sum(w.n_txt) * m.d) * 2 + 4.0 * (w.B + 1 + T)
     st = {}
 
     def prefill_stage(idx, count, kc, key):
-        o = compact(idx, count, kc, key)
+        o = compact(idx, count, kc, key, index_mode=True)
         if proj:
-            B.sp_project(model, vis_packed=o["vis_packed"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
+            B.sp_project(model, X=X, vis_src=o["vis_src"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
                          packed=o["packed"], rows_cap=o["rows_cap"], B=w.B, ws=st.get(key + "pw"))
         lens_cap = max(min(n, kc) + t for n, t in zip(w.n_vis, w.n_txt))
         res = B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=w.B, T_cap=o["T_cap"],
@@ -1021,10 +1026,10 @@ def scaling_rows(B, torch, dev, gen, selector, model, steps, warmup):
         st = {}
 
         def full_prefill():
-            o = B.sp_compact([N], [L], X=X, text=E, idx=full_idx, count=full_cnt, k_cap=N, projector_mode=True,
+            o = B.sp_compact([N], [L], X=X, text=E, idx=full_idx, count=full_cnt, k_cap=N, index_mode=True,
                              out=st.get("c"))
             st["c"] = o
-            B.sp_project(model, vis_packed=o["vis_packed"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
+            B.sp_project(model, X=X, vis_src=o["vis_src"], vis_row_map=o["vis_row_map"], vis_cu=o["vis_cu"],
                          packed=o["packed"], rows_cap=o["rows_cap"], B=1)
             r = B.sp_prefill(model, x=o["packed"], cu_seqlens=o["cu_seqlens"], pos=o["pos"], B=1, T_cap=o["T_cap"],
                              max_seqlen_cap=N + L, ws=st.get("ws"), hidden=st.get("h"))

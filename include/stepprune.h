@@ -248,6 +248,9 @@ SP_API sp_status sp_select(const sp_selector* s, const sp_select_in* in, const s
  *     that device current); make that first call before any stream capture.
  *   - All calls share the array and it keeps the last call's contents: calls
  *     whose GPU work overlaps (several streams or threads) race; serialise them.
+ *   - The device address found by the first call is kept for the process's
+ *     life: do not use this entry point across a device reset
+ *     (cudaDeviceReset tears down the context the address belongs to).
  */
 #define SP_SELECT_NOALLOC_SCRATCH_BYTES (64u << 20)
 SP_API sp_status sp_select_noalloc(const sp_selector* s, const sp_select_in* in, const sp_select_out* out,
@@ -346,10 +349,15 @@ typedef struct {
   void* packed;          /* DEVICE [T_cap, W_txt] bf16 */
   int* cu_seqlens;       /* DEVICE [B + 1] */
   int* pos;              /* DEVICE [T_cap] */
-  void* vis_packed;      /* DEVICE [sum_b min(n_vis[b], k_cap), W_vis] bf16, or NULL (direct) */
-  int* vis_row_map;      /* DEVICE [same rows] (projector mode) */
-  int* vis_cu;           /* DEVICE [B + 1] (projector mode) */
+  void* vis_packed;      /* DEVICE [sum_b min(n_vis[b], k_cap), W_vis] bf16, or NULL (direct / index mode) */
+  int* vis_row_map;      /* DEVICE [same rows] (projector and index modes) */
+  int* vis_cu;           /* DEVICE [B + 1] (projector and index modes) */
   int* err;              /* DEVICE error word or NULL */
+  int* vis_src;          /* DEVICE [same rows] int32, or NULL.  Index mode (vis_src set,
+                            vis_packed NULL): no visual row is copied; vis_src[i] is the row of
+                            X that kept visual row i comes from, and sp_project (io.vis_src)
+                            gathers those rows itself: Alg. 1 step 5's gather folded into the
+                            projector's operand load.  An invalid index gives vis_src -1. */
 } sp_compact_out;
 
 /* T_cap of a batch (host arithmetic; -1 on bad arguments). */
@@ -410,18 +418,24 @@ SP_API sp_status sp_model_create(const sp_model_cfg* cfg, const sp_model_weights
 SP_API void sp_model_destroy(sp_model* m);
 
 /*
- * Projector on the kept rows: packed[vis_row_map[i]] = P(vis_packed[i]) for
- * i < vis_cu[B] (device count), P = W1 x, or W2 GELU(W1 x).  rows_cap bounds
+ * Projector on the kept rows (Sec. 3.3, last paragraph: restored, then
+ * projected): packed[vis_row_map[i]] = P(x_i) for i < vis_cu[B] (device
+ * count), P = W1 x, or W2 GELU(W1 x), with x_i = vis_packed[i], or, when
+ * vis_src is given, x_i = X[vis_src[i]] read by the first GEMM's operand loads
+ * (row-gather TMA) so that the kept rows are never copied.  rows_cap bounds
  * vis_cu[B].
  */
 typedef struct {
   int B;
   int rows_cap;
-  const void* vis_packed;   /* DEVICE [rows_cap, proj_in] bf16 */
+  const void* vis_packed;   /* DEVICE [rows_cap, proj_in] bf16 (ignored with vis_src) */
   const int* vis_row_map;   /* DEVICE [rows_cap] */
   const int* vis_cu;        /* DEVICE [B + 1] */
   void* packed;             /* DEVICE [T_cap, d] bf16 (visual slots written) */
   int* err;
+  const void* X;            /* DEVICE [rows_X, proj_in] bf16 visual tokens (with vis_src) */
+  int rows_X;               /* rows of X (with vis_src) */
+  const int* vis_src;       /* DEVICE [rows_cap] rows of X (sp_compact's index mode), or NULL */
 } sp_project_io;
 
 SP_API size_t sp_project_workspace(const sp_model* m, int rows_cap);

@@ -87,7 +87,7 @@ class sp_compact_in(C.Structure):
 
 class sp_compact_out(C.Structure):
     _fields_ = [("packed", P), ("cu_seqlens", P), ("pos", P), ("vis_packed", P), ("vis_row_map", P),
-                ("vis_cu", P), ("err", P)]
+                ("vis_cu", P), ("err", P), ("vis_src", P)]
 
 
 class sp_model_cfg(C.Structure):
@@ -105,7 +105,7 @@ class sp_model_weights(C.Structure):
 
 class sp_project_io(C.Structure):
     _fields_ = [("B", C.c_int), ("rows_cap", C.c_int), ("vis_packed", P), ("vis_row_map", P), ("vis_cu", P),
-                ("packed", P), ("err", P)]
+                ("packed", P), ("err", P), ("X", P), ("rows_X", C.c_int), ("vis_src", P)]
 
 
 class sp_prefill_io(C.Structure):
@@ -407,10 +407,13 @@ def sp_vp_gate(*, X, noise, alpha, out=None, stream=None):
 
 # ----------------------------------------------------------------------------- compaction
 
-def sp_compact(n_vis, n_txt, *, X, text, idx, count, k_cap, projector_mode=False, stream=None,
+def sp_compact(n_vis, n_txt, *, X, text, idx, count, k_cap, projector_mode=False, index_mode=False, stream=None,
                out: Optional[Dict] = None) -> Dict:
     """Compaction into new zero-filled outputs, or into `out` (a dict a
-    previous call returned for the same sizes) without touching it first."""
+    previous call returned for the same sizes) without touching it first.
+    projector_mode: the kept visual rows go to out['vis_packed'] (with their
+    packed rows in 'vis_row_map'); index_mode: no visual row is copied,
+    out['vis_src'] holds the row of X each kept visual row comes from."""
     torch = _torch()
     dev = X.device
     keep: List = []
@@ -419,30 +422,26 @@ def sp_compact(n_vis, n_txt, *, X, text, idx, count, k_cap, projector_mode=False
     W_vis, W_txt = X.shape[1], text.shape[1]
     T_cap = sp_packed_cap(n_vis, n_txt, k_cap)
     rows_cap = sum(min(n, k_cap) for n in n_vis)
-    if out is not None:
-        if out["T_cap"] != T_cap or (projector_mode and out.get("rows_cap") != rows_cap):
-            raise ValueError("sp_compact: `out` was made for other sizes")
-        ci = sp_compact_in(len(n_vis), C.cast(nv, IP), C.cast(nt, IP), ptr(X), int(W_vis), ptr(text), int(W_txt),
-                           ptr(idx), int(k_cap), ptr(count))
-        co = sp_compact_out(ptr(out["packed"]), ptr(out["cu_seqlens"]), ptr(out["pos"]),
-                            ptr(out.get("vis_packed") if projector_mode else None),
-                            ptr(out.get("vis_row_map") if projector_mode else None),
-                            ptr(out.get("vis_cu") if projector_mode else None), ptr(out["err"]))
-        _check(lib().sp_compact(C.byref(ci), C.byref(co), _stream(stream)), "sp_compact")
-        return out
-    out = {"packed": torch.zeros((max(T_cap, 1), W_txt), dtype=torch.bfloat16, device=dev),
-           "cu_seqlens": torch.zeros(len(n_vis) + 1, dtype=torch.int32, device=dev),
-           "pos": torch.full((max(T_cap, 1),), -1, dtype=torch.int32, device=dev),
-           "err": torch.zeros(1, dtype=torch.int32, device=dev), "T_cap": T_cap}
-    if projector_mode:
-        out["vis_packed"] = torch.zeros((max(rows_cap, 1), W_vis), dtype=torch.bfloat16, device=dev)
-        out["vis_row_map"] = torch.full((max(rows_cap, 1),), -1, dtype=torch.int32, device=dev)
-        out["vis_cu"] = torch.zeros(len(n_vis) + 1, dtype=torch.int32, device=dev)
-        out["rows_cap"] = rows_cap
+    mode = "index" if index_mode else ("projector" if projector_mode else "direct")
+    if out is None:
+        out = {"packed": torch.zeros((max(T_cap, 1), W_txt), dtype=torch.bfloat16, device=dev),
+               "cu_seqlens": torch.zeros(len(n_vis) + 1, dtype=torch.int32, device=dev),
+               "pos": torch.full((max(T_cap, 1),), -1, dtype=torch.int32, device=dev),
+               "err": torch.zeros(1, dtype=torch.int32, device=dev), "T_cap": T_cap, "mode": mode}
+        if mode != "direct":
+            out["vis_row_map"] = torch.full((max(rows_cap, 1),), -1, dtype=torch.int32, device=dev)
+            out["vis_cu"] = torch.zeros(len(n_vis) + 1, dtype=torch.int32, device=dev)
+            out["rows_cap"] = rows_cap
+        if mode == "projector":
+            out["vis_packed"] = torch.zeros((max(rows_cap, 1), W_vis), dtype=torch.bfloat16, device=dev)
+        if mode == "index":
+            out["vis_src"] = torch.full((max(rows_cap, 1),), -1, dtype=torch.int32, device=dev)
+    elif out["T_cap"] != T_cap or out.get("mode") != mode or (mode != "direct" and out.get("rows_cap") != rows_cap):
+        raise ValueError("sp_compact: `out` was made for other sizes or another mode")
     ci = sp_compact_in(len(n_vis), C.cast(nv, IP), C.cast(nt, IP), ptr(X), int(W_vis), ptr(text), int(W_txt),
                        ptr(idx), int(k_cap), ptr(count))
     co = sp_compact_out(ptr(out["packed"]), ptr(out["cu_seqlens"]), ptr(out["pos"]), ptr(out.get("vis_packed")),
-                        ptr(out.get("vis_row_map")), ptr(out.get("vis_cu")), ptr(out["err"]))
+                        ptr(out.get("vis_row_map")), ptr(out.get("vis_cu")), ptr(out["err"]), ptr(out.get("vis_src")))
     _check(lib().sp_compact(C.byref(ci), C.byref(co), _stream(stream)), "sp_compact")
     return out
 
@@ -499,10 +498,14 @@ class Model:
             pass
 
 
-def sp_project(model: Model, *, vis_packed, vis_row_map, vis_cu, packed, rows_cap, B, stream=None, ws=None):
+def sp_project(model: Model, *, vis_row_map, vis_cu, packed, rows_cap, B, vis_packed=None, X=None, vis_src=None,
+               stream=None, ws=None):
+    """The projector on the kept rows: from vis_packed (projector-mode
+    compaction), or gathered from X by vis_src (index-mode compaction)."""
     torch = _torch()
     err = torch.zeros(1, dtype=torch.int32, device=packed.device)
-    io = sp_project_io(int(B), int(rows_cap), ptr(vis_packed), ptr(vis_row_map), ptr(vis_cu), ptr(packed), ptr(err))
+    io = sp_project_io(int(B), int(rows_cap), ptr(vis_packed), ptr(vis_row_map), ptr(vis_cu), ptr(packed), ptr(err),
+                       ptr(X), int(X.shape[0]) if X is not None else 0, ptr(vis_src))
     if ws is None:
         ws = workspace(lib().sp_project_workspace(model.handle, int(rows_cap)), packed.device)
     _check(lib().sp_project(model.handle, C.byref(io), ptr(ws), ws.numel(), _stream(stream)), "sp_project")

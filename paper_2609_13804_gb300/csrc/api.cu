@@ -753,14 +753,18 @@ static sp_status compact_impl(const sp_compact_in* in, const sp_compact_out* out
   if (in->W_vis <= 0 || in->W_vis % 8 || in->W_txt <= 0 || in->W_txt % 8)
     return fail(SP_ERR_SHAPE, "sp_compact: W_vis and W_txt must be positive multiples of 8");
   if (in->k_cap < 0) return fail(SP_ERR_SHAPE, "sp_compact: k_cap must be >= 0");
-  const bool direct = out->vis_packed == nullptr;
+  const bool index_mode = out->vis_src != nullptr;
+  if (index_mode && out->vis_packed) return fail(SP_ERR_INVALID_ARG, "sp_compact: vis_src and vis_packed are exclusive");
+  const bool direct = out->vis_packed == nullptr && !index_mode;
   if (direct && in->W_vis != in->W_txt) return fail(SP_ERR_SHAPE, "sp_compact: direct mode needs W_vis == W_txt");
-  if (!direct && (!out->vis_row_map || !out->vis_cu)) return fail(SP_ERR_INVALID_ARG, "sp_compact: vis_row_map and vis_cu required with vis_packed");
+  if (!direct && (!out->vis_row_map || !out->vis_cu))
+    return fail(SP_ERR_INVALID_ARG, "sp_compact: vis_row_map and vis_cu required with vis_packed / vis_src");
   if (!al16(in->X) || (in->text && !al16(in->text)) || !al16(out->packed) || (out->vis_packed && !al16(out->vis_packed)))
     return fail(SP_ERR_ALIGN, "sp_compact: row buffers must be 16-byte aligned");
   const int T_cap = sp_packed_cap(in->B, in->n_vis, in->n_txt, in->k_cap);
   SP_CUDA(compact_launch(bd, in->X, in->W_vis, in->text, in->W_txt, in->idx, in->k_cap, in->count, out->packed,
-                         out->cu_seqlens, out->pos, out->vis_packed, out->vis_row_map, out->vis_cu, T_cap, out->err, st),
+                         out->cu_seqlens, out->pos, out->vis_packed, out->vis_row_map, out->vis_cu, out->vis_src,
+                         T_cap, out->err, st),
           "compaction");
   return SP_OK;
 }
@@ -885,9 +889,12 @@ static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* 
   const sp_model_cfg& c = m->cfg;
   if (c.proj_kind == SP_PROJ_NONE) return SP_OK;
   if (io->B < 1 || io->B > SP_MAX_BATCH || io->rows_cap < 0) return fail(SP_ERR_SHAPE, "sp_project: bad B / rows_cap");
-  if (!io->vis_packed || !io->vis_row_map || !io->vis_cu || !io->packed)
-    return fail(SP_ERR_INVALID_ARG, "sp_project: vis_packed, vis_row_map, vis_cu and packed are required");
-  if (!al16(io->vis_packed) || !al16(io->packed)) return fail(SP_ERR_ALIGN, "sp_project: buffers must be 16-byte aligned");
+  const bool gather = io->vis_src != nullptr;
+  if ((!gather && !io->vis_packed) || !io->vis_row_map || !io->vis_cu || !io->packed)
+    return fail(SP_ERR_INVALID_ARG, "sp_project: vis_packed (or vis_src), vis_row_map, vis_cu and packed are required");
+  if (gather && (!io->X || io->rows_X < 1)) return fail(SP_ERR_INVALID_ARG, "sp_project: vis_src needs X and rows_X >= 1");
+  if ((!gather && !al16(io->vis_packed)) || (gather && !al16(io->X)) || !al16(io->packed))
+    return fail(SP_ERR_ALIGN, "sp_project: buffers must be 16-byte aligned");
   if (io->rows_cap == 0) return SP_OK;
   Carve cv(ws);
   void* tmp = nullptr;
@@ -906,8 +913,13 @@ static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* 
   }
   SP_CUDA(gemm_scratch_clear(gs, st), "GEMM scratch");
   std::string msg;
+  // the first GEMM's A: the packed kept rows, or the rows of X they come from
+  // (row-gather map: a box of one row, gathered four rows per copy)
   CUtensorMap tV;
-  if (!encode_tmap_bf16(&tV, io->vis_packed, io->rows_cap, c.proj_in, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  if (gather ? !encode_tmap_bf16(&tV, io->X, io->rows_X, c.proj_in, 1, &msg)
+             : !encode_tmap_bf16(&tV, io->vis_packed, io->rows_cap, c.proj_in, 128, &msg))
+    return fail(SP_ERR_CUDA, "%s", msg.c_str());
+  const int* a_rows = gather ? io->vis_src : nullptr;
   const int* M_dev = io->vis_cu + io->B;
   GemmEpi sc;
   sc.kind = EPI_SCATTER_BF16;
@@ -915,14 +927,16 @@ static sp_status project_impl(const sp_model* m, const sp_project_io* io, void* 
   sc.ldo = c.d;
   sc.row_map = io->vis_row_map;
   if (c.proj_kind == SP_PROJ_LINEAR) {
-    SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.d, sc, io->err, st, &gs), "projector");
+    SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.d, sc, io->err, st, &gs, nullptr, nullptr, a_rows),
+            "projector");
     return SP_OK;
   }
   GemmEpi g1;
   g1.kind = EPI_GELU_BF16;
   g1.out = tmp;
   g1.ldo = c.proj_hidden;
-  SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.proj_hidden, g1, io->err, st, &gs), "projector fc1");
+  SP_CUDA(gemm_bf16(tV, io->rows_cap, M_dev, m->p1, c.proj_hidden, g1, io->err, st, &gs, nullptr, nullptr, a_rows),
+          "projector fc1");
   CUtensorMap tT;
   if (!encode_tmap_bf16(&tT, tmp, io->rows_cap, c.proj_hidden, 128, &msg)) return fail(SP_ERR_CUDA, "%s", msg.c_str());
   SP_CUDA(gemm_bf16(tT, io->rows_cap, M_dev, m->p2, c.d, sc, io->err, st, &gs), "projector fc2");
@@ -1207,7 +1221,7 @@ sp_status plan_pipe(const sp_selector* s, const sp_model* m, const sp_select_in&
 struct PipeParts {
   void* packed;
   int* pos;
-  void* vis_packed;
+  int* vis_src;  // the projector gathers the kept rows from X (compaction's index mode)
   int* vis_row_map;
   int* vis_cu;
   void* scratch;
@@ -1220,7 +1234,7 @@ size_t pipe_ws(const sp_selector* s, const sp_model* m, const sp_select_in& sel,
   q.packed = cv.take<uint16_t>((size_t)std::max(pp.T_cap, 1) * m->cfg.d);
   q.pos = cv.take<int>((size_t)std::max(pp.T_cap, 1));
   const bool proj = m->cfg.proj_kind != SP_PROJ_NONE;
-  q.vis_packed = proj ? cv.take<uint16_t>((size_t)std::max(pp.rows_cap, 1) * s->cfg.D) : nullptr;
+  q.vis_src = proj ? cv.take<int>((size_t)std::max(pp.rows_cap, 1)) : nullptr;
   q.vis_row_map = proj ? cv.take<int>((size_t)std::max(pp.rows_cap, 1)) : nullptr;
   q.vis_cu = proj ? cv.take<int>(SP_MAX_BATCH + 1) : nullptr;
   SelPlan sp_;
@@ -1292,21 +1306,25 @@ static sp_status pipeline_impl(const sp_selector* s, const sp_model* m, const sp
   co.packed = q.packed;
   co.cu_seqlens = io->cu_seqlens;
   co.pos = q.pos;
-  co.vis_packed = q.vis_packed;
+  co.vis_src = q.vis_src;
   co.vis_row_map = q.vis_row_map;
   co.vis_cu = q.vis_cu;
   co.err = io->err;
   r = compact_impl(&ci, &co, st);
   if (r != SP_OK) return r;
   if (proj) {
+    int rows_X = 0;
+    for (int b = 0; b < si.B; ++b) rows_X += si.n_vis[b];
     sp_project_io pj = {};
     pj.B = si.B;
     pj.rows_cap = pp.rows_cap;
-    pj.vis_packed = q.vis_packed;
     pj.vis_row_map = q.vis_row_map;
     pj.vis_cu = q.vis_cu;
     pj.packed = q.packed;
     pj.err = io->err;
+    pj.X = si.X;
+    pj.rows_X = std::max(1, rows_X);
+    pj.vis_src = q.vis_src;
     r = project_impl(m, &pj, q.scratch, q.scratch_bytes, st);
     if (r != SP_OK) return r;
   }

@@ -178,6 +178,19 @@ SP_DEVINL void tma_gather4_2d(void* smem_dst, const void* tmap, uint64_t* bar, i
       : "memory");
 }
 
+// Row gather into this CTA's shared memory, completing on an mbarrier that may
+// live in the peer CTA of the pair (cluster address): tma_gather4_2d's CTA-pair
+// form (the A rows of a cta_group::2 GEMM).
+SP_DEVINL void tma_gather4_2d_pair(void* smem_dst, const void* tmap, uint32_t mbar_cluster_addr, int x, int r0,
+                                   int r1, int r2, int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];"
+      ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(r0), "r"(r1), "r"(r2),
+        "r"(r3), "r"(mbar_cluster_addr)
+      : "memory");
+}
+
 // 2-D tiled bulk tensor store shared -> global of one box (bulk-group
 // completion).  The same x alignment rule as for loads applies.
 SP_DEVINL void tma_store_2d(const void* tmap, const void* smem_src, int x, int y) {

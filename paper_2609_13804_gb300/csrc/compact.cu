@@ -7,6 +7,10 @@
 // Every block recomputes the (small) prefix sums of the per-image counts from
 // the device counts, so the kernel needs no host round trip and no second
 // launch; block 0 publishes cu_seqlens / vis_cu.
+//
+// Index mode (vis_src): the kept visual rows are not copied; the kernel writes,
+// for each, the row of X it comes from (with vis_row_map, its packed row), and
+// the projector's first GEMM gathers those rows from X as its operand.
 #include "common.cuh"
 #include "internal.h"
 
@@ -21,7 +25,7 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
                const __nv_bfloat16* __restrict__ text, int W_txt, const int* __restrict__ idx, int k_cap,
                const int* __restrict__ count, __nv_bfloat16* __restrict__ packed, int* __restrict__ cu,
                int* __restrict__ pos, __nv_bfloat16* __restrict__ vis_packed, int* __restrict__ vis_row_map,
-               int* __restrict__ vis_cu, int T_cap, int* err) {
+               int* __restrict__ vis_cu, int* __restrict__ vis_src, int T_cap, int* err) {
   __shared__ int s_cu[SP_MAX_BATCH + 1];
   __shared__ int s_vcu[SP_MAX_BATCH + 1];
   __shared__ int s_cnt[SP_MAX_BATCH];
@@ -75,12 +79,12 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
   // (12 loads per lane, 6 KB per warp in flight).
   constexpr int PPW = 3, PIECE16 = 128;
   const int V = s_vcu[B], Lt = bd.txt_off[B];
-  const int ppv = (nv16 + PIECE16 - 1) / PIECE16, ppt = (nt16 + PIECE16 - 1) / PIECE16;
+  const int ppv = vis_src ? 1 : (nv16 + PIECE16 - 1) / PIECE16, ppt = (nt16 + PIECE16 - 1) / PIECE16;
   const int NPv = V * ppv, NP = NPv + Lt * ppt;
   for (int p0 = gw * PPW; p0 < NP; p0 += nw * PPW) {
     const uint4* src[PPW];
     uint4* dst[PPW];
-    int nc[PPW], jv[PPW], vb[PPW], c0v[PPW];
+    int nc[PPW], jv[PPW], vb[PPW], c0v[PPW], vrv[PPW];
 #pragma unroll
     for (int u = 0; u < PPW; ++u) {
       const int pc = p0 + u;
@@ -88,6 +92,7 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
       jv[u] = -1;
       vb[u] = -1;
       c0v[u] = 0;
+      vrv[u] = -1;
       src[u] = nullptr;
       dst[u] = nullptr;
       if (pc >= NP) continue;
@@ -103,14 +108,15 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
         if (r >= T) continue;
         jv[u] = __ldg(idx + (size_t)lo * k_cap + local);  // resolved below, with every index load out
         vb[u] = lo;
+        vrv[u] = vr;
         const int c0 = sub * PIECE16;
         c0v[u] = c0;
-        nc[u] = min(PIECE16, nv16 - c0);
+        nc[u] = vis_src ? 0 : min(PIECE16, nv16 - c0);
         dst[u] = (vis_packed ? reinterpret_cast<uint4*>(vis_packed + (size_t)vr * W_vis)
                              : reinterpret_cast<uint4*>(packed + (size_t)r * W_txt)) + c0;
         if (sub == 0 && lane == 0) {
           pos[r] = local;
-          if (vis_packed) vis_row_map[vr] = r;
+          if (vis_packed || vis_src) vis_row_map[vr] = r;
         }
       } else {  // a piece of text row tr
         const int tp = pc - NPv;
@@ -135,11 +141,15 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
       if (vb[u] < 0) continue;
       const int n_img = bd.vis_off[vb[u] + 1] - bd.vis_off[vb[u]];
       if (jv[u] < 0 || jv[u] >= n_img) {
-        if (lane == 0) set_error(err, SP_DEVERR_INDEX);
+        if (lane == 0) {
+          set_error(err, SP_DEVERR_INDEX);
+          if (vis_src) vis_src[vrv[u]] = -1;  // (a gather of row -1 reads zeros)
+        }
         nc[u] = 0;
         continue;
       }
       src[u] = reinterpret_cast<const uint4*>(X + (size_t)(bd.vis_off[vb[u]] + jv[u]) * W_vis) + c0v[u];
+      if (vis_src && lane == 0) vis_src[vrv[u]] = bd.vis_off[vb[u]] + jv[u];
     }
     uint4 x[PPW][PIECE16 / 32];
 #pragma unroll
@@ -159,7 +169,7 @@ compact_kernel(const BatchDesc bd, const __nv_bfloat16* __restrict__ X, int W_vi
 
 cudaError_t compact_launch(const BatchDesc& bd, const void* X, int W_vis, const void* text, int W_txt,
                            const int* idx, int k_cap, const int* count, void* packed, int* cu,
-                           int* pos, void* vis_packed, int* vis_row_map, int* vis_cu, int T_cap,
+                           int* pos, void* vis_packed, int* vis_row_map, int* vis_cu, int* vis_src, int T_cap,
                            int* err, cudaStream_t st) {
   // pieces of at most 2 KB (one per visual row of 1,024 bf16, more for wider
   // rows), three per warp and pass
@@ -171,7 +181,7 @@ cudaError_t compact_launch(const BatchDesc& bd, const void* X, int W_vis, const 
                                       reinterpret_cast<const __nv_bfloat16*>(text), W_txt, idx, k_cap,
                                       count, reinterpret_cast<__nv_bfloat16*>(packed), cu, pos,
                                       reinterpret_cast<__nv_bfloat16*>(vis_packed), vis_row_map, vis_cu,
-                                      T_cap, err);
+                                      vis_src, T_cap, err);
   prof_end_launch(st, SP_K_COMPACT, 0.0, 0.0);
   return cudaGetLastError();
 }

@@ -67,6 +67,7 @@ struct KArgs {
   int swiglu_b;    // load B as SwiGLU gate | up halves whatever the epilogue
   float* sk_part;  // pair kernel: stream-K partial tiles [pairs][256][BN] (NULL: whole tiles only)
   int* sk_flags;   // pair kernel: [pairs][8] ready flags, zero between launches
+  const int* a_rows;  // A row r is row a_rows[r] of A's map (a row-gather map); NULL: r
 };
 
 // Column of A's tensor map holding the GEMM's k-coordinate k.
@@ -519,7 +520,60 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int KB = args.K / BK;
   const bool swb = (EPI == EPI_SWIGLU_BF16) || args.swiglu_b;
 
-  if (warp == 0) {
+  if (warp == 0 && args.a_rows) {
+    // ------------------------------------------------------------ producer, A rows gathered
+    // Each lane copies four of the tile's 128 A rows per K block with one
+    // tile::gather4 load (its map's box is 64 columns by one row); lane 0 arms
+    // the stage and loads B.  Rows past M read row 0 (their results are not
+    // stored); a row index outside A's map reads zeros.
+    int s = 0;
+    uint32_t ph = 0;
+    int issued = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      const int tile = t / ks, sp = t - tile * ks;
+      const int mb = tile % num_m, nb = tile / num_m;
+      const int m0 = mb * BM;
+      int b0, b1;
+      if (swb) {
+        b0 = nb * (BN / 2);
+        b1 = args.e.up_off + nb * (BN / 2);
+      } else {
+        b0 = nb * BN;
+        b1 = nb * BN + BN / 2;
+      }
+      int r[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int row = m0 + 4 * lane + q;
+        r[q] = row < M ? __ldg(args.a_rows + row) : 0;
+      }
+      const int kb0 = sp * KB / ks, kb1 = (sp + 1) * KB / ks;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!mbar_wait_warp(&empty[s], ph ^ 1u, err)) { ok = false; break; }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&full[s], C::A_BYTES + C::B_BYTES);
+          tma_load_2d(sB + s * C::B_BYTES, &tmB, &full[s], kb * BK, b0);
+          tma_load_2d(sB + s * C::B_BYTES + C::B_BYTES / 2, &tmB, &full[s], kb * BK, b1);
+        }
+        __syncwarp();
+        tma_gather4_2d(sA + s * C::A_BYTES + lane * (4 * BK * 2), &tmA, &full[s], a_col(args, kb * BK), r[0], r[1],
+                       r[2], r[3]);
+        ++issued;
+        if (++s == C::STAGES) { s = 0; ph ^= 1u; }
+      }
+    }
+    if (!ok && lane == 0) {
+      // the copies already in flight land before the CTA can exit
+      int n = min(issued, C::STAGES);
+      int ss = s;
+      uint32_t pp = ph;
+      for (int i = 0; i < n; ++i) {
+        if (--ss < 0) { ss = C::STAGES - 1; pp ^= 1u; }
+        mbar_wait(&full[ss], pp, err);
+      }
+    }
+  } else if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int s = 0;
@@ -818,7 +872,45 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   const Sched sc = make_sched(total, num_m, KB, npairs, pair, args.sk_part != nullptr && args.sk_flags != nullptr);
 
-  if (warp == 0) {
+  if (warp == 0 && args.a_rows) {
+    // ------------------------------------------------------------ producer (both CTAs), A rows gathered
+    // As the single-CTA kernel's: each lane copies four of this CTA's 128 A
+    // rows per K block (tile::gather4, the pair form signalling the even CTA's
+    // barrier); lane 0 waits, arms (even CTA) and loads this CTA's B half.
+    int s = 0;
+    uint32_t ph = 0;
+    Cursor cur;
+    Frag f;
+    while (sched_next(sc, cur, f)) {
+      const int mb = f.t % num_m, nb = f.t / num_m;
+      const int a_row = mb * 2 * BM + (int)rank * BM;
+      int b_row;
+      if (EPI == EPI_SWIGLU_BF16)
+        b_row = (rank == 0 ? 0 : args.e.up_off) + nb * (BN / 2);
+      else
+        b_row = nb * BN + (int)rank * (BN / 2);
+      int r[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int row = a_row + 4 * lane + q;
+        r[q] = row < M ? __ldg(args.a_rows + row) : 0;
+      }
+      bool ok = true;
+      for (int kb = f.k0; kb < f.k1; ++kb) {
+        if (!mbar_wait_warp(&empty[s], ph ^ 1u, err)) { ok = false; break; }
+        const uint32_t bar = mapa_shared(smem_u32(&full[s]), 0);
+        if (lane == 0) {
+          if (leader) mbar_arrive_expect_tx(&full[s], 2 * (C::A_BYTES + C::B_BYTES));
+          tma_load_2d_pair(sB + s * C::B_BYTES, &tmB, bar, kb * BK, b_row);
+        }
+        __syncwarp();
+        tma_gather4_2d_pair(sA + s * C::A_BYTES + lane * (4 * BK * 2), &tmA, bar, a_col(args, kb * BK), r[0], r[1],
+                            r[2], r[3]);
+        if (++s == C::STAGES) { s = 0; ph ^= 1u; }
+      }
+      if (!ok) break;
+    }
+  } else if (warp == 0) {
     // ------------------------------------------------------------ producer (both CTAs)
     if (lane == 0) {
       int s = 0;
@@ -1324,6 +1416,7 @@ cudaError_t gemm_swap_partials(const CUtensorMap& A16, int M_cap, const GemmB& B
   a.e.kind = EPI_F32;
   a.err = err;
   a.a_seg = 0;
+  a.a_rows = nullptr;
   a.a_map = 0;
   a.ksplit = ks;
   a.m_pad = N_acc;
@@ -1341,9 +1434,10 @@ cudaError_t gemm_swap_partials(const CUtensorMap& A16, int M_cap, const GemmB& B
 
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B, int N_acc,
                       const GemmEpi& e, int* err, cudaStream_t st, const GemmScratch* sk,
-                      const GemmASplit* as, const CUtensorMap* A16) {
+                      const GemmASplit* as, const CUtensorMap* A16, const int* a_rows) {
   if (M_cap <= 0) return cudaSuccess;
   const int sms = device_sm_count();
+  if (a_rows) A16 = nullptr;  // gathered A rows: not the weight-streaming form (M <= 32 rows)
   // Weight streaming for M <= 32 rows (generation steps): the weights are the
   // MMA's 128-row operand and the activations its 32 columns (C^T = B A^T),
   // each 128-row weight tile's K split into ranges over the SMs; the fp32
@@ -1384,6 +1478,7 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
   a.sk_part = nullptr;
   a.sk_flags = nullptr;
   a.a_seg = 0;
+  a.a_rows = nullptr;
   a.a_map = 0;
   a.ksplit = 1;
   a.m_pad = 0;
@@ -1393,6 +1488,7 @@ cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const G
     a.a_seg = as->seg;
     a.a_map = as->map;
   }
+  a.a_rows = a_rows;
   // output map for the TMA epilogue (box 32 rows x 128 bytes); the row-scatter
   // epilogue stores directly and needs none
   CUtensorMap tmO;

@@ -138,10 +138,15 @@ cudaError_t gemm_swap_partials(const CUtensorMap& A16, int M_cap, const GemmB& B
 // A16 (optional): A's tensor map with box rows 16.  With it, M_cap <= 32 and
 // split-K scratch, the GEMM streams the weights as the MMA's 128-row operand
 // (generation steps); the result and epilogue are the same.
+// a_rows (device, may be NULL): A row r is row a_rows[r] of the tensor A's
+// map describes, which then has a box of 64 columns by one row (the row-gather
+// form: encode_tmap_bf16 with box_rows 1): the gather of Algorithm 1 step 5
+// folded into the operand load (single-CTA and CTA-pair kernels; not the
+// weight-streaming form).
 cudaError_t gemm_bf16(const CUtensorMap& A, int M_cap, const int* M_dev, const GemmB& B,
                       int N_acc, const GemmEpi& e, int* err, cudaStream_t st,
                       const GemmScratch* sk = nullptr, const GemmASplit* as = nullptr,
-                      const CUtensorMap* A16 = nullptr);
+                      const CUtensorMap* A16 = nullptr, const int* a_rows = nullptr);
 
 // ------------------------------------------------------------- candidate precompute
 // out [rows, 3K] bf16 = the three bf16 parts of x [rows, K] (fp32, row stride ldx).
@@ -261,7 +266,7 @@ sp_status select_with_workspace(const sp_selector* s, const sp_select_in* in, co
 // ------------------------------------------------------------- compaction
 cudaError_t compact_launch(const BatchDesc& bd, const void* X, int W_vis, const void* text, int W_txt,
                            const int* idx, int k_cap, const int* count, void* packed, int* cu,
-                           int* pos, void* vis_packed, int* vis_row_map, int* vis_cu, int T_cap,
+                           int* pos, void* vis_packed, int* vis_row_map, int* vis_cu, int* vis_src, int T_cap,
                            int* err, cudaStream_t st);
 
 }  // namespace sp

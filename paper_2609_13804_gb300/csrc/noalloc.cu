@@ -14,7 +14,11 @@
 //   * a batch whose sp_select_workspace() exceeds it is rejected with
 //     SP_ERR_WORKSPACE before anything is launched;
 //   * every call shares the one array: calls whose GPU work overlaps (two
-//     streams, two host threads) race on it; serialise them.
+//     streams, two host threads) race on it; serialise them;
+//   * the array's device address is looked up once per device and kept for
+//     the life of the process: after cudaDeviceReset (or any other teardown of
+//     the device's primary context) it is stale, so do not use this entry
+//     point across a device reset.
 #include <cuda_runtime.h>
 
 #include <mutex>

@@ -86,7 +86,17 @@ def test_argument_checks_fail_before_any_launch(L):
     assert L.sp_compact(C.byref(ci), C.byref(co), None) == 2  # W_vis not a multiple of 8
     ci = b.sp_compact_in(1, C.cast(nv, b.IP), C.cast(nt, b.IP), 8, 8, 32, 8, 48, 4, 64)
     assert L.sp_compact(C.byref(ci), C.byref(co), None) == 3  # X misaligned
+    ci = b.sp_compact_in(1, C.cast(nv, b.IP), C.cast(nt, b.IP), 16, 8, 32, 8, 48, 4, 64)
+    co = b.sp_compact_out(80, 96, 112, 128, 144, 160, None, 176)
+    assert L.sp_compact(C.byref(ci), C.byref(co), None) == 1  # vis_src and vis_packed together
+    co = b.sp_compact_out(80, 96, 112, None, None, None, None, 176)
+    assert L.sp_compact(C.byref(ci), C.byref(co), None) == 1  # index mode without vis_row_map / vis_cu
     assert L.sp_profile_end(None, None, None, None) == 1       # not started
+
+
+def test_compact_and_project_io_layout():
+    assert C.sizeof(b.sp_compact_out) == 8 * 8
+    assert C.sizeof(b.sp_project_io) == 4 * 2 + 8 * 5 + 8 + 4 + 4 + 8
 
 
 def test_create_without_a_gpu_reports_instead_of_crashing(L):

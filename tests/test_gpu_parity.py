@@ -257,6 +257,60 @@ def test_projector_scatter(B, kind, rows):
     model.close()
 
 
+@pytest.mark.parametrize("kind,n_vis,keep,k_cap", [
+    ("mlp2", [576, 300, 10, 576], [300, 250, 0, 512], 576),   # 1,062 rows: whole tiles
+    ("linear", [576, 300, 10, 576], [60, 7, 10, 33], 576),
+    ("mlp2", [60, 7, 10, 40], [32, 7, 1, 30], 32)])            # rows_cap 81: split-K GEMM
+def test_projector_gather_equals_compact_then_project(B, kind, n_vis, keep, k_cap):
+    """Alg. 1 step 5 folded into the projector's operand load: the index-mode
+    compaction (no visual row copied, the source row of each kept row written)
+    followed by the projector gathering those rows of X gives the packed buffer
+    of the copying compaction + projector bit for bit; the source rows are
+    exactly the image offsets plus the kept indices."""
+    n_txt = [48, 0, 5, 13]
+    D = d = 1024
+    w = S.tiny_workload(52, [300], [1], D=D, d=d, n_heads=8, n_kv_heads=8, head_dim=128, ffn=1024, n_layers=1,
+                        proj_kind=kind)
+    w.model.proj_hidden = 2048
+    head = S.make_model_head(w)
+    model = B.Model(w.model, [S.make_layer_weights(w, 0)], head, DEV, max_pos=1024)
+    X = B.dev_bf16(S.bf16_round(S.normal(52, "X", (sum(n_vis), D))), DEV)
+    text = B.dev_bf16(S.bf16_round(S.normal(52, "T", (sum(n_txt), d), 0.02)), DEV)
+    rng = np.random.default_rng(52)
+    idx = np.full((4, k_cap), -1, np.int32)
+    idx_list = []
+    for b, (n, k) in enumerate(zip(n_vis, keep)):
+        l = np.sort(rng.choice(n, k, replace=False)).astype(np.int32)
+        idx[b, :k] = l
+        idx_list.append(l)
+    idx_d = torch.from_numpy(idx).to(DEV)
+    cnt_d = torch.tensor(keep, dtype=torch.int32, device=DEV)
+    oc = B.sp_compact(n_vis, n_txt, X=X, text=text, idx=idx_d, count=cnt_d, k_cap=k_cap, projector_mode=True)
+    e1 = B.sp_project(model, vis_packed=oc["vis_packed"], vis_row_map=oc["vis_row_map"], vis_cu=oc["vis_cu"],
+                      packed=oc["packed"], rows_cap=oc["rows_cap"], B=4)
+    oi = B.sp_compact(n_vis, n_txt, X=X, text=text, idx=idx_d, count=cnt_d, k_cap=k_cap, index_mode=True)
+    e2 = B.sp_project(model, X=X, vis_src=oi["vis_src"], vis_row_map=oi["vis_row_map"], vis_cu=oi["vis_cu"],
+                      packed=oi["packed"], rows_cap=oi["rows_cap"], B=4)
+    torch.cuda.synchronize()
+    assert int(oc["err"].item()) == 0 and int(oi["err"].item()) == 0 and int(e1.item()) == 0 and int(e2.item()) == 0
+    R = sum(keep)
+    offs = np.concatenate([[0], np.cumsum(n_vis)])
+    want_src = np.concatenate([offs[b] + idx_list[b] for b in range(4)])
+    np.testing.assert_array_equal(np_(oi["vis_src"])[:R], want_src)
+    np.testing.assert_array_equal(np_(oi["vis_row_map"])[:R], np_(oc["vis_row_map"])[:R])
+    np.testing.assert_array_equal(np_(oi["cu_seqlens"]), np_(oc["cu_seqlens"]))
+    T = int(np_(oc["cu_seqlens"])[-1])
+    np.testing.assert_array_equal(np_(oi["pos"])[:T], np_(oc["pos"])[:T])
+    a = oi["packed"][:T].view(torch.int16).cpu().numpy()
+    b_ = oc["packed"][:T].view(torch.int16).cpu().numpy()
+    np.testing.assert_array_equal(a, b_)
+    # and the projected rows are the projector of X's kept rows (the oracle, tolerance as the projector test)
+    ref = O.projector(np_(X)[want_src], head)
+    got = np_(oi["packed"])[np_(oi["vis_row_map"])[:R]]
+    assert np.abs(got - ref).max() <= 1e-2 * np.abs(ref).max()
+    model.close()
+
+
 # ------------------------------------------------------------------ prefill
 
 def _prefill_case(B, w, lens, n_layers, seed_name="packed", affine=True):

@@ -53,6 +53,28 @@ def test_noalloc_matches_sp_select_on_two_calls_in_a_row(B):
     selector.close()
 
 
+def test_noalloc_with_the_encoder_matches_sp_select_on_two_calls_in_a_row(B):
+    """The encoder path (text projection, encoder blocks, their GEMM scratch
+    and encoder buffers all in the static scratch): two calls with different
+    inputs, each bit-identical to sp_select's."""
+    w = S.tiny_workload(81, [40, 130, 7], [5, 0, 3], D=128, D_text=128, h=128, enc_head_dim=64, k_max=12)
+    s = w.selector
+    sel = S.make_selector_weights(w, ln_affine=True)
+    selector = B.Selector(s, sel, DEV)
+    for name, bias in (("a", [-1e30, 0.0, -0.1]), ("b", [0.02, -1e30, -1e30])):
+        X = B.dev_bf16(S.bf16_round(S.normal(81, "X" + name, (sum(w.n_vis), s.D))), DEV)
+        E = B.dev_bf16(S.bf16_round(S.normal(81, "E" + name, (sum(w.n_txt), s.D_text), 0.02)), DEV)
+        bd = B.dev_f32(np.array(bias, np.float32), DEV)
+        ref = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bd, k_max=w.k_max, memory=True)
+        got = B.sp_select(selector, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bd, k_max=w.k_max, no_alloc=True,
+                          memory=True)
+        torch.cuda.synchronize()
+        assert int(got["err"].item()) == 0 and int(ref["err"].item()) == 0
+        _same(got, ref)
+        np.testing.assert_array_equal(got["memory"].cpu().numpy(), ref["memory"].cpu().numpy())
+    selector.close()
+
+
 def test_noalloc_rejects_a_batch_beyond_its_scratch(B):
     w = S.llava15_7b_b16()
     s = S.SelectorShape(D=w.selector.D, D_text=w.selector.D_text, h=w.selector.h, n_enc_layers=0)
