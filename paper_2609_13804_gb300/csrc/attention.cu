@@ -19,15 +19,16 @@ namespace {
 //
 //   warps 0 / 3  TMA of head 0 / 1: the Q tile once per item, then per 64-key
 //                block the K and V blocks into two-stage rings
-//   warps 1 / 2  MMA issue of head 0 / 1 (warp 1 also allocates the 512 TMEM
-//                columns), software-pipelined by one key block: the scores of
-//                block j + 1 (S = Q K^T, M 128, N 64, both K-major from shared
-//                memory) go to the tensor pipe before O += P V of block j (P
-//                read from Tensor Memory where the softmax wrote it over its S,
-//                V an MN-major operand straight from its TMA block).  Two S / P
-//                buffers per head let the softmax of block j overlap the scores
-//                of block j + 1; S of block j + 2 reuses block j's buffer only
-//                once O += P V of block j has completed (its commit).
+//   warps 1 / 12 issue head 0 / 1's scores: S = Q K^T per 64-key block (M
+//                128, N 64, both K-major from shared memory) into one of the
+//                head's two S / P buffers (warp 1 also allocates the 512 TMEM
+//                columns); S of block j + 2 reuses block j's buffer only once
+//                O += P V of block j has completed (its commit)
+//   warps 2 / 13 issue head 0 / 1's O += P V (P read from Tensor Memory where
+//                the softmax wrote it over its S, V an MN-major operand straight
+//                from its TMA block).  Two issuing threads per head let one's
+//                barrier waits overlap the other's issue; two S / P buffers let
+//                the softmax of block j overlap the scores of block j + 1.
 //   warps 4-7   softmax of head 0, warps 8-11 of head 1: one thread per query
 //               row (= TMEM lane): S row from TMEM, mask (causal diagonal
 //               blocks, sequence tail), running max / sum in the exp2 domain, P
@@ -41,7 +42,7 @@ namespace {
 // keeps the rows past the packed length zero, or the tensor map ends there).
 namespace fa {
 
-constexpr int BQ = 128, BKV = 64, NTHR = 384;
+constexpr int BQ = 128, BKV = 64, NTHR = 448;
 constexpr float kRescaleLog2 = 8.f;  // rescale O once the max moved by more than this (log2 units)
 
 template <int DH>
@@ -61,15 +62,16 @@ struct Cfg {
   static constexpr uint32_t T_O = 256;
 };
 
-// Barriers.  Per head t: Q_FULL + t, Q_EMPTY + t, O_FULL + t, O_EMPTY + t,
-// MMA_DONE + t; per head t and stage / buffer b (= block index & 1): X + 2 t + b.
+// Barriers.  Per head t: Q_FULL + t, Q_EMPTY + t, O_FULL + t, O_EMPTY + t;
+// per head t and stage / buffer b (= block index & 1): X + 2 t + b; per head t
+// and issuer (0: scores, 1: P V): MMA_DONE + 2 t + issuer.
 // A slot's K is free once the scores that read it are complete (S_FULL), its
 // V once O += P V is (PV_DONE): no "empty" barriers.  The V block's bytes
 // complete on the P-ready barrier of its block (four softmax warps plus the
 // TMA thread's expect-tx arrive), so O += P V waits once for both.
 enum Bar {
   Q_FULL = 0, Q_EMPTY = 2, K_FULL = 4, S_FULL = 8, P_FULL = 12, PV_DONE = 16, O_FULL = 20, O_EMPTY = 22,
-  MMA_DONE = 24, N_BARS = 26
+  MMA_DONE = 24, N_BARS = 28
 };
 
 SP_DEVINL float ex2(float x) {
@@ -185,10 +187,14 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         mbar_wait(&bar[P_FULL + 2 * t + (gg & 1)], (gg >> 1) & 1, err);  // (V, and the block's P)
       }
     }
-  } else if (warp == 1 || warp == 2) {
-    // ------------------------------------------------------------ MMA issuer of head t
+  } else if (warp == 1 || warp == 2 || warp >= 12) {
+    // ------------------------------------------------------------ MMA issuers of head t
+    // Two threads per head: one issues the scores, the other O += P V, so
+    // that one's waits overlap the other's issue (tcgen05.commit tracks the
+    // issuing thread's own MMAs, and the two never write the same columns).
     if (lane == 0) {
-      const int t = warp - 1;
+      const int t = warp >= 12 ? 1 : 0;
+      const bool pv_issuer = warp == 2 || warp == 13;
       constexpr uint32_t IDESC_S = umma_idesc_bf16_f32(BQ, BKV);
       constexpr uint32_t IDESC_O = umma_idesc_bf16_f32(BQ, DH) | (1u << 16);  // B (V) MN-major
       // shared-memory descriptors of the stage bases; a K step adds its byte
@@ -201,53 +207,56 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       const uint32_t tS = tmem + t * 128, tO = tmem + C::T_O + t * DH;
       uint32_t g = 0, nitem = 0;
       bool ok = true;
-      // scores of global block gg (= block j of the current item)
-      auto issue_s = [&](uint32_t gg, bool last) -> bool {
-        const uint32_t b = gg & 1, ph = (gg >> 1) & 1;
-        // buffer b held P of block gg - 2: its O += P V must be complete
-        if (!mbar_wait(&bar[K_FULL + 2 * t + b], ph, err) ||
-            (gg >= 2 && !mbar_wait(&bar[PV_DONE + 2 * t + b], ph ^ 1u, err)))
-          return false;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk)
-          umma_bf16(tS + b * BKV, dQ + (((kk >> 2) * C::BOX_Q + (kk & 3) * 32) >> 4),
-                    (b ? dK1 : dK0) + (((kk >> 2) * C::BOX_KV + (kk & 3) * 32) >> 4), IDESC_S, kk ? 1u : 0u);
-        umma_commit(&bar[S_FULL + 2 * t + b]);
-        if (last) umma_commit(&bar[Q_EMPTY + t]);
-        return true;
-      };
-      // O += P V of global block gg (block j of the current item)
-      auto issue_pv = [&](uint32_t gg, int j, bool last) -> bool {
-        const uint32_t b = gg & 1, ph = (gg >> 1) & 1;
-        // (P_FULL completes once the softmax wrote P and this block's V landed)
-        if (!mbar_wait(&bar[P_FULL + 2 * t + b], ph, err) ||
-            (j == 0 && !mbar_wait(&bar[O_EMPTY + t], (nitem & 1) ^ 1u, err)))
-          return false;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < BKV / 16; ++kk)
-          umma_bf16_ta(tO, tS + b * BKV + kk * 8, (b ? dV1 : dV0) + ((kk * 2048) >> 4), IDESC_O, (j | kk) ? 1u : 0u);
-        umma_commit(&bar[PV_DONE + 2 * t + b]);
-        if (last) umma_commit(&bar[O_FULL + t]);
-        return true;
-      };
       for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
         Item I;
         if (!item_at(it, cu, B, HP, n_tiles, Hq, Hkv, causal, I)) continue;
-        ok = mbar_wait(&bar[Q_FULL + t], nitem & 1, err) && issue_s(g, I.nkv == 1);
-        for (int j = 0; ok && j < I.nkv; ++j) {
-          if (j + 1 < I.nkv) ok = issue_s(g + j + 1, j + 2 == I.nkv);
-          ok = ok && issue_pv(g + j, j, j + 1 == I.nkv);
+        if (!pv_issuer) {
+          // scores of every block: S(j) = Q K(j)^T into buffer j & 1
+          ok = mbar_wait(&bar[Q_FULL + t], nitem & 1, err);
+          for (int j = 0; ok && j < I.nkv; ++j) {
+            const uint32_t gg = g + j, b = gg & 1, ph = (gg >> 1) & 1;
+            // buffer b held P of block gg - 2: its O += P V must be complete
+            if (!mbar_wait(&bar[K_FULL + 2 * t + b], ph, err) ||
+                (gg >= 2 && !mbar_wait(&bar[PV_DONE + 2 * t + b], ph ^ 1u, err))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < DH / 16; ++kk)
+              umma_bf16(tS + b * BKV, dQ + (((kk >> 2) * C::BOX_Q + (kk & 3) * 32) >> 4),
+                        (b ? dK1 : dK0) + (((kk >> 2) * C::BOX_KV + (kk & 3) * 32) >> 4), IDESC_S, kk ? 1u : 0u);
+            umma_commit(&bar[S_FULL + 2 * t + b]);
+            if (j + 1 == I.nkv) umma_commit(&bar[Q_EMPTY + t]);
+          }
+        } else {
+          // O += P(j) V(j); P_FULL completes once the softmax wrote P and the
+          // block's V landed
+          for (int j = 0; ok && j < I.nkv; ++j) {
+            const uint32_t gg = g + j, b = gg & 1, ph = (gg >> 1) & 1;
+            if (!mbar_wait(&bar[P_FULL + 2 * t + b], ph, err) ||
+                (j == 0 && !mbar_wait(&bar[O_EMPTY + t], (nitem & 1) ^ 1u, err))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < BKV / 16; ++kk)
+              umma_bf16_ta(tO, tS + b * BKV + kk * 8, (b ? dV1 : dV0) + ((kk * 2048) >> 4), IDESC_O,
+                           (j | kk) ? 1u : 0u);
+            umma_commit(&bar[PV_DONE + 2 * t + b]);
+            if (j + 1 == I.nkv) umma_commit(&bar[O_FULL + t]);
+          }
         }
         g += I.nkv;
         ++nitem;
       }
-      umma_commit(&bar[MMA_DONE + t]);  // TMEM stays allocated until every issued MMA is done
-      mbar_wait(&bar[MMA_DONE + t], 0, err);
+      // TMEM stays allocated until every MMA this thread issued is done
+      umma_commit(&bar[MMA_DONE + 2 * t + (pv_issuer ? 1 : 0)]);
+      mbar_wait(&bar[MMA_DONE + 2 * t + (pv_issuer ? 1 : 0)], 0, err);
     }
     __syncwarp();
-  } else if (warp >= 4) {
+  } else if (warp >= 4 && warp < 12) {
     // ------------------------------------------------------------ softmax (row = TMEM lane)
     const int t = (warp - 4) >> 2;
     const int quad = warp & 3;
