@@ -68,7 +68,11 @@ struct Cfg {
 // A slot's K is free once the scores that read it are complete (S_FULL), its
 // V once O += P V is (PV_DONE): no "empty" barriers.  The V block's bytes
 // complete on the P-ready barrier of its block (four softmax warps plus the
-// TMA thread's expect-tx arrive), so O += P V waits once for both.
+// TMA thread's expect-tx arrive), so O += P V waits once for both.  Likewise
+// the K barrier of block j counts two arrivals, the TMA's (with K's bytes) and
+// the commit of O += P V of block j - 2 (the last reader of the S / P buffer
+// block j's scores will overwrite; the TMA arrives twice for the first two
+// blocks), so the scores wait once for both.
 enum Bar {
   Q_FULL = 0, Q_EMPTY = 2, K_FULL = 4, S_FULL = 8, P_FULL = 12, PV_DONE = 16, O_FULL = 20, O_EMPTY = 22,
   MMA_DONE = 24, N_BARS = 28
@@ -78,6 +82,12 @@ SP_DEVINL float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+SP_DEVINL float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
 }
 
 struct Item {
@@ -124,7 +134,10 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < N_BARS; ++i)
-      mbar_init(&bar[i], (i >= P_FULL && i < P_FULL + 4) ? 5 : (i == O_EMPTY || i == O_EMPTY + 1) ? 4 : 1);
+      mbar_init(&bar[i], (i >= P_FULL && i < P_FULL + 4) ? 5
+                         : (i == O_EMPTY || i == O_EMPTY + 1) ? 4
+                         : (i >= K_FULL && i < K_FULL + 4)    ? 2
+                                                              : 1);
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -168,6 +181,7 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           uint64_t* vfull = &bar[P_FULL + 2 * t + st];
           if (g >= 2 && !mbar_wait(&bar[S_FULL + 2 * t + st], pe, err)) { ok = false; break; }
           mbar_arrive_expect_tx(kfull, C::KV_BYTES);
+          if (g < 2) mbar_arrive(kfull);  // (no O += P V of block g - 2 arrives)
 #pragma unroll
           for (int bx = 0; bx < DH / 64; ++bx)
             tma_load_2d(sK + bx * C::BOX_KV, &tmKV, kfull, kcol + bx * 64, I.s0 + j * BKV);
@@ -215,9 +229,9 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           ok = mbar_wait(&bar[Q_FULL + t], nitem & 1, err);
           for (int j = 0; ok && j < I.nkv; ++j) {
             const uint32_t gg = g + j, b = gg & 1, ph = (gg >> 1) & 1;
-            // buffer b held P of block gg - 2: its O += P V must be complete
-            if (!mbar_wait(&bar[K_FULL + 2 * t + b], ph, err) ||
-                (gg >= 2 && !mbar_wait(&bar[PV_DONE + 2 * t + b], ph ^ 1u, err))) {
+            // K_FULL also counts the completion of O += P V of block gg - 2,
+            // the last reader of buffer b
+            if (!mbar_wait(&bar[K_FULL + 2 * t + b], ph, err)) {
               ok = false;
               break;
             }
@@ -245,6 +259,7 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
               umma_bf16_ta(tO, tS + b * BKV + kk * 8, (b ? dV1 : dV0) + ((kk * 2048) >> 4), IDESC_O,
                            (j | kk) ? 1u : 0u);
             umma_commit(&bar[PV_DONE + 2 * t + b]);
+            umma_commit(&bar[K_FULL + 2 * t + b]);  // (counts toward block gg + 2's K barrier)
             if (j + 1 == I.nkv) umma_commit(&bar[O_FULL + t]);
           }
         }
@@ -286,12 +301,14 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         }
         float mx[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) mx[e] = v[e];
+        for (int e = 0; e < 8; ++e) mx[e] = max3(v[e], v[e + 8], v[e + 16]);
 #pragma unroll
-        for (int c = 8; c < BKV; ++c) mx[c & 7] = fmaxf(mx[c & 7], v[c]);
-        const float mb =
-            fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) *
-            scale_log2;
+        for (int e = 0; e < 8; ++e) mx[e] = max3(mx[e], v[e + 24], v[e + 32]);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx[e] = max3(mx[e], v[e + 40], v[e + 48]);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], v[e + 56]);
+        const float mb = max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * scale_log2;
         // stale-max rule: move m (and rescale O and l) only when the block max exceeds it by > 2^8
         float corr = 1.f;
         bool moved = false;
