@@ -534,7 +534,8 @@ sp_status run_encoder(const sp_selector* s, const sp_select_in* in, const SelPla
     e1.out = QKV;
     e1.ldo = 3 * D;
     SP_CUDA(gemm_bf16(tA, p.T_enc, nullptr, s->enc_qkv[l], 3 * D, e1, err, st, &gs), "enc qkv");
-    SP_CUDA(attention_varlen(QKV, O, enc_cu, in->B, p.max_enc, p.T_enc, nh, nh, c.enc_head_dim, false, err, st),
+    SP_CUDA(attention_varlen(QKV, O, enc_cu, in->B, p.max_enc, p.T_enc, nh, nh, c.enc_head_dim, false,
+                             gs.attn_sched, err, st),
             "enc attention");
     GemmEpi e2;
     e2.kind = EPI_F32_ACC;
@@ -1054,7 +1055,7 @@ static sp_status prefill_impl(const sp_model* m, const sp_prefill_io* io, void* 
                        io->kv_S_cap, io->err, st), "kv cache");
     }
     SP_CUDA(attention_varlen(p.qkv, p.ob, io->cu_seqlens, io->B, io->max_seqlen_cap, T_cap, c.n_heads, c.n_kv_heads,
-                             c.head_dim, true, io->err, st), "attention");
+                             c.head_dim, true, gs.attn_sched, io->err, st), "attention");
     GemmEpi er;
     er.kind = EPI_F32_ACC;
     er.out = h32;

@@ -1366,7 +1366,7 @@ int gemm_pair_policy(int M_cap, int N_acc, int kind) {
 
 size_t gemm_scratch_bytes() {
   const size_t slots = (size_t)(device_sm_count() / 2);
-  return slots * kSlotFloats * sizeof(float) + slots * 8 * sizeof(int);
+  return slots * kSlotFloats * sizeof(float) + slots * 8 * sizeof(int) + 16 * sizeof(int);
 }
 
 GemmScratch gemm_scratch_at(void* p) {
@@ -1375,6 +1375,7 @@ GemmScratch gemm_scratch_at(void* p) {
   g.slots = device_sm_count() / 2;
   g.part = static_cast<float*>(p);
   g.flags = reinterpret_cast<int*>(g.part + (size_t)g.slots * kSlotFloats);
+  g.attn_sched = g.flags + (size_t)g.slots * 8;
   return g;
 }
 
@@ -1387,7 +1388,7 @@ size_t gemm_splitk_floats(int max_n_acc) {
 
 cudaError_t gemm_scratch_clear(const GemmScratch& g, cudaStream_t st) {
   if (!g.flags) return cudaSuccess;
-  return cudaMemsetAsync(g.flags, 0, (size_t)g.slots * 8 * sizeof(int), st);
+  return cudaMemsetAsync(g.flags, 0, (size_t)g.slots * 8 * sizeof(int) + 16 * sizeof(int), st);
 }
 
 bool make_gemm_b(GemmB* b, const void* w, int N, int K, std::string* msg) {

@@ -103,13 +103,15 @@ int gemm_pair_policy(int M_cap, int N_acc, int kind);
 // M_cap bounds it on the host.  N_out is the accumulator width (N of B, or the
 // tile columns for SWIGLU: 2 F).
 // Scratch of the CTA-pair GEMM's stream-K tail: per SM pair one fp32 256 x 256
-// partial tile and 8 ready flags.  The flags must be zero when a GEMM starts;
-// every launch leaves them zero, so one gemm_scratch_clear per API call does.
+// partial tile and 8 ready flags, then the attention's two scheduling counters.
+// The flags and counters must be zero when a kernel starts; every launch
+// leaves them zero, so one gemm_scratch_clear per API call does.
 // Without scratch (NULL) the GEMM runs whole tiles only.
 struct GemmScratch {
   float* part = nullptr;
   int* flags = nullptr;
   int slots = 0;
+  int* attn_sched = nullptr;  // the attention's ticket counter (two ints after the flags)
   float* splitk = nullptr;   // small-M split-K partial planes (NULL: no split)
   size_t splitk_floats = 0;
 };
@@ -195,9 +197,12 @@ cudaError_t lens_increment(int* lens, int* rope_pos, int B, int S_cap, cudaStrea
 // ------------------------------------------------------------- attention
 // Varlen attention over packed qkv [rows_cap, (Hq + 2 Hkv) dh] bf16 -> out [T, Hq dh] bf16
 // (rows of sequence b from cu_seqlens[b]; rows_cap bounds the buffer for TMA).
+// sched: two device ints, zero before the launch and left zero by it (the
+// work-item ticket counter; GemmScratch::attn_sched), or NULL for a static
+// assignment of the items to the CTAs.
 cudaError_t attention_varlen(const void* qkv, void* out, const int* cu_seqlens, int B,
                              int max_seqlen_cap, int rows_cap, int Hq, int Hkv, int dh, bool causal,
-                             int* err, cudaStream_t st);
+                             int* sched, int* err, cudaStream_t st);
 
 // ------------------------------------------------------------- selection
 // A pointer-decoder layer's runtime weights (decoders of several layers).
