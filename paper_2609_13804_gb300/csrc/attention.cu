@@ -101,15 +101,20 @@ struct Item {
   int s0, len, q0, h0, h1, kvh0, kvh1, nkv;
 };
 
-// Work item `it` of the static list: query tiles from the last (the most key
-// blocks under a causal mask) to the first; within a tile index, sequence-major,
-// then head pair.  Returns false for tiles past the sequence's end.
-SP_DEVINL bool item_at(int it, const int* __restrict__ cu, int B, int HP, int n_tiles, int Hq, int Hkv, bool causal,
-                       Item& I) {
-  const int per_tile = B * HP;
-  const int tile = n_tiles - 1 - it / per_tile;
-  const int rem = it - (it / per_tile) * per_tile;
-  const int b = rem / HP, hp = rem - (rem / HP) * HP;
+// Work item `it` of the static list.  The sequences go in chunks of S (sized
+// on the host so that a chunk's keys and values stay in L2 while its items
+// run); within a chunk, query tiles from the last (the most key blocks under a
+// causal mask) to the first, then sequence, then head pair.  Returns false for
+// tiles past the sequence's end.
+SP_DEVINL bool item_at(int it, const int* __restrict__ cu, int B, int HP, int n_tiles, int S, int Hq, int Hkv,
+                       bool causal, Item& I) {
+  const int ch = it / (n_tiles * S * HP);
+  const int b0 = ch * S, sc = min(S, B - b0);  // the chunk's first sequence and its sequence count
+  const int rem0 = it - ch * (n_tiles * S * HP);
+  const int per_tile = sc * HP;
+  const int tile = n_tiles - 1 - rem0 / per_tile;
+  const int rem = rem0 - (rem0 / per_tile) * per_tile;
+  const int b = b0 + rem / HP, hp = rem - (rem / HP) * HP;
   I.s0 = __ldg(cu + b);
   I.len = __ldg(cu + b + 1) - I.s0;
   I.q0 = tile * BQ;
@@ -128,7 +133,7 @@ template <int DH>
 __global__ void __launch_bounds__(NTHR, 1)
 attn_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
                __nv_bfloat16* __restrict__ out, const int* __restrict__ cu, int B, int Hq, int Hkv, int n_tiles,
-               int ld_out, int causal_i, float scale_log2, int* err) {
+               int seq_chunk, int ld_out, int causal_i, float scale_log2, int* err) {
   using C = Cfg<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -169,7 +174,7 @@ attn_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
       uint8_t* sQ = sm + C::OFF_Q + t * C::Q_BYTES;
       for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
         Item I;
-        if (!item_at(it, cu, B, HP, n_tiles, Hq, Hkv, causal, I)) continue;
+        if (!item_at(it, cu, B, HP, n_tiles, seq_chunk, Hq, Hkv, causal, I)) continue;
         if (!mbar_wait(&bar[Q_EMPTY + t], (nitem & 1) ^ 1u, err)) break;
         mbar_arrive_expect_tx(&bar[Q_FULL + t], C::Q_BYTES);
         const int qcol = (t ? I.h1 : I.h0) * DH;
@@ -230,7 +235,7 @@ attn_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
       bool ok = true;
       for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
         Item I;
-        if (!item_at(it, cu, B, HP, n_tiles, Hq, Hkv, causal, I)) continue;
+        if (!item_at(it, cu, B, HP, n_tiles, seq_chunk, Hq, Hkv, causal, I)) continue;
         if (!pv_issuer) {
           // scores of every block: S(j) = Q K(j)^T into buffer j & 1
           ok = mbar_wait(&bar[Q_FULL + t], nitem & 1, err);
@@ -289,7 +294,7 @@ attn_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
     bool ok = true;
     for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
       Item I;
-      if (!item_at(it, cu, B, HP, n_tiles, Hq, Hkv, causal, I)) continue;
+      if (!item_at(it, cu, B, HP, n_tiles, seq_chunk, Hq, Hkv, causal, I)) continue;
       const int qpos = I.q0 + r;  // query position in the sequence
       const int row_lim = qpos >= I.len ? 0 : (causal ? qpos + 1 : I.len);  // keys [0, row_lim) are visible
       float m = -INFINITY, l = 0.f;  // m: running max in log2 units
@@ -494,16 +499,21 @@ struct Item {
   int s0, len, q0, h, kvh, nkv;  // nkv == 0: no more items
 };
 
-// Work item `it` of the list: query tiles from the last (the most key blocks
-// under a causal mask) to the first; within a tile index, sequence-major, then
-// head.  Returns false for tiles past the sequence's end.
-SP_DEVINL bool item_at(int it, const int* __restrict__ cu, int B, int Hq, int n_tiles, int Hkv, bool causal,
+// Work item `it` of the list.  The sequences go in chunks of S (sized on the
+// host so that a chunk's keys and values stay in L2 while its items run);
+// within a chunk, query tiles from the last (the most key blocks under a causal
+// mask) to the first, then sequence, then head.  Returns false for tiles past
+// the sequence's end.
+SP_DEVINL bool item_at(int it, const int* __restrict__ cu, int B, int Hq, int n_tiles, int S, int Hkv, bool causal,
                        Item& I) {
-  const int per_tile = B * Hq;
-  const int tile = n_tiles - 1 - it / per_tile;
-  const int rem = it - (it / per_tile) * per_tile;
-  const int b = rem / Hq;
-  I.h = rem - b * Hq;
+  const int ch = it / (n_tiles * S * Hq);
+  const int b0 = ch * S, sc = min(S, B - b0);  // the chunk's first sequence and its sequence count
+  const int rem0 = it - ch * (n_tiles * S * Hq);
+  const int per_tile = sc * Hq;
+  const int tile = n_tiles - 1 - rem0 / per_tile;
+  const int rem = rem0 - (rem0 / per_tile) * per_tile;
+  const int b = b0 + rem / Hq;
+  I.h = rem - (rem / Hq) * Hq;
   I.s0 = __ldg(cu + b);
   I.len = __ldg(cu + b + 1) - I.s0;
   I.q0 = tile * BQ;
@@ -518,7 +528,7 @@ template <int DH>
 __global__ void __launch_bounds__(NTHR, 1)
 attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
                __nv_bfloat16* __restrict__ out, const int* __restrict__ cu, int B, int Hq, int Hkv, int n_tiles,
-               int ld_out, int causal_i, float scale_log2, int* sched, int* err) {
+               int seq_chunk, int ld_out, int causal_i, float scale_log2, int* sched, int* err) {
   using C = Cfg<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -583,7 +593,7 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         Item I;
         bool have = false;
         while (!have && ticket < n_items) {
-          have = item_at(ticket, cu, B, Hq, n_tiles, Hkv, causal, I);
+          have = item_at(ticket, cu, B, Hq, n_tiles, seq_chunk, Hkv, causal, I);
           ticket = nxt;
           nxt = ticket < n_items ? fetch() : n_items;
         }
@@ -889,6 +899,14 @@ attn_fa_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 }  // namespace fa
 }  // namespace
 
+// Sequences per item chunk: as many as keep their keys and values (at the
+// longest length the call allows) within 48 MB of the L2, at least one.
+static int attn_seq_chunk(int max_len, int Hkv, int dh, int B) {
+  const double kv = (double)max_len * Hkv * dh * 2 * 2;
+  const int s = kv > 0 ? (int)(48e6 / kv) : B;
+  return std::max(1, std::min(s, B));
+}
+
 template <int DH>
 cudaError_t launch_attn_fa(const void* qkv, void* out, const int* cu, int B, int max_len, int rows_cap, int Hq,
                            int Hkv, bool causal, float scale_log2, int* sched, int* err, cudaStream_t st) {
@@ -907,10 +925,12 @@ cudaError_t launch_attn_fa(const void* qkv, void* out, const int* cu, int B, int
       !encode_tmap_2d(&tkv, qkv, false, (uint64_t)rows_cap, (uint64_t)ld_qkv, 64, fa::BKV, nullptr))
     return cudaErrorInvalidValue;
   const int n_tiles = (max_len + fa::BQ - 1) / fa::BQ;
+  const int seq_chunk = attn_seq_chunk(max_len, Hkv, DH, B);
   const long n_items = (long)n_tiles * B * Hq;
   const int grid = (int)std::min<long>(n_items, (long)device_sm_count());
   return launch_pdl(fa::attn_fa_kernel<DH>, dim3(grid), dim3(fa::NTHR), C::SMEM, st, tq, tkv,
-                    reinterpret_cast<__nv_bfloat16*>(out), cu, B, Hq, Hkv, n_tiles, Hq * DH, causal ? 1 : 0,
+                    reinterpret_cast<__nv_bfloat16*>(out), cu, B, Hq, Hkv, n_tiles, seq_chunk, Hq * DH,
+                    causal ? 1 : 0,
                     scale_log2, sched, err);
 }
 
@@ -932,10 +952,12 @@ cudaError_t launch_attn_pair(const void* qkv, void* out, const int* cu, int B, i
       !encode_tmap_2d(&tkv, qkv, false, (uint64_t)rows_cap, (uint64_t)ld_qkv, 64, fa_pair::BKV, nullptr))
     return cudaErrorInvalidValue;
   const int n_tiles = (max_len + fa_pair::BQ - 1) / fa_pair::BQ;
+  const int seq_chunk = attn_seq_chunk(max_len, Hkv, DH, B);
   const long n_items = (long)n_tiles * B * ((Hq + 1) / 2);
   const int grid = (int)std::min<long>(n_items, (long)device_sm_count());
   return launch_pdl(fa_pair::attn_pair_kernel<DH>, dim3(grid), dim3(fa_pair::NTHR), C::SMEM, st, tq, tkv,
-                    reinterpret_cast<__nv_bfloat16*>(out), cu, B, Hq, Hkv, n_tiles, Hq * DH, causal ? 1 : 0,
+                    reinterpret_cast<__nv_bfloat16*>(out), cu, B, Hq, Hkv, n_tiles, seq_chunk, Hq * DH,
+                    causal ? 1 : 0,
                     scale_log2, err);
 }
 
