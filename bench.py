@@ -40,17 +40,33 @@ UNIT = "ms/batch"
 # (one 7B-dims layer at T = 1,792 rows, the benchmark's packed length within
 # 0.5%).  The figure belongs to the kernel sources with this digest; once they
 # change it is reported as null until a new capture replaces it.
-GEMM_TRAFFIC = {"bytes_per_launch": 163.7e6, "sources_sha256_16": "b9fa2d347c9187a4"}
+GEMM_TRAFFIC = {"bytes_per_launch": 165.9e6, "sources_sha256_16": "874a2a9205bb7f5b"}
 GEMM_SOURCES = ("paper_2609_13804_gb300/csrc/gemm_tc.cu", "paper_2609_13804_gb300/csrc/common.cuh")
 
 
-def gemm_traffic():
+# DRAM read + write bytes of one full-prefix attention launch (16 x 624 tokens,
+# 32 heads of 128, causal; the head-pair kernel) from the ncu capture summarised
+# in profiles/attn_pair_kernel_llava15-7b-dims_full_prefix.md, valid for the
+# kernel sources with this digest.
+ATTN_TRAFFIC = {"bytes_per_launch": 322.0e6, "sources_sha256_16": "3d5d1ecb3cd8060d"}
+ATTN_SOURCES = ("paper_2609_13804_gb300/csrc/attention.cu", "paper_2609_13804_gb300/csrc/common.cuh")
+
+
+def _digest(paths):
     import hashlib
     h = hashlib.sha256()
-    for rel in GEMM_SOURCES:
+    for rel in paths:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
-    return GEMM_TRAFFIC["bytes_per_launch"] if h.hexdigest()[:16] == GEMM_TRAFFIC["sources_sha256_16"] else None
+    return h.hexdigest()[:16]
+
+
+def gemm_traffic():
+    return GEMM_TRAFFIC["bytes_per_launch"] if _digest(GEMM_SOURCES) == GEMM_TRAFFIC["sources_sha256_16"] else None
+
+
+def attn_traffic():
+    return ATTN_TRAFFIC["bytes_per_launch"] if _digest(ATTN_SOURCES) == ATTN_TRAFFIC["sources_sha256_16"] else None
 
 
 PROBES_SRC = os.path.join(ROOT, "bench_probes.cu")
@@ -702,6 +718,7 @@ def run_ours(args):
             "compaction_128_images_hbm_frac": big_bytes / (big_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
             "compaction_note": ("16-image figures: one call after an L2 flush, events around it (launch latency "
                                 "included); 128 images: 402 MB moved per call, back to back"),
+            "roofline_attention": attention_roofline(attn_full_ms, attn_full_flops, m.n_layers, pk, workloads),
             "attention_full_prefix": {
                 "ms": attn_full_ms, "layers": m.n_layers, "sequences": w.B, "seq_len": full_lens[0],
                 "algorithmic_tflops": attn_full_flops / (attn_full_ms * 1e-3) / 1e12,
@@ -779,6 +796,27 @@ def device_model(B, m, dev, gen, torch, max_pos):
         head["proj_W1"] = (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
         head["proj_W2"] = (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)
     return B.Model(m, layers, head, dev, max_pos=max_pos)
+
+
+def attention_roofline(ms, flops, layers, pk, workloads):
+    """The attention kernels against the dense bf16 peak (burst: the launches
+    are timed one by one): the full prefix of the 16-image batch (16 x 624
+    tokens, the head-pair kernel) and, when the per-workload pass ran, the
+    InternVL3 full prefix (4 x 3,424 tokens, GQA 28/4, the two-stream kernel)."""
+    achieved = flops / (ms * 1e-3) / 1e12
+    out = {"kernel": "attn_pair_kernel (tcgen05; sequences up to 1,280 tokens)", "bound": "tensor",
+           "workload": "llava15-7b-b16 full prefix: 16 x 624 tokens, 32 heads of 128, causal",
+           "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s", "frac": achieved / pk["bf16"],
+           "peak_source": pk["source"] + " bf16 burst", "traffic": attn_traffic(),
+           "traffic_unit": "DRAM bytes per launch (one layer)", "launches": layers,
+           "algorithmic": "4 H d_h sum L(L+1)/2 flops per layer (causal)"}
+    w = (workloads or {}).get("internvl3-tiles-b4")
+    if isinstance(w, dict) and w.get("full_prefix"):
+        fp = w["full_prefix"]
+        out["long"] = {"kernel": "attn_fa_kernel (tcgen05, two softmax streams, dynamic scheduling)",
+                       "workload": "internvl3-tiles-b4 full prefix: 4 x 3,424 tokens, GQA 28/4, 28 layers",
+                       "achieved": fp.get("attention_tflops"), "frac": fp.get("attention_frac_of_bf16_burst")}
+    return out
 
 
 def attn_flops(m, lens, causal=True):
