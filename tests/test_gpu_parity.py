@@ -427,6 +427,23 @@ def test_prefill_empty_sequences(B):
     _prefill_case(B, w, [0, 5, 0, 130, 1, 0], 2)
 
 
+def test_prefill_long_with_empty_and_single_token_sequences(B):
+    # above 1,280 tokens the two-stream attention kernel runs: zero-length and
+    # one-token sequences share its item list with a long one (ragged last
+    # tile, GQA 4 / 2, head dim 64); two layers, so the second launch relies on
+    # the first leaving the work-ticket counter zero
+    w = S.tiny_workload(65, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=2)
+    _prefill_case(B, w, [0, 1300, 1, 0, 5], 2)
+
+
+@pytest.mark.parametrize("n", [1280, 1281])
+def test_prefill_at_the_attention_kernel_switch(B, n):
+    # the longest sequence the call allows picks the attention kernel: 1,280
+    # tokens the head-pair kernel, 1,281 the two-stream one (a one-row last tile)
+    w = S.tiny_workload(66, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=1)
+    _prefill_case(B, w, [n, 3], 1)
+
+
 def test_prefill_qwen_gqa_dims(B):
     w = S.qwen25vl_varres_b8()
     _prefill_case(B, w, [75, 300], 1)
