@@ -345,7 +345,9 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": value, "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "images": w.B, "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
+            "config": {"workload": w.name, "images": w.B, "global_images": wg.B,
+                       "sharding": "each rank its share of one global batch (replicas.shard_images); no collective",
+                       "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
                        "layers": w.model.n_layers},
             "extrapolated": True, "samples_timed": len(samples), "measured": measured,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle", "sample": sample,
@@ -377,7 +379,15 @@ def run_ours(args):
             dist.barrier()
         torch.cuda.synchronize()
 
-    w = S.llava15_7b_b16(seed=1002 + rank)
+    # the global batch holds `world` replicas' worth of images (weak scaling),
+    # drawn once from one seed; each rank takes its share of the images
+    # (longest-first greedy on the token counts: replicas.shard_images) and
+    # runs it on an identical copy of the weights
+    from paper_2609_13804_gb300.replicas import shard_images
+    w1 = S.llava15_7b_b16()
+    wg = dataclasses.replace(w1, n_vis=list(w1.n_vis) * world, n_txt=list(w1.n_txt) * world)
+    mine = shard_images(wg.n_vis, wg.n_txt, world, rank)
+    w = dataclasses.replace(w1, n_vis=[wg.n_vis[b] for b in mine], n_txt=[wg.n_txt[b] for b in mine])
     s, m = w.selector, w.model
     sel_w = S.make_selector_weights(w)
     selector = B.Selector(s, sel_w, dev)
@@ -388,7 +398,11 @@ def run_ours(args):
             "proj_W1": (torch.randn((m.proj_hidden, m.proj_in), device=dev, generator=gen) * 0.02).to(torch.bfloat16),
             "proj_W2": (torch.randn((m.d, m.proj_hidden), device=dev, generator=gen) * 0.02).to(torch.bfloat16)}
     model = B.Model(m, layers, head, dev, max_pos=4096)
-    inp = S.make_inputs(w)
+    inp_g = S.make_inputs(wg)
+    ov, ot = np.cumsum([0] + list(wg.n_vis)), np.cumsum([0] + list(wg.n_txt))
+    inp = {"X": np.concatenate([inp_g["X"][ov[b]:ov[b + 1]] for b in mine]),
+           "E_text": np.concatenate([inp_g["E_text"][ot[b]:ot[b + 1]] for b in mine])}
+    del inp_g
     X = B.dev_bf16(inp["X"], dev)
     E = B.dev_bf16(inp["E_text"], dev)
     n_ep = len(w.episodes())
@@ -694,7 +708,9 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": False, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": w.name, "images": w.B, "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
+            "config": {"workload": w.name, "images": w.B, "global_images": wg.B,
+                       "sharding": "each rank its share of one global batch (replicas.shard_images); no collective",
+                       "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
                        "layers": m.n_layers, "d": m.d, "selector_h": s.h, "k_max": w.k_max,
                        "mean_kept": float(counts.mean()), "packed_tokens": T,
                        "l2": "inputs larger than L2: 13.5 GB of weights streamed every step"},
