@@ -48,7 +48,7 @@ GEMM_SOURCES = ("paper_2609_13804_gb300/csrc/gemm_tc.cu", "paper_2609_13804_gb30
 # 32 heads of 128, causal; the head-pair kernel) from the ncu capture summarised
 # in profiles/attn_pair_kernel_llava15-7b-dims_full_prefix.md, valid for the
 # kernel sources with this digest.
-ATTN_TRAFFIC = {"bytes_per_launch": 322.0e6, "sources_sha256_16": "3d5d1ecb3cd8060d"}
+ATTN_TRAFFIC = {"bytes_per_launch": 322.0e6, "sources_sha256_16": "544923811917fe9d"}
 ATTN_SOURCES = ("paper_2609_13804_gb300/csrc/attention.cu", "paper_2609_13804_gb300/csrc/common.cuh")
 
 

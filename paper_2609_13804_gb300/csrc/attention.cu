@@ -16,13 +16,14 @@ constexpr int kPairMaxLen = 1280;
 
 // ===========================================================================
 // Short sequences (up to kPairMaxLen keys): persistent tcgen05 flash attention
-// over head pairs.  One CTA per SM walks a static list of work items; an item
+// over head pairs.  One CTA per SM walks a static list of work items (in chunks
+// of sequences whose keys and values fit in L2, longest tiles first); an item
 // is 128 query rows (one tile) of one sequence for a PAIR of query heads
-// (2p, 2p + 1).  Two items (the pair's heads) are in flight per CTA, which is
-// what keeps the tensor pipe busy when a tile has only one or two key blocks.  Each head of the pair has its own pipeline in
-// the CTA (its TMA thread, its MMA-issuing thread, its softmax warpgroup, its
-// TMEM columns); the two share the SM's tensor pipe, which interleaves them,
-// and the issue work of two threads.
+// (2p, 2p + 1).  Two tiles (the pair's heads) are in flight per CTA, which is
+// what keeps the tensor pipe busy when a tile has only one or two key blocks.
+// Each head of the pair has its own pipeline in the CTA (its TMA thread, its
+// two MMA-issuing threads, its softmax warpgroup, its TMEM columns); the two
+// share the SM's tensor pipe, which interleaves them.
 //
 //   warps 0 / 3  TMA of head 0 / 1: the Q tile once per item, then per 64-key
 //                block the K and V blocks into two-stage rings
@@ -406,11 +407,13 @@ attn_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 }  // namespace fa_pair
 
 // ===========================================================================
-// Longer sequences: persistent tcgen05 flash attention.  One CTA per SM takes work items from a
-// global ticket counter (or a static stride when no counter is given); an item
-// is 128 query rows (one tile) of one head of one sequence, and the item list
-// runs from the tiles with the most key blocks to those with the fewest, so
-// that the dynamic assignment balances the SMs.
+// Longer sequences: persistent tcgen05 flash attention.  One CTA per SM takes
+// work items from a global ticket counter (the last CTA out leaves it zero for
+// the next launch; without a counter, a static stride); an item is 128 query
+// rows (one tile) of one head of one sequence.  Within chunks of sequences whose
+// keys and values fit in L2, the item list runs from the tiles with the most
+// key blocks to those with the fewest, so that the dynamic assignment balances
+// the SMs.
 //
 //   warp 0      scheduler + TMA: takes the tickets, publishes each item to the
 //               other roles through a four-entry ring in shared memory, and loads
