@@ -345,9 +345,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": value, "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "images": w.B, "global_images": wg.B,
-                       "sharding": "each rank its share of one global batch (replicas.shard_images); no collective",
-                       "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
+            "config": {"workload": w.name, "images": w.B, "visual_tokens": w.n_vis[0], "text_tokens": w.n_txt[0],
                        "layers": w.model.n_layers},
             "extrapolated": True, "samples_timed": len(samples), "measured": measured,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle", "sample": sample,
