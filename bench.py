@@ -585,21 +585,32 @@ def run_ours(args):
     # ---- generation over the pruned prefix vs the full prefix (one token per
     #      sequence per step, 32 layers; the cache contents do not change the
     #      work, so a zeroed cache with the prefix lengths stands in)
-    def decode_ms(lens, steps=20, warm=3):
-        S_cap = max(lens) + warm + steps + 8
+    def decode_ms(lens, steps=20, warm=3, graph=False):
+        """ms per generation step: each step issued through sp_decode, or (graph)
+        one step captured in a CUDA graph and replayed (the step is
+        capture-safe: the lengths live and advance on the device)."""
+        S_cap = max(lens) + warm + 2 * steps + 8
         kv = B.kv_cache(model, w.B, S_cap)
         x_new = (torch.randn((w.B, m.d), device=dev, generator=gen) * 0.5).to(torch.bfloat16)
+        hid = torch.zeros((w.B, m.d), dtype=torch.float32, device=dev)
         lens_d = torch.tensor(lens, dtype=torch.int32, device=dev)
-        o = B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap)
+        o = B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, hidden=hid)
         ws_d = o["_ws"]
         for _ in range(warm - 1):
-            B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws_d)
+            B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws_d, hidden=hid)
+        step = lambda: B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws_d, hidden=hid)
+        if graph:
+            g = torch.cuda.CUDAGraph()
+            torch.cuda.synchronize()
+            with torch.cuda.graph(g):
+                step()
+            step = g.replay
         lens_d.copy_(torch.tensor(lens, dtype=torch.int32, device=dev))
         torch.cuda.synchronize()
         a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
         for _ in range(steps):
-            B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws_d)
+            step()
         b_.record()
         torch.cuda.synchronize()
         del kv
@@ -609,6 +620,11 @@ def run_ours(args):
     full_lens = [n + t for n, t in zip(w.n_vis, w.n_txt)]
     dec_pruned_ms = decode_ms(pruned_lens)
     dec_full_ms = decode_ms(full_lens)
+    try:
+        dec_graph_ms = decode_ms(pruned_lens, graph=True)
+    except Exception as ex:  # (a capture the runtime refuses: reported, not fatal)
+        print(f"decode graph capture: {ex}", file=sys.stderr)
+        dec_graph_ms = None
     qkv_w = (m.n_heads + 2 * m.n_kv_heads) * m.head_dim
     weight_bytes = 2.0 * m.n_layers * (m.d * qkv_w + m.n_heads * m.head_dim * m.d + 3 * m.d * m.ffn)
 
@@ -745,6 +761,9 @@ def run_ours(args):
             "token_ratio": (sum(w.n_vis) + sum(w.n_txt)) / T,
             "kept_counts": counts.tolist(),
             "decode": {"ms_per_step_pruned_prefix": dec_pruned_ms, "ms_per_step_full_prefix": dec_full_ms,
+                       "ms_per_step_pruned_prefix_cuda_graph": dec_graph_ms,
+                       "hbm_frac_pruned_cuda_graph": ((weight_bytes + cache_bytes(pruned_lens)) / (dec_graph_ms * 1e-3)
+                                                      / 1e9 / pk["hbm_gbs"]) if dec_graph_ms else None,
                        "speedup": dec_full_ms / dec_pruned_ms, "sequences": w.B,
                        "hbm_gbs_pruned": (weight_bytes + cache_bytes(pruned_lens)) / (dec_pruned_ms * 1e-3) / 1e9,
                        "hbm_frac_pruned": (weight_bytes + cache_bytes(pruned_lens)) / (dec_pruned_ms * 1e-3) / 1e9
