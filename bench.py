@@ -467,6 +467,21 @@ def run_ours(args):
     pk = peaks()
     achieved = flops / (gemm_ms * 1e-3) / 1e12
 
+    # ---- the per-step distribution: max(K, 20) more steps, an event pair around
+    #      each (async records, no synchronisation between steps)
+    n_dist = max(args.steps, 20)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_dist + 1)]
+    barrier()
+    evs[0].record(st)
+    for i in range(n_dist):
+        pipe(X, E, bias)
+        evs[i + 1].record(st)
+    torch.cuda.synchronize()
+    per_step = sorted(evs[i].elapsed_time(evs[i + 1]) for i in range(n_dist))
+    pct = lambda q: per_step[min(n_dist - 1, int(round(q * (n_dist - 1))))]
+    step_dist = {"steps": n_dist, "p10_ms": pct(0.1), "median_ms": pct(0.5), "p90_ms": pct(0.9),
+                 "min_ms": per_step[0], "max_ms": per_step[-1]}
+
     # ---- side measurements (outside the timed region)
     def timed(fn, reps=5):
         a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -739,6 +754,7 @@ def run_ours(args):
             "clocks": clk.summary(),
             "stages_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()},
             "ms_per_step_with_launch_events": ms_step_profiled,
+            "step_distribution": step_dist,
             "select_us_per_image": 1e3 * select_ms / w.B,
             "selection": sel_report,
             "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,
