@@ -323,11 +323,11 @@ def cores():
         return os.cpu_count()
 
 
-def run_reference(args):
+def run_reference(args, w=None):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    w = S.llava15_7b_b16()
+    w = w or S.llava15_7b_b16()
     samples, parts = [], []
     for i in range(args.warmup + args.steps):
         v, part = cpu_oracle_sample(w, b=i % w.B)
