@@ -399,30 +399,39 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     __syncthreads();
   };
   // rows [rank R / C, +R / C) of W [R, h] (fp32) times the shared vector x;
-  // half a warp per row, two rows per half-warp at a time; each result is
-  // pushed into dst[row] of every CTA
+  // half a warp per row, MR rows per half-warp at a time (their loads in
+  // flight together; each row's sum in the same order whatever MR is); each
+  // result is pushed into dst[row] of every CTA
+  constexpr int MR = 4;
   auto matvec_f32_push = [&](const float* W, int R, const float* x, float* dst) {
     const int Rc = R / C, r0 = rank * Rc, hl = lane & 15, hw = lane >> 4;
     const int cu = h / 4;  // float4 chunks per row
     const float4* x4 = reinterpret_cast<const float4*>(x);
-    for (int rb = (warp * 2 + hw) * 2; rb < Rc; rb += NW * 4) {
-      const float4* wa = reinterpret_cast<const float4*>(W + (size_t)(r0 + rb) * h);
-      const float4* wb = reinterpret_cast<const float4*>(W + (size_t)(r0 + min(rb + 1, Rc - 1)) * h);
-      float sv[2] = {0.f, 0.f};
+    for (int rb = (warp * 2 + hw) * MR; rb < Rc; rb += NW * 2 * MR) {
+      const float4* wr[MR];
+#pragma unroll
+      for (int i = 0; i < MR; ++i) wr[i] = reinterpret_cast<const float4*>(W + (size_t)(r0 + min(rb + i, Rc - 1)) * h);
+      float sv[MR];
+#pragma unroll
+      for (int i = 0; i < MR; ++i) sv[i] = 0.f;
 #pragma unroll 4
       for (int u = hl; u < cu; u += 16) {
         const float4 xv = x4[u];
-        sv[0] += dot4(xv, __ldg(wa + u));
-        sv[1] += dot4(xv, __ldg(wb + u));
+        float4 wv[MR];
+#pragma unroll
+        for (int i = 0; i < MR; ++i) wv[i] = __ldg(wr[i] + u);
+#pragma unroll
+        for (int i = 0; i < MR; ++i) sv[i] += dot4(xv, wv[i]);
       }
 #pragma unroll
       for (int o = 8; o > 0; o >>= 1) {
-        sv[0] += __shfl_xor_sync(0xffffffffu, sv[0], o);
-        sv[1] += __shfl_xor_sync(0xffffffffu, sv[1], o);
+#pragma unroll
+        for (int i = 0; i < MR; ++i) sv[i] += __shfl_xor_sync(0xffffffffu, sv[i], o);
       }
       if (hl < C) {
-        *cluster.map_shared_rank(dst + r0 + rb, hl) = sv[0];
-        if (rb + 1 < Rc) *cluster.map_shared_rank(dst + r0 + rb + 1, hl) = sv[1];
+#pragma unroll
+        for (int i = 0; i < MR; ++i)
+          if (rb + i < Rc) *cluster.map_shared_rank(dst + r0 + rb + i, hl) = sv[i];
       }
     }
   };
@@ -431,35 +440,43 @@ select_kernel(const BatchDesc bd, const SelectArgs a, int n_loc_max, int keys_in
     const int Rc = R / C, r0 = rank * Rc, hl = lane & 15, hw = lane >> 4;
     const int cu = K / 8;  // 8-element chunks per row
     const float4* x4 = reinterpret_cast<const float4*>(x);
-    for (int rb = (warp * 2 + hw) * 2; rb < Rc; rb += NW * 4) {
-      const uint4* wa = reinterpret_cast<const uint4*>(W + (size_t)(r0 + rb) * K);
-      const uint4* wb = reinterpret_cast<const uint4*>(W + (size_t)(r0 + min(rb + 1, Rc - 1)) * K);
-      float sv[2] = {0.f, 0.f};
+    for (int rb = (warp * 2 + hw) * MR; rb < Rc; rb += NW * 2 * MR) {
+      const uint4* wr[MR];
+#pragma unroll
+      for (int i = 0; i < MR; ++i) wr[i] = reinterpret_cast<const uint4*>(W + (size_t)(r0 + min(rb + i, Rc - 1)) * K);
+      float sv[MR];
+#pragma unroll
+      for (int i = 0; i < MR; ++i) sv[i] = 0.f;
 #pragma unroll 4
       for (int u = hl; u < cu; u += 16) {
         const float4 xa = x4[2 * u], xb = x4[2 * u + 1];
-        const uint4 pa = __ldg(wa + u), pb = __ldg(wb + u);
-        const uint32_t qa[4] = {pa.x, pa.y, pa.z, pa.w}, qb[4] = {pb.x, pb.y, pb.z, pb.w};
         const float xs[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+        uint4 pw[MR];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float2 fa = unpack_bf16x2(qa[k]), fb = unpack_bf16x2(qb[k]);
-          sv[0] += fa.x * xs[2 * k] + fa.y * xs[2 * k + 1];
-          sv[1] += fb.x * xs[2 * k] + fb.y * xs[2 * k + 1];
+        for (int i = 0; i < MR; ++i) pw[i] = __ldg(wr[i] + u);
+#pragma unroll
+        for (int i = 0; i < MR; ++i) {
+          const uint32_t q[4] = {pw[i].x, pw[i].y, pw[i].z, pw[i].w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float2 f = unpack_bf16x2(q[k]);
+            sv[i] += f.x * xs[2 * k] + f.y * xs[2 * k + 1];
+          }
         }
       }
 #pragma unroll
       for (int o = 8; o > 0; o >>= 1) {
-        sv[0] += __shfl_xor_sync(0xffffffffu, sv[0], o);
-        sv[1] += __shfl_xor_sync(0xffffffffu, sv[1], o);
+#pragma unroll
+        for (int i = 0; i < MR; ++i) sv[i] += __shfl_xor_sync(0xffffffffu, sv[i], o);
       }
       if (act) {
-        sv[0] = gelu_erf(sv[0]);
-        sv[1] = gelu_erf(sv[1]);
+#pragma unroll
+        for (int i = 0; i < MR; ++i) sv[i] = gelu_erf(sv[i]);
       }
       if (hl < C) {
-        *cluster.map_shared_rank(dst + r0 + rb, hl) = sv[0];
-        if (rb + 1 < Rc) *cluster.map_shared_rank(dst + r0 + rb + 1, hl) = sv[1];
+#pragma unroll
+        for (int i = 0; i < MR; ++i)
+          if (rb + i < Rc) *cluster.map_shared_rank(dst + r0 + rb + i, hl) = sv[i];
       }
     }
   };
