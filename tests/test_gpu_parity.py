@@ -638,6 +638,55 @@ def _decode_case(B, w, lens, n_layers, steps=2):
     model.close()
 
 
+def test_decode_steps_replay_in_a_cuda_graph(B):
+    """A generation step is capture-safe (lengths live and advance on the
+    device, no host synchronisation): the same steps issued one by one and
+    replayed from a captured CUDA graph give the same bits, hidden states and
+    cache alike (Llama-7B dims, one layer, weight-streaming GEMMs)."""
+    w = S.llava15_7b_b16()
+    m = w.model
+    L = S.make_layer_weights(w, 0, norm_affine=True)
+    head = S.make_model_head(w, norm_affine=True)
+    model = B.Model(m, [L], head, DEV, max_pos=512)
+    lens = [112, 240, 64, 17]
+    nb, steps = len(lens), 3
+    S_cap = max(lens) + steps + 8
+    x_new = B.dev_bf16(S.bf16_round(S.normal(w.seed, "decode_graph", (nb, m.d), 0.5)), DEV)
+    rng = np.random.default_rng(5)
+    init = (torch.from_numpy(rng.standard_normal((1, 2, nb, S_cap, m.n_kv_heads * m.head_dim)).astype(np.float32))
+            .to(torch.bfloat16).to(DEV))
+    runs = []
+    for graph in (False, True):
+        kv = init.clone()
+        lens_d = torch.tensor(lens, dtype=torch.int32, device=DEV)
+        hid = torch.zeros((nb, m.d), dtype=torch.float32, device=DEV)
+        ws = B.sp_decode(model, x=x_new, lens=torch.tensor(lens, dtype=torch.int32, device=DEV), kv=init.clone(),
+                         max_len_cap=S_cap, hidden=torch.zeros_like(hid))["_ws"]
+        torch.cuda.synchronize()
+        step = lambda: B.sp_decode(model, x=x_new, lens=lens_d, kv=kv, max_len_cap=S_cap, ws=ws, hidden=hid)
+        outs = []
+        if graph:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                step()
+            lens_d.copy_(torch.tensor(lens, dtype=torch.int32, device=DEV))  # (capture does not run the step)
+            for _ in range(steps):
+                g.replay()
+                outs.append(hid.clone())
+        else:
+            for _ in range(steps):
+                step()
+                outs.append(hid.clone())
+        torch.cuda.synchronize()
+        runs.append(([o.cpu() for o in outs], kv.cpu(), lens_d.cpu()))
+    (h0, kv0, l0), (h1, kv1, l1) = runs
+    assert torch.equal(l0, l1) and l0.tolist() == [n + steps for n in lens]
+    for a, b in zip(h0, h1):
+        assert torch.equal(a, b)
+    assert torch.equal(kv0, kv1)
+    model.close()
+
+
 def test_decode_tiny_gqa_ragged(B):
     w = S.tiny_workload(62, [1], [1], D=128, d=128, n_heads=4, n_kv_heads=2, head_dim=64, ffn=256, n_layers=2)
     _decode_case(B, w, [5, 130, 1, 64], 2)
