@@ -482,6 +482,26 @@ def run_ours(args):
     step_dist = {"steps": n_dist, "p10_ms": pct(0.1), "median_ms": pct(0.5), "p90_ms": pct(0.9),
                  "min_ms": per_step[0], "max_ms": per_step[-1]}
 
+    # ---- the same step captured once in a CUDA graph and replayed K times
+    #      (the call is capture-safe); reported beside the value
+    graph_ms = None
+    try:
+        gph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gph):
+            pipe(X, E, bias)
+        gph.replay()
+        barrier()
+        ev4, ev5 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev4.record(st)
+        for _ in range(args.steps):
+            gph.replay()
+        ev5.record(st)
+        barrier()
+        graph_ms = max_over_ranks(ev4.elapsed_time(ev5) / args.steps, dev)
+        del gph
+    except Exception as ex:  # (a capture the runtime refuses: reported, not fatal)
+        print(f"pipeline graph capture: {ex}", file=sys.stderr)
+
     # ---- side measurements (outside the timed region)
     def timed(fn, reps=5):
         a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -755,6 +775,7 @@ def run_ours(args):
             "stages_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()},
             "ms_per_step_with_launch_events": ms_step_profiled,
             "step_distribution": step_dist,
+            "ms_per_step_cuda_graph": graph_ms,
             "select_us_per_image": 1e3 * select_ms / w.B,
             "selection": sel_report,
             "compaction_gbs": comp_bytes / (compact_ms * 1e-3) / 1e9,

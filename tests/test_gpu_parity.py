@@ -495,6 +495,20 @@ def test_pipeline_end_to_end_without_encoder(B):
     np.testing.assert_array_equal(oi.numpy(), np_(pipe.idx))
     np.testing.assert_array_equal(ocu.numpy(), cu)
     np.testing.assert_array_equal(oh.numpy()[:T], np_(pipe.hidden)[:T])
+    # the call is capture-safe (no host synchronisation, sizes from caps): a
+    # CUDA graph of it replays to the same bytes
+    ref_idx, ref_h = pipe.idx.clone(), pipe.hidden.clone()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        pipe(Xd, Ed, bd)
+    pipe.idx.fill_(-7)
+    pipe.hidden.zero_()
+    pipe.cu.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(pipe.idx, ref_idx)
+    np.testing.assert_array_equal(np_(pipe.cu), cu)
+    assert torch.equal(pipe.hidden[:T], ref_h[:T])
     selector.close()
     model.close()
 
