@@ -513,6 +513,92 @@ def test_pipeline_end_to_end_without_encoder(B):
     model.close()
 
 
+def test_pipeline_groups_g5_without_encoder(B):
+    """sp_pipeline with candidate groups of 64 and five tokens per round (the
+    AnyRes / Qwen / InternVL form), selection straight on the visual tokens so
+    that it is exact end to end: indices, offsets and hidden states against the
+    oracle's whole path."""
+    w = S.tiny_workload(73, [200, 64, 130], [9, 3, 5], D=128, D_text=256, h=128, d=256, n_heads=4,
+                        n_kv_heads=2, head_dim=64, ffn=256, n_layers=2, k_max=20, proj_kind="mlp2",
+                        group_size=64, g=5)
+    w.model.proj_hidden = 256
+    s = w.selector
+    sel = S.make_selector_weights(w, ln_affine=True)
+    PT.scale_decoder(sel, 4.0)
+    sel["enc"] = []
+    inp = S.make_inputs(w)
+    X, E = inp["X"], inp["E_text"]
+    # episodes: 64, 64, 64, 8 | 64 | 64, 64, 2 candidates
+    biases = PT.calibrate_biases(X, w.n_vis, sel, k_max=w.k_max, g=w.g, group_size=w.group_size,
+                                 targets=[10, 20, 5, 8, 15, 20, 10, 2])
+    layers = [S.make_layer_weights(w, l, norm_affine=True) for l in range(2)]
+    head = S.make_model_head(w, norm_affine=True)
+    shape = S.SelectorShape(D=s.D, D_text=s.D_text, h=s.h, n_enc_layers=0)
+    selector = B.Selector(shape, sel, DEV)
+    model = B.Model(w.model, layers, head, DEV, max_pos=512)
+    pipe = B.Pipeline(selector, model, w.n_vis, w.n_txt, group_size=w.group_size, g=w.g, k_max=w.k_max)
+    pipe(B.dev_bf16(X, DEV), B.dev_bf16(E, DEV), B.dev_f32(biases, DEV))
+    torch.cuda.synchronize()
+    assert int(pipe.err.item()) == 0
+    ref = O.run_pipeline(X, E, w.n_vis, w.n_txt, sel, shape, head, layers, w.model, k_max=w.k_max, g=w.g,
+                         group_size=w.group_size, stop_bias=biases, store="bf16")
+    counts = np_(pipe.count)
+    for b in range(w.B):
+        assert list(np_(pipe.idx)[b][:counts[b]]) == list(ref["idx"][b])
+    cu = np_(pipe.cu)
+    np.testing.assert_array_equal(cu, ref["cu_seqlens"])
+    T = int(cu[-1])
+    r = PT.hidden_close(np_(pipe.hidden)[:T], ref["hidden"], "grouped pipeline")
+    print("grouped g=5 pipeline: kept", counts.tolist(), "max-abs %.3e mean-rel %.3e" % r)
+    selector.close()
+    model.close()
+
+
+def test_pipeline_with_encoder_equals_its_stages(B):
+    """The chained call with the 2-block encoder, candidate groups and g = 5
+    gives the bytes of its stages called one by one through the C ABI
+    (sp_select -> sp_compact (index mode) -> sp_project -> sp_prefill), each
+    of which is compared with the oracle on its own."""
+    w = S.tiny_workload(74, [200, 64, 130], [9, 3, 5], D=128, D_text=256, h=128, d=256, n_heads=4,
+                        n_kv_heads=2, head_dim=64, ffn=256, n_layers=2, k_max=20, proj_kind="mlp2",
+                        group_size=64, g=5, enc_head_dim=64)
+    w.model.proj_hidden = 256
+    sel = S.make_selector_weights(w, ln_affine=True)
+    inp = S.make_inputs(w)
+    layers = [S.make_layer_weights(w, l, norm_affine=True) for l in range(2)]
+    head = S.make_model_head(w, norm_affine=True)
+    selector = B.Selector(w.selector, sel, DEV)
+    model = B.Model(w.model, layers, head, DEV, max_pos=512)
+    Xd, Ed = B.dev_bf16(inp["X"], DEV), B.dev_bf16(inp["E_text"], DEV)
+    n_ep = len(w.episodes())
+    # a STOP bias far below / above the logits keeps each group to k_max / stops it at once
+    assert n_ep == 8  # 64, 64, 64, 8 | 64 | 64, 64, 2 candidates
+    bd = B.dev_f32(np.array([-1.5, 1.5, -1.5, 1.5, -1.5, 1.5, -1.5, -1.5], np.float32), DEV)
+    pipe = B.Pipeline(selector, model, w.n_vis, w.n_txt, group_size=w.group_size, g=w.g, k_max=w.k_max)
+    pipe(Xd, Ed, bd)
+    r = B.sp_select(selector, w.n_vis, w.n_txt, X=Xd, E_text=Ed, stop_bias=bd, group_size=w.group_size, g=w.g,
+                    k_max=w.k_max, k_cap=pipe.k_cap, traces=False)
+    c = B.sp_compact(w.n_vis, w.n_txt, X=Xd, text=Ed, idx=r["idx"], count=r["count"], k_cap=pipe.k_cap,
+                     index_mode=True)
+    B.sp_project(model, vis_row_map=c["vis_row_map"], vis_cu=c["vis_cu"], packed=c["packed"],
+                 rows_cap=c["rows_cap"], B=w.B, X=Xd, vis_src=c["vis_src"])
+    max_len = max(min(n, pipe.k_cap) + t for n, t in zip(w.n_vis, w.n_txt))
+    p = B.sp_prefill(model, x=c["packed"], cu_seqlens=c["cu_seqlens"], pos=c["pos"], B=w.B, T_cap=c["T_cap"],
+                     max_seqlen_cap=max_len)
+    torch.cuda.synchronize()
+    assert int(pipe.err.item()) == 0 and int(c["err"].item()) == 0 and int(p["err"].item()) == 0
+    counts = np_(pipe.count)
+    assert counts.tolist() == np_(r["count"]).tolist() and 0 < counts.sum() < sum(w.n_vis)
+    np.testing.assert_array_equal(np_(pipe.idx), np_(r["idx"]))
+    cu = np_(pipe.cu)
+    np.testing.assert_array_equal(cu, np_(c["cu_seqlens"]))
+    T = int(cu[-1])
+    np.testing.assert_array_equal(np_(pipe.hidden)[:T], np_(p["hidden"])[:T])
+    print("pipeline with encoder: kept", counts.tolist(), "of", w.n_vis)
+    selector.close()
+    model.close()
+
+
 def test_prefill_llava15_b16_32layers_sampled(B):
     """The benchmark's prefill launch: 32 Llama-7B-dims layers over 16 packed
     sequences (kept counts 16..192 + 48 text tokens).
