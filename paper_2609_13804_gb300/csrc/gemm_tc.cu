@@ -22,6 +22,7 @@
 #include <algorithm>
 #include <cstdlib>
 #include <cstring>
+#include <type_traits>
 
 #include "common.cuh"
 #include "internal.h"
@@ -1211,22 +1212,63 @@ __global__ void __launch_bounds__(256) splitk_reduce_t_kernel(const float* __res
   if (c >= cols || m0 >= M) return;
   const int mn = min(8, M - m0);
   const size_t plane = (size_t)N_acc * 32;
-  auto sum8 = [&](int n, float (&v)[8]) {
+  // Sums 8 rows of NC columns over the ks ranges, in range order.  The loads
+  // of four ranges (for every column) go out before their adds, so a thread
+  // waits on L2 about ks / 4 times instead of ks * NC times.
+  auto sum_cols = [&](auto nc_tag, const int* n, float (*v)[8]) {
+    constexpr int NC = decltype(nc_tag)::value;
+    const float* p[NC];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) v[i] = 0.f;
-    const float* p = part + (size_t)n * 32 + m0;
-    for (int s = 0; s < ks; ++s) {
-      const float4 a = __ldcg(reinterpret_cast<const float4*>(p + s * plane));
-      const float4 b = __ldcg(reinterpret_cast<const float4*>(p + s * plane) + 1);
-      v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
-      v[4] += b.x; v[5] += b.y; v[6] += b.z; v[7] += b.w;
+    for (int k = 0; k < NC; ++k) {
+      p[k] = part + (size_t)n[k] * 32 + m0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[k][i] = 0.f;
+    }
+    int s = 0;
+    for (; s + 4 <= ks; s += 4) {
+      float4 a[4][NC][2];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+#pragma unroll
+        for (int k = 0; k < NC; ++k) {
+          a[j][k][0] = __ldcg(reinterpret_cast<const float4*>(p[k] + (s + j) * plane));
+          a[j][k][1] = __ldcg(reinterpret_cast<const float4*>(p[k] + (s + j) * plane) + 1);
+        }
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+#pragma unroll
+        for (int k = 0; k < NC; ++k) {
+          v[k][0] += a[j][k][0].x; v[k][1] += a[j][k][0].y; v[k][2] += a[j][k][0].z; v[k][3] += a[j][k][0].w;
+          v[k][4] += a[j][k][1].x; v[k][5] += a[j][k][1].y; v[k][6] += a[j][k][1].z; v[k][7] += a[j][k][1].w;
+        }
+    }
+    for (; s < ks; ++s)
+#pragma unroll
+      for (int k = 0; k < NC; ++k) {
+        const float4 a0 = __ldcg(reinterpret_cast<const float4*>(p[k] + s * plane));
+        const float4 a1 = __ldcg(reinterpret_cast<const float4*>(p[k] + s * plane) + 1);
+        v[k][0] += a0.x; v[k][1] += a0.y; v[k][2] += a0.z; v[k][3] += a0.w;
+        v[k][4] += a1.x; v[k][5] += a1.y; v[k][6] += a1.z; v[k][7] += a1.w;
+      }
+  };
+  auto sum8 = [&](int n, float (&v)[8]) {
+    const int nn[1] = {n};
+    sum_cols(std::integral_constant<int, 1>{}, nn, &v);
+  };
+  auto sum8x2 = [&](int n0, int n1, float (&v)[8], float (&u)[8]) {
+    const int nn[2] = {n0, n1};
+    float vu[2][8];
+    sum_cols(std::integral_constant<int, 2>{}, nn, vu);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      v[i] = vu[0][i];
+      u[i] = vu[1][i];
     }
   };
   float v[8];
   if (e.kind == EPI_SWIGLU_BF16) {
     float u[8];
-    sum8(c, v);
-    sum8(e.up_off + c, u);
+    sum8x2(c, e.up_off + c, v, u);
     __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(e.out) + c;
     #pragma unroll
     for (int i = 0; i < 8; ++i)
@@ -1240,8 +1282,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_t_kernel(const float* __res
     if (hb < e.rope_cols) {
       if (i0 >= half) return;  // the pair's first element writes both
       float u[8];
-      sum8(c, v);
-      sum8(c + half, u);
+      sum8x2(c, c + half, v, u);
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         if (i >= mn) break;

@@ -121,3 +121,59 @@ def test_encoder_memory_qwen_dims(B):
           f"max-abs / rms {rel64:.3e} mean-rel {mrel64:.3e}")
     assert rel <= PT.HID_MAX_ABS, rel
     assert mrel64 <= PT.HID_MEAN_REL, mrel64
+
+
+def test_pipeline_equals_its_stages_qwen_dims(B):
+    """The chained call at the Qwen2.5-VL-7B dims (8 images of 256..4,096
+    tokens; the 3,584-wide two-block encoder, whose 56 heads of 64 over up to
+    4,160 rows take the streamed attention kernel; groups of 1,024 with g = 5;
+    GQA 28/4; no projector), one decoder layer: the same bytes as its stages
+    called one by one (sp_select -> sp_compact -> sp_prefill).  Weights and
+    inputs are drawn on the device (both sides read the same bytes); STOP biases
+    keep about 11% of every group."""
+    import dataclasses
+    import os
+    import sys
+    sys.path.insert(0, os.path.abspath(os.path.join(os.path.dirname(__file__), "..")))
+    import bench
+    w = S.qwen25vl_varres_b8()
+    w = dataclasses.replace(w, model=dataclasses.replace(w.model, n_layers=1))
+    s = w.selector
+    gen = torch.Generator(device=DEV)
+    gen.manual_seed(2604)
+    sel = B.Selector(s, bench.device_selector_weights(s, DEV, gen, torch), DEV)
+    model = bench.device_model(B, w.model, DEV, gen, torch, max_pos=4096 + 256)
+    X = torch.randn((sum(w.n_vis), s.D), device=DEV, generator=gen).to(torch.bfloat16)
+    E = (torch.randn((sum(w.n_txt), s.D_text), device=DEV, generator=gen) * 0.02).to(torch.bfloat16)
+    eps = w.episodes()
+    cal = B.sp_select(sel, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=B.dev_f32(np.full(len(eps), -1e30), DEV),
+                      group_size=w.group_size, g=w.g, k_max=w.k_max)
+    torch.cuda.synchronize()
+    gaps, rounds = np_(cal["gap"]), np_(cal["rounds"])
+    targets, _ = bench.episode_targets(w)
+    biases, _ = S.stop_biases([gaps[e, :rounds[e]] for e in range(len(eps))], targets, g=w.g, k_max=w.k_max,
+                              n_cand=[n for (_, _, n) in eps])
+    bd = B.dev_f32(biases, DEV)
+    pipe = B.Pipeline(sel, model, w.n_vis, w.n_txt, group_size=w.group_size, g=w.g, k_max=w.k_max)
+    pipe(X, E, bd)
+    r = B.sp_select(sel, w.n_vis, w.n_txt, X=X, E_text=E, stop_bias=bd, group_size=w.group_size, g=w.g,
+                    k_max=w.k_max, k_cap=pipe.k_cap, traces=False)
+    c = B.sp_compact(w.n_vis, w.n_txt, X=X, text=E, idx=r["idx"], count=r["count"], k_cap=pipe.k_cap)
+    max_len = max(min(n, pipe.k_cap) + t for n, t in zip(w.n_vis, w.n_txt))
+    p = B.sp_prefill(model, x=c["packed"], cu_seqlens=c["cu_seqlens"], pos=c["pos"], B=w.B, T_cap=c["T_cap"],
+                     max_seqlen_cap=max_len)
+    torch.cuda.synchronize()
+    assert int(pipe.err.item()) == 0 and int(c["err"].item()) == 0 and int(p["err"].item()) == 0
+    counts = np_(pipe.count)
+    assert counts.tolist() == np_(r["count"]).tolist()
+    assert 0.05 * sum(w.n_vis) < counts.sum() < 0.2 * sum(w.n_vis)
+    np.testing.assert_array_equal(np_(pipe.idx), np_(r["idx"]))
+    cu = np_(pipe.cu)
+    np.testing.assert_array_equal(cu, np_(c["cu_seqlens"]))
+    T = int(cu[-1])
+    h = np_(pipe.hidden)[:T]
+    assert np.isfinite(h).all()
+    np.testing.assert_array_equal(h, np_(p["hidden"])[:T])
+    print("qwen-dims pipeline: kept", counts.tolist(), "of", w.n_vis)
+    sel.close()
+    model.close()
